@@ -1,0 +1,240 @@
+"""CPU oracle of the M+Adam optimizer step (arxiv 2607.10611) -- ctypes wrapper.
+
+TEST INFRASTRUCTURE ONLY.  The oracle is a plain, single-threaded C
+implementation (mpadam_oracle.c) of Algorithm 1 with the options of
+Algorithm 2 (Appendix A), in IEEE binary32 as the paper's FP32-compute /
+low-precision-storage round trip prescribes (Appendix B).  Only the tests, the
+smoke check and the benchmark's CPU-baseline leg may import this package; the
+CUDA library never does, and this package imports nothing from it.
+
+Arrays are numpy: float32 for FP32, uint16 bit patterns for BF16, uint8 codes
+for E4M3.  Functions update their arguments in place where stated.
+"""
+from __future__ import annotations
+
+import ctypes
+import math
+from typing import List, Optional, Sequence
+
+import numpy as np
+
+from . import build as _build
+
+F32, BF16, E4M3 = 0, 1, 2
+DTYPES = {"f32": F32, "bf16": BF16, "e4m3": E4M3}
+ALIGN = 8
+
+_LIB = None
+
+
+class HParams(ctypes.Structure):
+    _fields_ = [
+        ("lr_add", ctypes.c_float), ("lr_mul", ctypes.c_float),
+        ("beta1", ctypes.c_float), ("beta2", ctypes.c_float),
+        ("eps", ctypes.c_float), ("tau", ctypes.c_float),
+        ("rmax_pos", ctypes.c_float), ("rmax_neg", ctypes.c_float),
+        ("g_max", ctypes.c_float), ("dmult_max", ctypes.c_float),
+        ("w_max", ctypes.c_float), ("wd_add", ctypes.c_float),
+        ("bias_correction", ctypes.c_int32), ("stochastic", ctypes.c_int32),
+        ("seed", ctypes.c_uint64),
+    ]
+
+
+class Scalars(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_float) for n in
+                ("b1", "b2", "omb1", "omb2", "ka", "c2", "km", "ln2", "eps", "tau",
+                 "lo", "hi", "gmax", "wmax", "kwd")] + \
+               [("gmax_on", ctypes.c_int32), ("wmax_on", ctypes.c_int32), ("wd_on", ctypes.c_int32)]
+
+
+DEFAULTS = dict(lr_add=1e-3, lr_mul=1e-3, beta1=0.9, beta2=0.999, eps=1e-8, tau=1e-8,
+                rmax_pos=0.75, rmax_neg=0.75, g_max=math.inf, dmult_max=math.inf,
+                w_max=math.inf, wd_add=0.0, bias_correction=1, stochastic=0, seed=0)
+
+
+def hparams(**kw) -> HParams:
+    d = dict(DEFAULTS)
+    for k, val in kw.items():
+        if k not in d:
+            raise KeyError(k)
+        d[k] = val
+    return HParams(**d)
+
+
+def lib() -> ctypes.CDLL:
+    global _LIB
+    if _LIB is None:
+        path = _build.build()
+        L = ctypes.CDLL(str(path))
+        P, i64, i32, u64 = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32, ctypes.c_uint64
+        L.orc_philox4x32_10.argtypes = [P, P, P]
+        L.orc_rng_lane.argtypes = [u64, u64, u64, i32]
+        L.orc_rng_lane.restype = ctypes.c_uint32
+        L.orc_bf16_rne.argtypes = [ctypes.c_float]; L.orc_bf16_rne.restype = ctypes.c_uint16
+        L.orc_bf16_sr.argtypes = [ctypes.c_float, ctypes.c_uint32]; L.orc_bf16_sr.restype = ctypes.c_uint16
+        L.orc_e4m3_rne.argtypes = [ctypes.c_float]; L.orc_e4m3_rne.restype = ctypes.c_uint8
+        L.orc_e4m3_sr.argtypes = [ctypes.c_float, ctypes.c_uint32]; L.orc_e4m3_sr.restype = ctypes.c_uint8
+        L.orc_e4m3_decode.argtypes = [ctypes.c_uint8]; L.orc_e4m3_decode.restype = ctypes.c_float
+        L.orc_fp8_next_exponent.argtypes = [ctypes.c_float, i32]; L.orc_fp8_next_exponent.restype = i32
+        L.orc_scalars_for_step.argtypes = [P, i64, P]; L.orc_scalars_for_step.restype = i32
+        L.orc_step_elements.argtypes = [i64, P, i64, i32, i32, i32, P, P, P, P, P, P, i64, i32, i32, P]
+        L.orc_step_elements.restype = i32
+        L.orc_e4m3_amax.argtypes = [i64, P, i32]; L.orc_e4m3_amax.restype = ctypes.c_float
+        L.orc_bf16_rne_n.argtypes = [i64, P, P]
+        L.orc_bf16_sr_n.argtypes = [i64, P, P, P]
+        L.orc_e4m3_rne_n.argtypes = [i64, P, P]
+        L.orc_e4m3_sr_n.argtypes = [i64, P, P, P]
+        L.orc_e4m3_decode_n.argtypes = [i64, P, P]
+        L.orc_rng_lanes_n.argtypes = [u64, u64, i32, i64, P, P]
+        L.orc_philox_n.argtypes = [i64, P, P, P]
+        L.orc_update_elements_n.argtypes = [P, i64, i64, P, P, P, P, P, P, P, P, P]
+        L.orc_update_elements_n.restype = i32
+        _LIB = L
+    return _LIB
+
+
+def _p(a: np.ndarray):
+    return ctypes.c_void_p(a.ctypes.data)
+
+
+def _c(a, dtype):
+    return np.ascontiguousarray(a, dtype=dtype)
+
+
+# --------------------------------------------------------------------------
+# Random bits
+# --------------------------------------------------------------------------
+def philox4x32_10(ctr: Sequence[int], key: Sequence[int]) -> np.ndarray:
+    c = _c(ctr, np.uint32).reshape(-1)
+    k = _c(key, np.uint32)
+    out = np.zeros(c.size, np.uint32)
+    lib().orc_philox_n(c.size // 4, _p(c), _p(k), _p(out))
+    return out
+
+
+def rng_lanes(seed: int, t: int, idx, storage: int) -> np.ndarray:
+    """Random bits the step draws for global element indices `idx` at step t:
+    16-bit lanes for BF16 storage, 32-bit lanes for E4M3 storage."""
+    i = _c(idx, np.uint64)
+    out = np.zeros(i.size, np.uint32)
+    lib().orc_rng_lanes_n(seed, t, storage, i.size, _p(i), _p(out))
+    return out
+
+
+# --------------------------------------------------------------------------
+# Storage formats
+# --------------------------------------------------------------------------
+def bf16_rne(x) -> np.ndarray:
+    x = _c(x, np.float32); out = np.zeros(x.size, np.uint16)
+    lib().orc_bf16_rne_n(x.size, _p(x), _p(out)); return out
+
+
+def bf16_sr(x, r16) -> np.ndarray:
+    x = _c(x, np.float32); r = _c(r16, np.uint32); out = np.zeros(x.size, np.uint16)
+    lib().orc_bf16_sr_n(x.size, _p(x), _p(r), _p(out)); return out
+
+
+def bf16_decode(h) -> np.ndarray:
+    return (_c(h, np.uint16).astype(np.uint32) << 16).view(np.float32)
+
+
+def e4m3_rne(x) -> np.ndarray:
+    x = _c(x, np.float32); out = np.zeros(x.size, np.uint8)
+    lib().orc_e4m3_rne_n(x.size, _p(x), _p(out)); return out
+
+
+def e4m3_sr(x, r32) -> np.ndarray:
+    x = _c(x, np.float32); r = _c(r32, np.uint32); out = np.zeros(x.size, np.uint8)
+    lib().orc_e4m3_sr_n(x.size, _p(x), _p(r), _p(out)); return out
+
+
+def e4m3_decode(q) -> np.ndarray:
+    q = _c(q, np.uint8); out = np.zeros(q.size, np.float32)
+    lib().orc_e4m3_decode_n(q.size, _p(q), _p(out)); return out
+
+
+def fp8_next_exponent(amax: float, e_cur: int) -> int:
+    return int(lib().orc_fp8_next_exponent(ctypes.c_float(amax), int(e_cur)))
+
+
+def e4m3_amax(q, e: int) -> float:
+    q = _c(q, np.uint8)
+    return float(lib().orc_e4m3_amax(q.size, _p(q), int(e)))
+
+
+# --------------------------------------------------------------------------
+# The update
+# --------------------------------------------------------------------------
+def scalars(hp: HParams, t: int) -> Scalars:
+    s = Scalars()
+    if lib().orc_scalars_for_step(ctypes.byref(hp), t, ctypes.byref(s)) != 0:
+        raise ValueError("invalid hyper-parameters or step")
+    return s
+
+
+def update_elements(hp: HParams, t: int, w, g, m, v, ve):
+    """The binary32 update without storage rounding: returns (wn, m1, v1, ve1)."""
+    arrs = [_c(a, np.float32) for a in (w, g, m, v, ve)]
+    n = arrs[0].size
+    outs = [np.zeros(n, np.float32) for _ in range(4)]
+    rc = lib().orc_update_elements_n(ctypes.byref(hp), t, n, *map(_p, arrs), *map(_p, outs))
+    if rc != 0:
+        raise ValueError("invalid hyper-parameters or step")
+    return tuple(outs)
+
+
+def step_elements(hp: HParams, t: int, wdt: int, gdt: int, mdt: int, w, g, m, v, ve,
+                  gidx=None, gidx0: int = 0, e_cur: int = 0, e_next: int = 0) -> float:
+    """One step over host arrays updated in place; returns max |updated w|
+    (finite values; meaningful for E4M3 storage)."""
+    for a in (w, g, m, v, ve):
+        assert a.flags.c_contiguous
+    n = w.size
+    idx = None if gidx is None else _c(gidx, np.int64)
+    amax = ctypes.c_float(0.0)
+    rc = lib().orc_step_elements(
+        n, None if idx is None else _p(idx), gidx0, wdt, gdt, mdt,
+        _p(w), _p(g), _p(m), _p(v), _p(ve), ctypes.byref(hp), t, e_cur, e_next,
+        ctypes.byref(amax))
+    if rc != 0:
+        raise ValueError("invalid arguments")
+    return float(amax.value)
+
+
+def global_offsets(numels) -> List[int]:
+    """First global element index of each tensor: the previous tensor's end
+    rounded up to a multiple of 8."""
+    offs, o = [], 0
+    for n in numels:
+        offs.append(o)
+        o = -(-(o + int(n)) // ALIGN) * ALIGN
+    return offs
+
+
+def fp8_init(tensors, exps: Sequence[int]) -> List[list]:
+    """Per-tensor FP8 state [exponent, amax] before the first step: amax is the
+    largest |decoded stored weight|."""
+    return [[int(e), e4m3_amax(t["w"], int(e))] for t, e in zip(tensors, exps)]
+
+
+def step(tensors, *, wdt: int, gdt: int, mdt: int, hp: HParams, t: int,
+         fp8_state: Optional[List[list]] = None) -> None:
+    """One optimizer step over a tensor list.  tensors: list of dicts of 1-D
+    numpy arrays w, g, m, v, ve (updated in place).  For E4M3 storage,
+    fp8_state[k] = [exponent the stored weights use, largest |w| before this
+    step]; it is advanced in place: the weights are re-encoded with the
+    exponent chosen from that largest |w|, and the new largest |w| is recorded."""
+    offs = global_offsets([d["w"].size for d in tensors])
+    for k, d in enumerate(tensors):
+        if d["w"].size == 0:
+            continue
+        if wdt == E4M3:
+            e_cur, a_cur = fp8_state[k]
+            e_next = fp8_next_exponent(a_cur, e_cur)
+            a_next = step_elements(hp, t, wdt, gdt, mdt, d["w"], d["g"], d["m"], d["v"], d["ve"],
+                                   gidx0=offs[k], e_cur=e_cur, e_next=e_next)
+            fp8_state[k][0] = e_next
+            fp8_state[k][1] = a_next
+        else:
+            step_elements(hp, t, wdt, gdt, mdt, d["w"], d["g"], d["m"], d["v"], d["ve"],
+                          gidx0=offs[k])

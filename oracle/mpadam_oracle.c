@@ -1,0 +1,396 @@
+/*
+ * mpadam_oracle.c -- plain, slow, single-threaded CPU oracle of the M+Adam
+ * optimizer step (arxiv 2607.10611).
+ *
+ * TEST INFRASTRUCTURE ONLY: it exists to check the CUDA library, and only the
+ * tests, the smoke check and the benchmark's CPU-baseline leg may call it.
+ * It shares no code with the CUDA path.
+ *
+ * What it follows:
+ *   - Algorithm 1 (Sec. 4.1, "M+Adam: additive-multiplicative update"):
+ *     Adam moments with bias correction, the exponent gradient
+ *     g_e = (ln 2) w g, its second moment, the proposal
+ *     u~ = -eta_m g_e / (sqrt(v_e-hat) + eps), rho = max(|w|, tau),
+ *     u_m = u~ / rho and the combination w + w u_m + u_a.
+ *   - Sec. 4.1: u_m = clip(u~ / rho).
+ *   - Algorithm 2 (Appendix A): the optional clamp of the normalised exponent
+ *     gradient at g_max, the relative bounds [-(0.75 - eps0), 0.75], the
+ *     optional cap |log2(1 + u_m)| <= d_mult,max, the optional weight clip
+ *     w_max and the optional additive (decoupled) weight decay; bias
+ *     correction switched off reproduces Algorithm 2's raw moments.
+ *   - Eq. for AdamW in Sec. 3: the decoupled decay term eta * lambda * w.
+ *   - Appendix B, "bf16 round trip": each step is computed in FP32 and the
+ *     parameter is rounded into its storage format right away.
+ *
+ * Readings where the paper leaves the arithmetic open (each also listed in
+ * the design notes of the repository):
+ *   - bias correction is folded into two per-step scalars: eta_a u-hat =
+ *     eta_a mu / (1 - beta1^t) and sqrt(v-hat) = sqrt(v) / sqrt(1 - beta2^t);
+ *   - the log2 / exp2 round trip of the step cap is the equivalent clamp of
+ *     u_m to [2^-d - 1, 2^d - 1] (log2(1+u) is increasing), merged with the
+ *     0.75 bounds; bounds are rounded towards zero into binary32;
+ *   - clamp_a(x) = max(-a, min(x, a)) uses IEEE minNum/maxNum (C fminf and
+ *     fmaxf); optional clips are skipped entirely when switched off;
+ *   - fused multiply-adds: mu, nu and nu_e updates, the two denominators and
+ *     w + w u_m are each one fmaf();
+ *   - stochastic rounding keys a Philox4x32-10 stream by (seed, step, global
+ *     element index); the global index of a tensor's first element is the
+ *     previous tensor's end rounded up to a multiple of 8;
+ *   - FP8 storage is OCP E4M3 (bias 7, max 448, no infinities, NaN 0x7F)
+ *     with a per-tensor power-of-two scale chosen from the previous step's
+ *     largest |w| (delayed scaling), saturating encode;
+ *   - NaN stores as 0x7FFF in BF16 and 0x7F in E4M3.
+ */
+#include "mpadam_oracle.h"
+
+#include <math.h>
+#include <string.h>
+
+static float f_from_bits(uint32_t b) { float f; memcpy(&f, &b, sizeof f); return f; }
+static uint32_t bits_from_f(float f) { uint32_t b; memcpy(&b, &f, sizeof b); return b; }
+
+/* 2^k as binary32 for -126 <= k <= 127 (exact). */
+static float pow2_int(int32_t k) { return f_from_bits((uint32_t)(k + 127) << 23); }
+
+/* ------------------------------------------------------------------------ */
+/* Philox4x32-10: J. K. Salmon, M. A. Moraes, R. O. Dror, D. E. Shaw,        */
+/* "Parallel random numbers: as easy as 1, 2, 3", SC'11.  Ten rounds of the  */
+/* four-word Philox S-box; each round multiplies words 0 and 2 by the two    */
+/* round multipliers, swaps the products' halves across the block and mixes  */
+/* the high halves with words 1 and 3 and the round key.  The key advances   */
+/* by the two Weyl constants after every round.                              */
+/* ------------------------------------------------------------------------ */
+void orc_philox4x32_10(const uint32_t ctr[4], const uint32_t key[2], uint32_t out[4]) {
+  const uint32_t mult0 = 0xD2511F53u, mult1 = 0xCD9E8D57u;
+  const uint32_t weyl0 = 0x9E3779B9u, weyl1 = 0xBB67AE85u;
+  uint32_t x0 = ctr[0], x1 = ctr[1], x2 = ctr[2], x3 = ctr[3];
+  uint32_t k0 = key[0], k1 = key[1];
+  for (int round = 0; round < 10; ++round) {
+    uint64_t prod0 = (uint64_t)mult0 * (uint64_t)x0;
+    uint64_t prod1 = (uint64_t)mult1 * (uint64_t)x2;
+    uint32_t hi0 = (uint32_t)(prod0 >> 32), lo0 = (uint32_t)prod0;
+    uint32_t hi1 = (uint32_t)(prod1 >> 32), lo1 = (uint32_t)prod1;
+    uint32_t y0 = hi1 ^ x1 ^ k0;
+    uint32_t y1 = lo1;
+    uint32_t y2 = hi0 ^ x3 ^ k1;
+    uint32_t y3 = lo0;
+    x0 = y0; x1 = y1; x2 = y2; x3 = y3;
+    k0 += weyl0;
+    k1 += weyl1;
+  }
+  out[0] = x0; out[1] = x1; out[2] = x2; out[3] = x3;
+}
+
+uint32_t orc_rng_lane(uint64_t seed, uint64_t t, uint64_t i, int32_t storage) {
+  uint32_t key[2] = {(uint32_t)seed, (uint32_t)(seed >> 32)};
+  uint32_t out[4];
+  if (storage == ORC_BF16) {
+    /* 8 lanes of 16 bits per block: lane L is half (L mod 2) of word L/2. */
+    uint64_t block = i / 8;
+    uint32_t lane = (uint32_t)(i % 8);
+    uint32_t ctr[4] = {(uint32_t)block, (uint32_t)(block >> 32), (uint32_t)t, (uint32_t)(t >> 32)};
+    orc_philox4x32_10(ctr, key, out);
+    uint32_t word = out[lane / 2];
+    return (lane % 2 == 0) ? (word & 0xFFFFu) : (word >> 16);
+  }
+  /* 4 lanes of 32 bits per block. */
+  uint64_t block = i / 4;
+  uint32_t lane = (uint32_t)(i % 4);
+  uint32_t ctr[4] = {(uint32_t)block, (uint32_t)(block >> 32), (uint32_t)t, (uint32_t)(t >> 32)};
+  orc_philox4x32_10(ctr, key, out);
+  return out[lane];
+}
+
+/* ------------------------------------------------------------------------ */
+/* BF16: the upper 16 bits of a binary32.                                    */
+/* ------------------------------------------------------------------------ */
+float orc_bf16_decode(uint16_t h) { return f_from_bits((uint32_t)h << 16); }
+
+uint16_t orc_bf16_rne(float x) {
+  if (isnan(x)) return 0x7FFFu;
+  uint32_t b = bits_from_f(x);
+  uint32_t upper = b >> 16;
+  uint32_t lower = b & 0xFFFFu;
+  /* nearest; ties to the even upper half.  A carry out of the mantissa moves
+   * to the next binade, and past the largest finite value to infinity. */
+  if (lower > 0x8000u || (lower == 0x8000u && (upper & 1u))) upper += 1;
+  return (uint16_t)upper;
+}
+
+uint16_t orc_bf16_sr(float x, uint32_t r16) {
+  if (isnan(x)) return 0x7FFFu;
+  uint32_t b = bits_from_f(x);
+  uint32_t upper = b >> 16;           /* the neighbour towards zero */
+  uint32_t lower = b & 0xFFFFu;       /* distance to it, in 2^-16 of a bf16 ulp */
+  /* away from zero with probability lower / 2^16: exactly unbiased. */
+  if ((r16 & 0xFFFFu) < lower) upper += 1;
+  return (uint16_t)upper;
+}
+
+/* ------------------------------------------------------------------------ */
+/* E4M3 (OCP FP8, "fn" variant): 1 sign, 4 exponent (bias 7), 3 mantissa     */
+/* bits; largest finite 448 (0x7E); 0x7F / 0xFF are NaN; subnormal step 2^-9 */
+/* ------------------------------------------------------------------------ */
+float orc_e4m3_decode(uint8_t q) {
+  uint32_t mag = q & 0x7Fu;
+  if (mag == 0x7Fu) return NAN;
+  uint32_t e = mag >> 3, f = mag & 7u;
+  double val = (e == 0) ? ldexp((double)f, -9) : ldexp((double)(8u + f), (int)e - 10);
+  return (float)((q & 0x80u) ? -val : val);
+}
+
+/* |x| (finite, below 448) = (code + rem / 2^shift) * ulp, ulp the E4M3
+ * spacing at |x|, code the E4M3 magnitude code truncated towards zero. */
+static void e4m3_split(uint32_t abits, uint32_t* code, uint64_t* rem, int32_t* shift) {
+  uint32_t ef = abits >> 23, mant = abits & 0x7FFFFFu;
+  uint64_t sig; int32_t e;
+  if (ef == 0) { sig = mant; e = -126; }       /* binary32 subnormal */
+  else { sig = mant | 0x800000u; e = (int32_t)ef - 127; }
+  /* |x| = sig * 2^(e - 23) */
+  if (e >= -6) {                               /* E4M3 normal: ulp = 2^(e-3) */
+    *shift = 20;
+    *code = (uint32_t)(((e + 7) << 3) + (int32_t)(sig >> 20) - 8);
+    *rem = sig & 0xFFFFFu;
+  } else {                                     /* E4M3 subnormal: ulp = 2^-9 */
+    *shift = 14 - e;                           /* |x| / 2^-9 = sig * 2^(e - 14) */
+    if (*shift >= 64) { *code = 0; *rem = sig; }
+    else { *code = (uint32_t)(sig >> *shift); *rem = sig & ((1ull << *shift) - 1ull); }
+  }
+}
+
+uint8_t orc_e4m3_rne(float x) {
+  if (isnan(x)) return 0x7Fu;
+  uint32_t b = bits_from_f(x);
+  uint32_t sign = (b >> 24) & 0x80u;
+  uint32_t abits = b & 0x7FFFFFFFu;
+  if (abits >= bits_from_f(448.0f)) return (uint8_t)(sign | 0x7Eu);   /* saturate */
+  uint32_t code; uint64_t rem; int32_t shift;
+  e4m3_split(abits, &code, &rem, &shift);
+  if (shift <= 40) {  /* for larger shifts rem < 2^24 is far below one half */
+    uint64_t half = 1ull << (shift - 1);
+    if (rem > half || (rem == half && (code & 1u))) code += 1;
+  }
+  if (code > 0x7Eu) code = 0x7Eu;
+  return (uint8_t)(sign | code);
+}
+
+uint8_t orc_e4m3_sr(float x, uint32_t r32) {
+  if (isnan(x)) return 0x7Fu;
+  uint32_t b = bits_from_f(x);
+  uint32_t sign = (b >> 24) & 0x80u;
+  uint32_t abits = b & 0x7FFFFFFFu;
+  if (abits >= bits_from_f(448.0f)) return (uint8_t)(sign | 0x7Eu);
+  uint32_t code; uint64_t rem; int32_t shift;
+  e4m3_split(abits, &code, &rem, &shift);
+  /* threshold = floor(fraction * 2^32); away from zero iff r < threshold */
+  uint64_t thr;
+  if (shift <= 32) thr = rem << (32 - shift);
+  else if (shift - 32 >= 64) thr = 0;
+  else thr = rem >> (shift - 32);
+  if ((uint64_t)r32 < thr) code += 1;
+  if (code > 0x7Eu) code = 0x7Eu;
+  return (uint8_t)(sign | code);
+}
+
+int32_t orc_fp8_next_exponent(float amax, int32_t e_cur) {
+  if (!(amax > 0.0f) || isinf(amax)) return e_cur;   /* nothing to fit: keep */
+  int x;
+  float f = frexpf(amax, &x);                        /* amax = f 2^x, f in [0.5, 1) */
+  /* smallest k with amax <= 448 2^k = 0.875 2^(9+k) */
+  int32_t k = (f <= 0.875f) ? x - 9 : x - 8;
+  if (k < -100) k = -100;
+  if (k > 100) k = 100;
+  return k;
+}
+
+float orc_e4m3_amax(int64_t n, const uint8_t* q, int32_t e) {
+  float amax = 0.0f;
+  float scale = pow2_int(e);
+  for (int64_t k = 0; k < n; ++k) {
+    float val = orc_e4m3_decode(q[k]);
+    if (isnan(val)) continue;
+    float a = fabsf(val * scale);
+    if (a > amax) amax = a;
+  }
+  return amax;
+}
+
+/* ------------------------------------------------------------------------ */
+/* Per-step scalars                                                          */
+/* ------------------------------------------------------------------------ */
+static float to_f32_toward_zero(double x) {
+  float f = (float)x;
+  if (x > 0.0 && (double)f > x) f = nextafterf(f, 0.0f);
+  if (x < 0.0 && (double)f < x) f = nextafterf(f, 0.0f);
+  return f;
+}
+
+static int finite_pos(float x) { return isfinite(x) && x > 0.0f; }
+
+int32_t orc_scalars_for_step(const orc_hparams* hp, int64_t t, orc_scalars* s) {
+  if (t < 1) return -1;
+  if (!(isfinite(hp->lr_add) && hp->lr_add >= 0.0f)) return -1;
+  if (!(isfinite(hp->lr_mul) && hp->lr_mul >= 0.0f)) return -1;
+  if (!(hp->beta1 >= 0.0f && hp->beta1 < 1.0f)) return -1;
+  if (!(hp->beta2 >= 0.0f && hp->beta2 < 1.0f)) return -1;
+  if (!finite_pos(hp->eps) || !finite_pos(hp->tau)) return -1;
+  if (!finite_pos(hp->rmax_pos)) return -1;
+  if (!(finite_pos(hp->rmax_neg) && hp->rmax_neg < 1.0f)) return -1;
+  if (!(hp->g_max > 0.0f) || !(hp->dmult_max > 0.0f) || !(hp->w_max > 0.0f)) return -1;
+  if (!(isfinite(hp->wd_add) && hp->wd_add >= 0.0f)) return -1;
+
+  double b1 = hp->beta1, b2 = hp->beta2;
+  double bc1 = 1.0, bc2 = 1.0;
+  if (hp->bias_correction) {
+    bc1 = 1.0 - pow(b1, (double)t);
+    bc2 = 1.0 - pow(b2, (double)t);
+  }
+  s->b1 = hp->beta1;
+  s->b2 = hp->beta2;
+  s->omb1 = (float)(1.0 - b1);
+  s->omb2 = (float)(1.0 - b2);
+  s->ka = (float)(-(double)hp->lr_add / bc1);
+  s->c2 = (float)(1.0 / sqrt(bc2));
+  s->km = -hp->lr_mul;
+  s->ln2 = (float)0.69314718055994530942;
+  s->eps = hp->eps;
+  s->tau = hp->tau;
+  double d = hp->dmult_max;
+  double hi = fmin((double)hp->rmax_pos, exp2(d) - 1.0);
+  double lo = fmax(-(double)hp->rmax_neg, exp2(-d) - 1.0);
+  s->hi = to_f32_toward_zero(hi);
+  s->lo = to_f32_toward_zero(lo);
+  s->gmax_on = isfinite(hp->g_max) ? 1 : 0;
+  s->gmax = s->gmax_on ? hp->g_max : 0.0f;
+  s->wmax_on = isfinite(hp->w_max) ? 1 : 0;
+  s->wmax = s->wmax_on ? hp->w_max : 0.0f;
+  s->wd_on = hp->wd_add != 0.0f ? 1 : 0;
+  s->kwd = (float)((double)hp->lr_add * (double)hp->wd_add);
+  return 0;
+}
+
+/* ------------------------------------------------------------------------ */
+/* The canonical per-element update (Algorithm 1 + Algorithm 2 options)      */
+/* ------------------------------------------------------------------------ */
+void orc_update_element(const orc_scalars* s, float w, float g, float m, float v, float ve,
+                        float* wn_out, float* m_out, float* v_out, float* ve_out) {
+  /* additive branch: Adam moments */
+  float m1 = fmaf(s->b1, m, s->omb1 * g);                 /* mu <- b1 mu + (1-b1) g */
+  float v1 = fmaf(s->b2, v, s->omb2 * (g * g));           /* nu <- b2 nu + (1-b2) g^2 */
+  /* u_a = -eta_a mu-hat / (sqrt(nu-hat) + eps) */
+  float den_a = fmaf(sqrtf(v1), s->c2, s->eps);
+  float ua = (s->ka * m1) / den_a;
+  if (s->wd_on) ua = ua - s->kwd * w;                     /* decoupled additive decay */
+
+  /* multiplicative branch */
+  float ge = (s->ln2 * w) * g;                            /* g_e = (ln 2) w g */
+  float ve1 = fmaf(s->b2, ve, s->omb2 * (ge * ge));       /* nu_e <- b2 nu_e + (1-b2) g_e^2 */
+  float den_e = fmaf(sqrtf(ve1), s->c2, s->eps);
+  float n = ge / den_e;                                   /* normalised exponent gradient */
+  if (s->gmax_on) n = fmaxf(-s->gmax, fminf(n, s->gmax));
+  float rho = fmaxf(fabsf(w), s->tau);                    /* rho = max(|w|, tau) */
+  float um = (s->km * n) / rho;                           /* u_m = u~ / rho, u~ = -eta_m n */
+  um = fmaxf(s->lo, fminf(um, s->hi));                    /* relative bounds and step cap */
+
+  /* combine: w + w u_m + u_a */
+  float wn = fmaf(w, um, w) + ua;
+  if (s->wmax_on) wn = fmaxf(-s->wmax, fminf(wn, s->wmax));
+
+  *wn_out = wn; *m_out = m1; *v_out = v1; *ve_out = ve1;
+}
+
+/* ------------------------------------------------------------------------ */
+/* One step over a run of elements                                           */
+/* ------------------------------------------------------------------------ */
+static float load_elem(const void* p, int64_t k, int32_t dt) {
+  if (dt == ORC_F32) return ((const float*)p)[k];
+  if (dt == ORC_BF16) return orc_bf16_decode(((const uint16_t*)p)[k]);
+  return orc_e4m3_decode(((const uint8_t*)p)[k]);
+}
+
+static void store_moment(void* p, int64_t k, int32_t dt, float x) {
+  if (dt == ORC_F32) ((float*)p)[k] = x;
+  else ((uint16_t*)p)[k] = orc_bf16_rne(x);
+}
+
+int32_t orc_step_elements(int64_t n, const int64_t* gidx, int64_t gidx0,
+                          int32_t wdt, int32_t gdt, int32_t mdt,
+                          void* w, const void* g, void* m, void* v, void* ve,
+                          const orc_hparams* hp, int64_t t,
+                          int32_t e_cur, int32_t e_next, float* amax) {
+  if (wdt != ORC_F32 && wdt != ORC_BF16 && wdt != ORC_E4M3) return -1;
+  if (gdt != ORC_F32 && gdt != ORC_BF16) return -1;
+  if (mdt != ORC_F32 && mdt != ORC_BF16) return -1;
+  if (e_cur < -100 || e_cur > 100 || e_next < -100 || e_next > 100) return -1;
+  orc_scalars s;
+  if (orc_scalars_for_step(hp, t, &s) != 0) return -1;
+  float dec_scale = pow2_int(e_cur);
+  float enc_scale = pow2_int(-e_next);
+
+  for (int64_t k = 0; k < n; ++k) {
+    uint64_t i = (uint64_t)(gidx ? gidx[k] : gidx0 + k);
+    float wk = load_elem(w, k, wdt);
+    if (wdt == ORC_E4M3) wk = wk * dec_scale;
+    float gk = load_elem(g, k, gdt);
+    float mk = load_elem(m, k, mdt);
+    float vk = load_elem(v, k, mdt);
+    float vek = load_elem(ve, k, mdt);
+
+    float wn, m1, v1, ve1;
+    orc_update_element(&s, wk, gk, mk, vk, vek, &wn, &m1, &v1, &ve1);
+
+    if (wdt == ORC_F32) {
+      ((float*)w)[k] = wn;
+    } else if (wdt == ORC_BF16) {
+      uint16_t h = hp->stochastic ? orc_bf16_sr(wn, orc_rng_lane(hp->seed, (uint64_t)t, i, ORC_BF16))
+                                  : orc_bf16_rne(wn);
+      ((uint16_t*)w)[k] = h;
+    } else {
+      if (isfinite(wn) && fabsf(wn) > *amax) *amax = fabsf(wn);
+      float x = wn * enc_scale;
+      uint8_t q = hp->stochastic ? orc_e4m3_sr(x, orc_rng_lane(hp->seed, (uint64_t)t, i, ORC_E4M3))
+                                 : orc_e4m3_rne(x);
+      ((uint8_t*)w)[k] = q;
+    }
+    store_moment(m, k, mdt, m1);
+    store_moment(v, k, mdt, v1);
+    store_moment(ve, k, mdt, ve1);
+  }
+  return 0;
+}
+
+/* ------------------------------------------------------------------------ */
+/* Array helpers for the tests: plain loops over the scalar functions above. */
+/* ------------------------------------------------------------------------ */
+void orc_bf16_rne_n(int64_t n, const float* x, uint16_t* out) {
+  for (int64_t k = 0; k < n; ++k) out[k] = orc_bf16_rne(x[k]);
+}
+void orc_bf16_sr_n(int64_t n, const float* x, const uint32_t* r16, uint16_t* out) {
+  for (int64_t k = 0; k < n; ++k) out[k] = orc_bf16_sr(x[k], r16[k]);
+}
+void orc_e4m3_rne_n(int64_t n, const float* x, uint8_t* out) {
+  for (int64_t k = 0; k < n; ++k) out[k] = orc_e4m3_rne(x[k]);
+}
+void orc_e4m3_sr_n(int64_t n, const float* x, const uint32_t* r32, uint8_t* out) {
+  for (int64_t k = 0; k < n; ++k) out[k] = orc_e4m3_sr(x[k], r32[k]);
+}
+void orc_e4m3_decode_n(int64_t n, const uint8_t* q, float* out) {
+  for (int64_t k = 0; k < n; ++k) out[k] = orc_e4m3_decode(q[k]);
+}
+void orc_rng_lanes_n(uint64_t seed, uint64_t t, int32_t storage, int64_t n,
+                     const uint64_t* idx, uint32_t* out) {
+  for (int64_t k = 0; k < n; ++k) out[k] = orc_rng_lane(seed, t, idx[k], storage);
+}
+void orc_philox_n(int64_t n, const uint32_t* ctr, const uint32_t* key, uint32_t* out) {
+  for (int64_t k = 0; k < n; ++k) orc_philox4x32_10(ctr + 4 * k, key, out + 4 * k);
+}
+int32_t orc_update_elements_n(const orc_hparams* hp, int64_t t, int64_t n,
+                              const float* w, const float* g, const float* m,
+                              const float* v, const float* ve,
+                              float* wn, float* m1, float* v1, float* ve1) {
+  orc_scalars s;
+  if (orc_scalars_for_step(hp, t, &s) != 0) return -1;
+  for (int64_t k = 0; k < n; ++k)
+    orc_update_element(&s, w[k], g[k], m[k], v[k], ve[k], wn + k, m1 + k, v1 + k, ve1 + k);
+  return 0;
+}

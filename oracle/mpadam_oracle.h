@@ -1,0 +1,115 @@
+/*
+ * mpadam_oracle.h -- plain single-threaded CPU oracle of the M+Adam optimizer
+ * step (arxiv 2607.10611, Algorithm 1 with the options of Algorithm 2,
+ * Appendix A).
+ *
+ * TEST INFRASTRUCTURE ONLY. Only the test suite, the smoke check and the CPU
+ * baseline leg of the benchmark may load this library. The product library
+ * (include/mpadam.h, the CUDA kernels) shares no code, header, table or
+ * helper with this file, and neither side includes or links the other.
+ *
+ * Arithmetic model: every per-element operation is an IEEE-754 binary32
+ * operation with round-to-nearest-even (the paper's toy diagnostic, Sec. 5.1
+ * and Appendix B, computes each step in FP32 and rounds the parameter
+ * immediately).  Fused multiply-adds appear only where written as fmaf().
+ * Build with -ffp-contract=off so the compiler adds no others.
+ */
+#ifndef MPADAM_ORACLE_H
+#define MPADAM_ORACLE_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Element formats. */
+enum { ORC_F32 = 0, ORC_BF16 = 1, ORC_E4M3 = 2 };
+
+/* Hyper-parameters (Algorithm 1 inputs; Algorithm 2 optional clips). */
+typedef struct {
+  float lr_add;          /* eta_a */
+  float lr_mul;          /* eta_m */
+  float beta1, beta2;    /* moment decay rates */
+  float eps;             /* stabiliser, > 0 */
+  float tau;             /* threshold of rho = max(|w|, tau), > 0 */
+  float rmax_pos;        /* upper bound of u_m (0.75 in Algorithm 2) */
+  float rmax_neg;        /* magnitude of the lower bound, 0.75 - eps0 */
+  float g_max;           /* clamp of the normalised exponent gradient; +inf = off */
+  float dmult_max;       /* cap on |log2(1 + u_m)|; +inf = off */
+  float w_max;           /* final weight clip; +inf = off */
+  float wd_add;          /* decoupled additive weight decay lambda; 0 = off */
+  int32_t bias_correction; /* 1: Algorithm 1 (u-hat, v-hat); 0: Algorithm 2 */
+  int32_t stochastic;    /* 0: round to nearest even, 1: stochastic rounding */
+  uint64_t seed;         /* Philox key */
+} orc_hparams;
+
+/* Per-step binary32 scalars, each computed in binary64 and rounded once. */
+typedef struct {
+  float b1, b2;      /* beta1, beta2 */
+  float omb1, omb2;  /* 1 - beta1, 1 - beta2 */
+  float ka;          /* -eta_a / (1 - beta1^t)   (or -eta_a without bias correction) */
+  float c2;          /* 1 / sqrt(1 - beta2^t)    (or 1) */
+  float km;          /* -eta_m */
+  float ln2;         /* ln 2 */
+  float eps, tau;
+  float lo, hi;      /* bounds of u_m: rmax and the log2 step cap merged */
+  float gmax, wmax, kwd;
+  int32_t gmax_on, wmax_on, wd_on;
+} orc_scalars;
+
+/* Philox4x32-10 block function (Salmon et al., SC'11). */
+void orc_philox4x32_10(const uint32_t ctr[4], const uint32_t key[2], uint32_t out[4]);
+
+/* Random bits drawn for global element index i at step t:
+ * BF16 storage: 16 bits, E4M3 storage: 32 bits. */
+uint32_t orc_rng_lane(uint64_t seed, uint64_t t, uint64_t i, int32_t storage);
+
+uint16_t orc_bf16_rne(float x);
+uint16_t orc_bf16_sr(float x, uint32_t r16);
+float    orc_bf16_decode(uint16_t h);
+uint8_t  orc_e4m3_rne(float x);
+uint8_t  orc_e4m3_sr(float x, uint32_t r32);
+float    orc_e4m3_decode(uint8_t q);
+
+/* Per-tensor power-of-two scale exponent for the next encode. */
+int32_t  orc_fp8_next_exponent(float amax, int32_t e_cur);
+
+/* 0 on success, -1 on invalid hyper-parameters or t < 1. */
+int32_t  orc_scalars_for_step(const orc_hparams* hp, int64_t t, orc_scalars* out);
+
+/* The canonical per-element update in binary32. */
+void orc_update_element(const orc_scalars* s, float w, float g, float m, float v, float ve,
+                        float* wn, float* m1, float* v1, float* ve1);
+
+/* One optimizer step over n elements held in host arrays, updated in place.
+ * Element k has global index gidx[k] (or gidx0 + k when gidx is NULL).
+ * E4M3 weights decode with 2^e_cur and encode with 2^e_next; *amax is raised
+ * to the largest finite |updated weight| seen.  Returns 0 or -1. */
+int32_t orc_step_elements(int64_t n, const int64_t* gidx, int64_t gidx0,
+                          int32_t wdt, int32_t gdt, int32_t mdt,
+                          void* w, const void* g, void* m, void* v, void* ve,
+                          const orc_hparams* hp, int64_t t,
+                          int32_t e_cur, int32_t e_next, float* amax);
+
+/* Largest finite |decoded E4M3 weight| of a tensor stored with exponent e. */
+float orc_e4m3_amax(int64_t n, const uint8_t* q, int32_t e);
+
+/* Array forms of the scalar functions (plain loops), for the tests. */
+void orc_bf16_rne_n(int64_t n, const float* x, uint16_t* out);
+void orc_bf16_sr_n(int64_t n, const float* x, const uint32_t* r16, uint16_t* out);
+void orc_e4m3_rne_n(int64_t n, const float* x, uint8_t* out);
+void orc_e4m3_sr_n(int64_t n, const float* x, const uint32_t* r32, uint8_t* out);
+void orc_e4m3_decode_n(int64_t n, const uint8_t* q, float* out);
+void orc_rng_lanes_n(uint64_t seed, uint64_t t, int32_t storage, int64_t n,
+                     const uint64_t* idx, uint32_t* out);
+void orc_philox_n(int64_t n, const uint32_t* ctr, const uint32_t* key, uint32_t* out);
+int32_t orc_update_elements_n(const orc_hparams* hp, int64_t t, int64_t n,
+                              const float* w, const float* g, const float* m,
+                              const float* v, const float* ve,
+                              float* wn, float* m1, float* v1, float* ve1);
+
+#ifdef __cplusplus
+}
+#endif
+#endif

@@ -1,0 +1,327 @@
+"""Seeded synthetic optimizer-step inputs shaped like LLM parameter sets.
+
+This module is the only code shared by the oracle-side tests and the CUDA-side
+tests/benchmark.  It draws weights, gradients and optimizer states; it holds
+none of the M+Adam arithmetic (no moment update, no rounding rule, no scale
+rule).  The FP8 initial weights are produced with torch's own float8_e4m3fn
+cast of a pre-scaled draw, with a per-role power-of-two exponent chosen from
+the draw's standard deviation: an input recipe, not the optimizer's delayed
+scale rule.
+
+Stand-ins: the paper trains LLaMA-style decoders on C4/EN (Sec. 5.2, the
+model-architecture table of Appendix C).  An optimizer step needs no data, so
+the workloads here are parameter lists with the shapes of GPT-2 small and of
+LLaMA-style 1.5B / 7B models, plus a flat tensor and a ragged stress list;
+values are seeded random draws, not trained weights.
+
+Layout: tensor k's first element has global index off[k], where off[0] = 0 and
+off[k+1] is off[k] + numel[k] rounded up to a multiple of 8 (the library's
+documented element-index layout).  With ``layout="flat"`` every array kind
+(w, g, m, v, ve) is one allocation indexed by that global index, and tensors are
+views into it; with ``layout="separate"`` each tensor is its own allocation.
+"""
+from __future__ import annotations
+
+import math
+from dataclasses import dataclass, field, replace
+from typing import Dict, List, Optional
+
+import torch
+
+ALIGN = 8  # elements; tensor starts in the global index space
+
+
+@dataclass(frozen=True)
+class TensorSpec:
+    name: str
+    numel: int
+    role: str  # "matrix" | "embedding" | "bias" | "norm" | "flat"
+
+
+@dataclass(frozen=True)
+class Workload:
+    name: str
+    specs: tuple
+    weight_dtype: str          # "bf16" | "e4m3"
+    grad_dtype: str            # "f32" | "bf16"
+    moment_dtype: str          # "f32" | "bf16"
+    rounding: str              # "nearest" | "stochastic"
+    steps: int
+    seed: int = 0
+    w_std: float = 0.02
+    zero_frac: float = 0.0     # fraction of weights set exactly to 0
+    grad: tuple = ("normal", 1e-3)  # ("normal", s) | ("normal_logu", lo, hi) | ("student_t_logu", nu, lo, hi)
+    norm_gain: float = 1.0     # initial value of norm gains
+    bias_zero: bool = True     # biases start at exactly 0
+    description: str = ""
+
+    @property
+    def numels(self) -> List[int]:
+        return [s.numel for s in self.specs]
+
+    @property
+    def n_params(self) -> int:
+        return sum(self.numels)
+
+
+def global_offsets(numels) -> List[int]:
+    """Start index of each tensor in the padded global element index space."""
+    offs, o = [], 0
+    for n in numels:
+        offs.append(o)
+        o = (o + int(n) + ALIGN - 1) // ALIGN * ALIGN
+    return offs
+
+
+def global_length(numels) -> int:
+    o = 0
+    for n in numels:
+        o = (o + int(n) + ALIGN - 1) // ALIGN * ALIGN
+    return o
+
+
+# ---------------------------------------------------------------------------
+# Parameter-list shapes
+# ---------------------------------------------------------------------------
+def gpt2_specs(layers=12, d=768, vocab=50257, ctx=1024) -> tuple:
+    """GPT-2 small layout (tied LM head): wte, wpe, per-block LN/attn/MLP, ln_f."""
+    s = [TensorSpec("wte", vocab * d, "embedding"), TensorSpec("wpe", ctx * d, "embedding")]
+    for i in range(layers):
+        p = f"h{i}."
+        s += [
+            TensorSpec(p + "ln_1.weight", d, "norm"), TensorSpec(p + "ln_1.bias", d, "bias"),
+            TensorSpec(p + "attn.c_attn.weight", d * 3 * d, "matrix"),
+            TensorSpec(p + "attn.c_attn.bias", 3 * d, "bias"),
+            TensorSpec(p + "attn.c_proj.weight", d * d, "matrix"),
+            TensorSpec(p + "attn.c_proj.bias", d, "bias"),
+            TensorSpec(p + "ln_2.weight", d, "norm"), TensorSpec(p + "ln_2.bias", d, "bias"),
+            TensorSpec(p + "mlp.c_fc.weight", d * 4 * d, "matrix"),
+            TensorSpec(p + "mlp.c_fc.bias", 4 * d, "bias"),
+            TensorSpec(p + "mlp.c_proj.weight", 4 * d * d, "matrix"),
+            TensorSpec(p + "mlp.c_proj.bias", d, "bias"),
+        ]
+    s += [TensorSpec("ln_f.weight", d, "norm"), TensorSpec("ln_f.bias", d, "bias")]
+    return tuple(s)
+
+
+def llama_specs(layers, d, ffn, vocab) -> tuple:
+    """LLaMA-style decoder: embed, per layer q/k/v/o, SwiGLU gate/up/down and two
+    RMSNorm gains, final norm, untied LM head."""
+    s = [TensorSpec("embed_tokens", vocab * d, "embedding")]
+    for i in range(layers):
+        p = f"layers.{i}."
+        s += [
+            TensorSpec(p + "self_attn.q_proj", d * d, "matrix"),
+            TensorSpec(p + "self_attn.k_proj", d * d, "matrix"),
+            TensorSpec(p + "self_attn.v_proj", d * d, "matrix"),
+            TensorSpec(p + "self_attn.o_proj", d * d, "matrix"),
+            TensorSpec(p + "mlp.gate_proj", d * ffn, "matrix"),
+            TensorSpec(p + "mlp.up_proj", d * ffn, "matrix"),
+            TensorSpec(p + "mlp.down_proj", ffn * d, "matrix"),
+            TensorSpec(p + "input_layernorm", d, "norm"),
+            TensorSpec(p + "post_attention_layernorm", d, "norm"),
+        ]
+    s += [TensorSpec("norm", d, "norm"), TensorSpec("lm_head", vocab * d, "matrix")]
+    return tuple(s)
+
+
+def ragged_specs(n_tensors, max_log2, seed) -> tuple:
+    """Sizes round(exp(U[0, ln 2^max_log2])): log-uniform in [1, 2^max_log2]."""
+    g = torch.Generator().manual_seed(10_000 + seed)
+    u = torch.rand(n_tensors, generator=g, dtype=torch.float64)
+    sizes = torch.round(torch.exp(u * (max_log2 * math.log(2.0)))).to(torch.int64).clamp_min(1)
+    return tuple(TensorSpec(f"t{i}", int(n), "flat") for i, n in enumerate(sizes.tolist()))
+
+
+def _flat1m():
+    return Workload(
+        name="flat_1m", specs=(TensorSpec("flat", 1 << 20, "flat"),),
+        weight_dtype="bf16", grad_dtype="f32", moment_dtype="f32", rounding="nearest",
+        steps=10, zero_frac=0.01, grad=("normal", 1e-3),
+        description="single flat tensor of 1,048,576 params: bf16 w ~N(0,0.02) with 1% zeros, "
+                    "fp32 g ~N(0,1e-3), fp32 moments, round-to-nearest")
+
+
+def _gpt2(layers=12, d=768, vocab=50257, ctx=1024, name="gpt2_124m"):
+    return Workload(
+        name=name, specs=gpt2_specs(layers, d, vocab, ctx),
+        weight_dtype="bf16", grad_dtype="bf16", moment_dtype="f32", rounding="stochastic",
+        steps=100, grad=("normal_logu", 1e-5, 1e-2),
+        description="GPT-2-small-shaped list: bf16 w ~N(0,0.02) (LN gains 1, biases 0), bf16 g "
+                    "with per-tensor std log-uniform [1e-5,1e-2], fp32 moments, stochastic rounding")
+
+
+def _llama15(layers=24, d=2048, ffn=5632, vocab=32000, name="llama_1p5b"):
+    return Workload(
+        name=name, specs=llama_specs(layers, d, ffn, vocab),
+        weight_dtype="e4m3", grad_dtype="bf16", moment_dtype="f32", rounding="stochastic",
+        steps=10, grad=("student_t_logu", 3.0, 1e-5, 1e-2),
+        description="LLaMA-style 1.5B list (24 layers, d=2048, ffn 5632, vocab 32000): E4M3 weights "
+                    "with per-tensor power-of-two scale, bf16 Student-t(3) grads scaled per tensor "
+                    "(std log-uniform [1e-5,1e-2]), fp32 moments, stochastic rounding")
+
+
+def _llama7(layers=32, d=4096, ffn=11008, vocab=32000, name="llama_7b"):
+    return Workload(
+        name=name, specs=llama_specs(layers, d, ffn, vocab),
+        weight_dtype="bf16", grad_dtype="bf16", moment_dtype="bf16", rounding="stochastic",
+        steps=10, grad=("normal_logu", 1e-6, 1e-2),
+        description="LLaMA-style 7B list (32 layers, d=4096, ffn 11008, vocab 32000): bf16 weights, "
+                    "bf16 grads with per-tensor std log-uniform [1e-6,1e-2], bf16 moments, "
+                    "stochastic rounding")
+
+
+def _ragged(n=20000, max_log2=22, name="ragged_20k", rounding="stochastic"):
+    return Workload(
+        name=name, specs=ragged_specs(n, max_log2, 0),
+        weight_dtype="bf16", grad_dtype="bf16", moment_dtype="f32", rounding=rounding,
+        steps=10, zero_frac=0.30, grad=("normal", 1e-3),
+        description=f"ragged list of {n} tensors, sizes log-uniform [1, 2^{max_log2}], 30% zero "
+                    "weights, bf16 w/g, fp32 moments")
+
+
+CONFIGS: Dict[str, Workload] = {
+    "flat_1m": _flat1m(),
+    "gpt2_124m": _gpt2(),
+    "llama_1p5b": _llama15(),
+    "llama_7b": _llama7(),
+    "ragged_20k": _ragged(),
+}
+
+# Same distributions and formats at sizes the oracle finishes in seconds,
+# still spanning many 2048-element CTA tiles and ragged tails.
+SMALL: Dict[str, Workload] = {
+    "flat_1m": replace(_flat1m(), specs=(TensorSpec("flat", (1 << 16) + 5, "flat"),), name="flat_small"),
+    "gpt2_124m": _gpt2(layers=2, d=64, vocab=1003, ctx=64, name="gpt2_small"),
+    "llama_1p5b": _llama15(layers=2, d=128, ffn=344, vocab=517, name="llama15_small"),
+    "llama_7b": _llama7(layers=2, d=128, ffn=344, vocab=517, name="llama7_small"),
+    "ragged_20k": _ragged(n=300, max_log2=13, name="ragged_small"),
+}
+
+
+# ---------------------------------------------------------------------------
+# Materialisation
+# ---------------------------------------------------------------------------
+_TORCH = {"f32": torch.float32, "bf16": torch.bfloat16, "e4m3": torch.uint8}
+
+
+def _gen(device, seed, k, salt):
+    g = torch.Generator(device=device)
+    g.manual_seed((seed * 1_000_003 + k * 7919 + salt) % (2**63 - 1))
+    return g
+
+
+def _grad_std(wl: Workload, k: int) -> float:
+    kind = wl.grad[0]
+    if kind == "normal":
+        return float(wl.grad[1])
+    lo, hi = (wl.grad[1], wl.grad[2]) if kind == "normal_logu" else (wl.grad[2], wl.grad[3])
+    u = torch.rand(1, generator=_gen("cpu", wl.seed, k, 5), dtype=torch.float64).item()
+    return math.exp(math.log(lo) + u * (math.log(hi) - math.log(lo)))
+
+
+def fp8_initial_exponent(role: str, w_std: float, norm_gain: float) -> int:
+    """Power-of-two exponent the synthetic FP8 weights are first stored with:
+    6 sigma (or the norm gain) fits under E4M3's largest finite value 448."""
+    top = norm_gain if role == "norm" else 6.0 * w_std
+    if role == "bias":
+        top = 6.0 * w_std
+    return int(math.ceil(math.log2(top / 448.0)))
+
+
+@dataclass
+class Materialized:
+    workload: Workload
+    offsets: List[int]
+    length: int
+    w: List[torch.Tensor]
+    g: List[torch.Tensor]
+    m: List[torch.Tensor]
+    v: List[torch.Tensor]
+    ve: List[torch.Tensor]
+    fp8_exp: Optional[List[int]] = None
+    flat: Dict[str, torch.Tensor] = field(default_factory=dict)
+
+
+def _alloc(kind_dtype, numels, offsets, length, device, layout):
+    if layout == "flat":
+        base = torch.zeros(length, dtype=kind_dtype, device=device)
+        return base, [base[o:o + n] for o, n in zip(offsets, numels)]
+    return None, [torch.zeros(n, dtype=kind_dtype, device=device) for n in numels]
+
+
+def materialize(wl: Workload, device="cpu", layout="separate", warm_state=False) -> Materialized:
+    """Draw the workload's tensors on `device` (values depend on the device's
+    generator).  warm_state=True also draws non-zero moments (as after some
+    training), for checks beyond the first step."""
+    numels = wl.numels
+    offsets = global_offsets(numels)
+    length = global_length(numels)
+    wdt, gdt, mdt = _TORCH[wl.weight_dtype], _TORCH[wl.grad_dtype], _TORCH[wl.moment_dtype]
+    flat = {}
+    fw, w = _alloc(wdt, numels, offsets, length, device, layout)
+    fg, g = _alloc(gdt, numels, offsets, length, device, layout)
+    fm, m = _alloc(mdt, numels, offsets, length, device, layout)
+    fv, v = _alloc(mdt, numels, offsets, length, device, layout)
+    fve, ve = _alloc(mdt, numels, offsets, length, device, layout)
+    if layout == "flat":
+        flat = {"w": fw, "g": fg, "m": fm, "v": fv, "ve": fve}
+    fp8_exp = [] if wl.weight_dtype == "e4m3" else None
+
+    for k, spec in enumerate(wl.specs):
+        n = spec.numel
+        if n == 0:
+            if fp8_exp is not None:
+                fp8_exp.append(0)
+            continue
+        gw = _gen(device, wl.seed, k, 1)
+        # weights
+        if spec.role == "norm":
+            wf = torch.full((n,), wl.norm_gain, dtype=torch.float32, device=device)
+        elif spec.role == "bias" and wl.bias_zero:
+            wf = torch.zeros(n, dtype=torch.float32, device=device)
+        else:
+            wf = torch.randn(n, generator=gw, dtype=torch.float32, device=device) * wl.w_std
+            if wl.zero_frac > 0:
+                z = torch.rand(n, generator=gw, device=device) < wl.zero_frac
+                wf[z] = 0.0
+        if wl.weight_dtype == "e4m3":
+            e0 = fp8_initial_exponent(spec.role, wl.w_std, wl.norm_gain)
+            fp8_exp.append(e0)
+            q = (wf * (2.0 ** -e0)).clamp_(-448.0, 448.0).to(torch.float8_e4m3fn)
+            w[k].copy_(q.view(torch.uint8))
+        else:
+            w[k].copy_(wf.to(wdt))
+        # gradients
+        gg = _gen(device, wl.seed, k, 2)
+        sd = _grad_std(wl, k)
+        if wl.grad[0] == "student_t_logu":
+            nu = float(wl.grad[1])
+            z = torch.randn(n, generator=gg, dtype=torch.float32, device=device)
+            chi = torch.zeros(n, dtype=torch.float32, device=device)
+            for _ in range(int(nu)):
+                chi += torch.randn(n, generator=gg, dtype=torch.float32, device=device) ** 2
+            gf = z / torch.sqrt(chi / nu) * sd
+        else:
+            gf = torch.randn(n, generator=gg, dtype=torch.float32, device=device) * sd
+        g[k].copy_(gf.to(gdt))
+        # optimizer states
+        if warm_state:
+            gs = _gen(device, wl.seed, k, 3)
+            wabs = wf.abs() + 1e-3
+            mf = 0.3 * sd * torch.randn(n, generator=gs, dtype=torch.float32, device=device)
+            vf = (sd * (0.5 + torch.rand(n, generator=gs, device=device))) ** 2
+            vef = (0.69314718 * sd * wabs * (0.5 + torch.rand(n, generator=gs, device=device))) ** 2
+            m[k].copy_(mf.to(mdt))
+            v[k].copy_(vf.to(mdt))
+            ve[k].copy_(vef.to(mdt))
+    return Materialized(wl, offsets, length, w, g, m, v, ve, fp8_exp, flat)
+
+
+def to_numpy_bits(t: torch.Tensor):
+    """Host numpy view: float32 stays float32, bfloat16 becomes uint16 bits,
+    uint8 (E4M3 codes) stays uint8."""
+    t = t.detach().to("cpu").contiguous()
+    if t.dtype == torch.bfloat16:
+        return t.view(torch.int16).numpy().view("uint16").copy()
+    return t.numpy().copy()
