@@ -1,0 +1,386 @@
+#!/usr/bin/env python3
+"""Benchmark of the fused M+Adam optimizer step on GB300.
+
+One "step" is one mpadam_step over the whole tensor list (every element read
+and written once).  Default workload: the LLaMA-style 7B parameter list (bf16
+weights, grads and moments, stochastic rounding); the 1.5B list (E4M3
+weights, fp32 moments) is measured in the same run as a secondary line.
+
+    python bench.py [--steps K] [--warmup W] [--config llama_7b] [--impl reference]
+
+Prints ONE JSON line (rank 0).  `value` is Gparams/s of the device-timed
+step with inputs resident in HBM (all inputs are larger than L2, so no flush
+is needed); `e2e` is the same metric through mpadam_step_host with pinned
+host gradients in and updated weights out inside the timed region;
+`roofline` relates the kernel's algorithmic bytes per launch, over its
+CUDA-event duration, to the measured HBM copy bandwidth; `cpu_baseline`
+times the CPU oracle on a bounded sample.  `--impl reference` times the
+oracle itself as the reference arm.  Under torchrun every rank runs its own
+replica of the workload (weak scaling; no collective on the data path).
+"""
+from __future__ import annotations
+
+import argparse
+import csv
+import hashlib
+import json
+import math
+import os
+import subprocess
+import sys
+import time
+from datetime import datetime
+from pathlib import Path
+
+ROOT = Path(__file__).resolve().parent
+sys.path.insert(0, str(ROOT))
+
+METRIC = "fused M+Adam step Gparams/s and HBM GB/s as % of GB300 peak (1 GPU)"
+UNIT = "Gparams/s"
+BYTES = {"f32": 4, "bf16": 2, "e4m3": 1}
+
+
+def algorithmic_bytes_per_param(wl) -> int:
+    """Reads + writes of one element: w (r+w), g (r), mu, nu, nu_e (r+w)."""
+    return 2 * BYTES[wl.weight_dtype] + BYTES[wl.grad_dtype] + 6 * BYTES[wl.moment_dtype]
+
+
+def measured_peaks():
+    p = ROOT / "MEASURED_PEAKS.json"
+    if p.exists():
+        d = json.loads(p.read_text())
+        return float(d["hbm_gbs"]), "measured"
+    return 6800.0, "fallback"
+
+
+def kernel_source_hash() -> str:
+    h = hashlib.sha256()
+    for f in sorted((ROOT / "paper_2607_10611_gb300" / "csrc").glob("*")):
+        h.update(f.read_bytes())
+    return h.hexdigest()[:16]
+
+
+def recorded_traffic(workload: str):
+    """DRAM bytes per launch from the committed ncu summary, if it was taken
+    on the current kernel sources (else None)."""
+    p = ROOT / "profiles" / "traffic.json"
+    if not p.exists():
+        return None
+    d = json.loads(p.read_text())
+    e = d.get(workload)
+    if not e or e.get("kernel_sources_sha256_16") != kernel_source_hash():
+        return None
+    return e.get("dram_bytes_per_launch")
+
+
+# ---------------------------------------------------------------------------
+# clocks
+# ---------------------------------------------------------------------------
+class ClockSampler:
+    FIELDS = ("timestamp,index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int, path: Path):
+        self.path = path
+        self.proc = None
+        try:
+            self.fh = open(path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100", "-i", str(gpu_index)], stdout=self.fh, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+            self.fh.close()
+
+    def summary(self, t0: float, t1: float):
+        if self.proc is None or not self.path.exists():
+            return None
+        rows = []
+        for r in csv.reader(self.path.read_text().splitlines()):
+            if len(r) < 10:
+                continue
+            try:
+                ts = datetime.strptime(r[0].strip(), "%Y/%m/%d %H:%M:%S.%f").timestamp()
+                rows.append((ts, float(r[2]), float(r[3]), [x.strip() for x in r[6:10]]))
+            except ValueError:
+                continue
+        inside = [x for x in rows if t0 - 0.05 <= x[0] <= t1 + 0.05] or rows[-3:]
+        if not inside:
+            return None
+        mhz = sorted(x[1] for x in inside)
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for x in inside for i, v in enumerate(x[3]) if v.lower() == "active"})
+        return {"sm_mhz": mhz[len(mhz) // 2], "sm_max_mhz": max(x[2] for x in inside),
+                "reasons": reasons, "samples": len(inside)}
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle timing (baseline / reference arm)
+# ---------------------------------------------------------------------------
+def oracle_sample(wl, n_elems: int):
+    """The first n_elems elements of the workload's tensor list, drawn on the
+    host (same distributions and formats)."""
+    import workloads as W
+    specs, total = [], 0
+    for s in wl.specs:
+        if total >= n_elems:
+            break
+        take = min(s.numel, n_elems - total)
+        specs.append(W.TensorSpec(s.name, take, s.role))
+        total += take
+    from dataclasses import replace
+    return replace(wl, specs=tuple(specs)), total
+
+
+def host_lists(mt):
+    """Host numpy copies of a CPU-drawn workload for the oracle, and its FP8
+    state before the first step."""
+    import oracle
+    import workloads as W
+    tensors = [dict(w=W.to_numpy_bits(mt.w[k]), g=W.to_numpy_bits(mt.g[k]), m=W.to_numpy_bits(mt.m[k]),
+                    v=W.to_numpy_bits(mt.v[k]), ve=W.to_numpy_bits(mt.ve[k])) for k in range(len(mt.w))]
+    fp8 = oracle.fp8_init(tensors, mt.fp8_exp) if mt.fp8_exp is not None else None
+    return tensors, fp8
+
+
+def time_oracle(wl, target_s: float, t_step: int = 1):
+    """Time the oracle for one step over a sample sized for ~target_s seconds."""
+    import oracle
+    import workloads as W
+    rate = None
+    n = 1 << 18
+    while True:
+        swl, got = oracle_sample(wl, n)
+        mt = W.materialize(swl, "cpu")
+        tensors, fp8 = host_lists(mt)
+        hp = oracle.hparams(stochastic=1 if wl.rounding == "stochastic" else 0, seed=wl.seed)
+        kw = dict(wdt=oracle.DTYPES[wl.weight_dtype], gdt=oracle.DTYPES[wl.grad_dtype],
+                  mdt=oracle.DTYPES[wl.moment_dtype], hp=hp, t=t_step, fp8_state=fp8)
+        t0 = time.perf_counter()
+        oracle.step(tensors, **kw)
+        dt = time.perf_counter() - t0
+        rate = got / dt
+        if dt >= 0.5 * target_s or got < n:
+            return got, dt, rate
+        n = int(min(rate * target_s, 1 << 29))
+
+
+# ---------------------------------------------------------------------------
+# GPU arm
+# ---------------------------------------------------------------------------
+def run_gpu(wl, steps: int, warmup: int, rank: int, e2e_steps: int):
+    import torch
+    import workloads as W
+    from paper_2607_10611_gb300 import build
+    from paper_2607_10611_gb300.optimizer import MPAdam
+
+    build()
+    dev = torch.device("cuda", torch.cuda.current_device())
+    mt = W.materialize(wl, dev, layout="flat")
+    opt = MPAdam(mt.w, mt.m, mt.v, mt.ve, weight_dtype=wl.weight_dtype, grad_dtype=wl.grad_dtype,
+                 moment_dtype=wl.moment_dtype, rounding=wl.rounding, seed=wl.seed + rank,
+                 fp8_exp=mt.fp8_exp)
+    stream = torch.cuda.current_stream(dev)
+    gptrs = [g.data_ptr() for g in mt.g]
+    t = 1
+    for _ in range(warmup):
+        opt.step_ptrs(gptrs, t, stream.cuda_stream)
+        t += 1
+    torch.cuda.synchronize()
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+    region0, region1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if torch.distributed.is_initialized():
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    wall0 = time.time()
+    region0.record(stream)
+    for i in range(steps):
+        starts[i].record(stream)
+        opt.step_ptrs(gptrs, t, stream.cuda_stream)
+        ends[i].record(stream)
+        t += 1
+    region1.record(stream)
+    torch.cuda.synchronize()
+    wall1 = time.time()
+    if torch.distributed.is_initialized():
+        torch.distributed.barrier()
+    total_ms = region0.elapsed_time(region1)
+    launch_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
+    res = {"total_ms": total_ms, "launch_ms": launch_ms, "wall": (wall0, wall1),
+           "grid": opt.launch_info()}
+
+    # end to end through the host-buffer entry point
+    if e2e_steps > 0:
+        hg = torch.empty(mt.flat["g"].shape, dtype=mt.flat["g"].dtype, pin_memory=True)
+        hg.copy_(mt.flat["g"])
+        hw = torch.empty(mt.flat["w"].shape, dtype=mt.flat["w"].dtype, pin_memory=True)
+        hgs = [hg[o:o + x.numel()] for o, x in zip(mt.offsets, mt.g)]
+        hws = [hw[o:o + x.numel()] for o, x in zip(mt.offsets, mt.w)]
+        opt.step_host(hgs, hws, t)  # warm (allocates the staging buffer)
+        t += 1
+        torch.cuda.synchronize()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(e2e_steps):
+            opt.step_host(hgs, hws, t)
+            t += 1
+        e1.record(stream)
+        torch.cuda.synchronize()
+        res["e2e_ms"] = e0.elapsed_time(e1) / e2e_steps
+        res["h2d"] = sum(x.numel() for x in mt.g) * BYTES[wl.grad_dtype]
+        res["d2h"] = sum(x.numel() for x in mt.w) * BYTES[wl.weight_dtype]
+        del hg, hw, hgs, hws
+    opt.close()
+    del mt, opt
+    torch.cuda.synchronize()
+    torch.cuda.empty_cache()
+    return res
+
+
+def summarize(wl, res, n_gpus, peak, peak_kind):
+    n = wl.n_params
+    ms = res["total_ms"] / len(res["launch_ms"])
+    bpp = algorithmic_bytes_per_param(wl)
+    launch = sorted(res["launch_ms"])
+    avg_launch = sum(launch) / len(launch)
+    achieved = bpp * n / (avg_launch * 1e-3) / 1e9
+    out = {
+        "workload": wl.name, "params": n, "tensors": len(wl.specs),
+        "ms_per_step": ms, "gparams_per_s": n_gpus * n / (ms * 1e-3) / 1e9,
+        "hbm_gbs": bpp * n / (ms * 1e-3) / 1e9,
+        "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
+                     "frac": round(achieved / peak, 4), "traffic": recorded_traffic(wl.name),
+                     "peak_source": peak_kind, "bytes_per_param": bpp,
+                     "kernel": "mpadam::step_kernel", "launch_ms_avg": round(avg_launch, 4),
+                     "launch_ms_min": round(launch[0], 4), "launch_ms_max": round(launch[-1], 4)},
+    }
+    if "e2e_ms" in res:
+        out["e2e"] = {"value": n_gpus * n / (res["e2e_ms"] * 1e-3) / 1e9, "unit": UNIT,
+                      "h2d_bytes_per_step": res["h2d"], "d2h_bytes_per_step": res["d2h"],
+                      "ms_per_step": res["e2e_ms"]}
+    return out
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--config", default="llama_7b")
+    ap.add_argument("--secondary", default="llama_1p5b", help="'' to skip")
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    args = ap.parse_args()
+    warmup = max(3, args.warmup)
+
+    import workloads as W
+    wl = W.CONFIGS[args.config]
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+
+    if args.impl == "reference":
+        # the oracle is the reference: rank 0 only, on the host cores
+        if rank != 0:
+            return
+        per_step = []
+        sample_desc = None
+        for i in range(warmup + args.steps):
+            got, dt, rate = time_oracle(wl, target_s=1.0, t_step=1 + i)
+            if i >= warmup:
+                per_step.append((got, dt))
+            sample_desc = f"first {got} elements of the {wl.name} list per step, one step each"
+        elems = sum(g for g, _ in per_step)
+        secs = sum(d for _, d in per_step)
+        value = elems / secs / 1e9
+        line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+                "steps": args.steps, "warmup": warmup, "ms_per_step": 1e3 * wl.n_params / (value * 1e9),
+                "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+                "data": "synthetic",
+                "config": {"workload": wl.name, "params": wl.n_params, "tensors": len(wl.specs)},
+                "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
+                                 "sample": sample_desc},
+                "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+        print(json.dumps(line), flush=True)
+        return
+
+    import torch
+    if world > 1:
+        torch.distributed.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
+        torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", "0")))
+    peak, peak_kind = measured_peaks()
+    out_dir = ROOT / "gpurun_out"
+    out_dir.mkdir(exist_ok=True)
+    gpu_index = int(os.environ.get("LOCAL_RANK", "0"))
+    sampler = ClockSampler(gpu_index, out_dir / f"clocks_rank{rank}.csv") if rank == 0 else None
+    time.sleep(0.3 if sampler else 0)
+
+    res = run_gpu(wl, args.steps, warmup, rank, args.e2e_steps if rank == 0 else 0)
+    total_ms = res["total_ms"]
+    if world > 1:
+        tt = torch.tensor([total_ms], device="cuda")
+        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
+        total_ms = float(tt.item())
+        res["total_ms"] = total_ms
+    clocks = sampler.summary(*res["wall"]) if sampler else None
+    main_sum = summarize(wl, res, world, peak, peak_kind)
+
+    secondary = []
+    if args.secondary and rank == 0 and world == 1:
+        for name in args.secondary.split(","):
+            wl2 = W.CONFIGS[name]
+            r2 = run_gpu(wl2, args.steps, warmup, rank, 0)
+            s2 = summarize(wl2, r2, 1, peak, peak_kind)
+            s2["clocks"] = sampler.summary(*r2["wall"]) if sampler else None
+            secondary.append(s2)
+    if sampler:
+        sampler.stop()
+    if rank != 0:
+        if world > 1:
+            torch.distributed.destroy_process_group()
+        return
+
+    cpu = None
+    if world == 1 or rank == 0:
+        got, dt, rate = time_oracle(wl, target_s=args.cpu_seconds)
+        cpu = {"value": rate / 1e9, "unit": UNIT, "cores": 1, "kind": "oracle",
+               "sample": f"one step over the first {got} elements of the {wl.name} list "
+                         f"({dt:.1f} s, single thread)"}
+
+    ms = main_sum["ms_per_step"]
+    line = {
+        "metric": METRIC, "value": round(main_sum["gparams_per_s"], 3), "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": warmup, "ms_per_step": round(ms, 4), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": {"workload": wl.name, "params": wl.n_params, "tensors": len(wl.specs),
+                   "weights": wl.weight_dtype, "grads": wl.grad_dtype, "moments": wl.moment_dtype,
+                   "rounding": wl.rounding, "l2": "inputs larger than L2 (no flush needed)",
+                   "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
+                   "grid": res["grid"][0], "threads": res["grid"][1]},
+        "hbm_gbs": round(main_sum["hbm_gbs"], 1),
+        "hbm_frac_of_peak": round(main_sum["hbm_gbs"] / peak, 4),
+        "roofline": main_sum["roofline"],
+        "cpu_baseline": cpu,
+        "e2e": main_sum.get("e2e"),
+        "gpu_launches": args.steps,
+        "clocks": clocks,
+        "secondary": secondary,
+    }
+    print(json.dumps(line), flush=True)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

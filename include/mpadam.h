@@ -1,0 +1,207 @@
+/*
+ * mpadam.h -- C ABI of the GB300 (sm_103a) fused M+Adam optimizer step.
+ *
+ * M+Adam (arxiv 2607.10611) updates every parameter w with two branches:
+ *   additive (Algorithm 1, Sec. 4.1):   mu, nu Adam moments with bias
+ *       correction, u_a = -eta_a mu-hat / (sqrt(nu-hat) + eps);
+ *   multiplicative (Algorithm 1, Sec. 4.1): exponent gradient
+ *       g_e = (ln 2) w g, second moment nu_e, proposal
+ *       u~ = -eta_m g_e / (sqrt(nu_e-hat) + eps), rho = max(|w|, tau),
+ *       u_m = clip(u~ / rho);
+ * and combines them as w <- w + w u_m + u_a, then rounds w straight back into
+ * its low-precision storage format (Appendix B's FP32-compute / BF16-storage
+ * round trip; FP8 master weights of Sec. 5.2).  Algorithm 2 (Appendix A) adds
+ * the optional clamp g_max of the normalised exponent gradient, the relative
+ * bounds [-(0.75 - eps0), 0.75], the optional per-step cap |log2(1 + u_m)| <=
+ * d_mult,max, the optional weight clip w_max and decoupled weight decay.
+ *
+ * One mpadam_step() is one fused pass over every element of a tensor list:
+ * each element is read once (w, g, mu, nu, nu_e) and written once (w, mu, nu,
+ * nu_e) by a single kernel launch.
+ *
+ * Arithmetic: IEEE binary32, round-to-nearest-even, with fused multiply-adds
+ * exactly where the canonical sequence below has them; results are
+ * bit-for-bit reproducible for a given (inputs, config, step).  Per element:
+ *   mu'  = fma(b1, mu, (1-b1) g)          nu'  = fma(b2, nu, (1-b2) (g g))
+ *   u_a  = (ka mu') / fma(sqrt(nu'), c2, eps)   [ - (eta_a lambda) w ]
+ *   g_e  = ((ln 2) w) g                   nu_e'= fma(b2, nu_e, (1-b2) (g_e g_e))
+ *   n    = g_e / fma(sqrt(nu_e'), c2, eps)      [ clamped to +-g_max ]
+ *   u_m  = ((-eta_m) n) / max(|w|, tau),  clamped to [lo, hi]
+ *   w'   = fma(w, u_m, w) + u_a                 [ clipped to +-w_max ]
+ * with per-step binary32 scalars computed in binary64 and rounded once:
+ *   ka = -eta_a / (1 - beta1^t), c2 = 1 / sqrt(1 - beta2^t) (both without
+ *   the beta terms when bias_correction = 0), hi = min(rmax_pos, 2^d - 1) and
+ *   lo = max(-rmax_neg, 2^-d - 1) rounded towards zero (d = dmult_max), which
+ *   is the log2/exp2 cap of Algorithm 2 written as the equivalent clamp.
+ * The updated moments are stored from the unrounded binary32 values.
+ *
+ * Storage rounding (the paper cites stochastic rounding but gives no
+ * formula; these are this library's definitions):
+ *   BF16 nearest: round-to-nearest-even; NaN stores 0x7FFF.
+ *   BF16 stochastic: round away from zero iff R16 < (low 16 bits of the
+ *     binary32), R16 the element's 16 random bits (exactly unbiased).
+ *   E4M3 (OCP FP8 "fn": bias 7, largest finite 448, NaN 0x7F): the value is
+ *     first multiplied by 2^-e (per-tensor power-of-two scale); nearest-even
+ *     or stochastic (away iff R32 < floor(fraction * 2^32)); |x| >= 448 and
+ *     infinities saturate to +-448; NaN stores 0x7F.
+ *   Random bits: Philox4x32-10 (Salmon et al., SC'11) with key = seed and
+ *     counter = (block lo, block hi, step lo, step hi).  Global element index
+ *     i draws, for BF16 storage, 16-bit lane i mod 8 of block i div 8 (lane
+ *     L is the low half of word L/2 when L is even, the high half when odd),
+ *     and for E4M3 storage word i mod 4 of block i div 4.
+ *   Global element index: tensor k's element j has index off[k] + j, where
+ *     off[0] = 0 and off[k+1] = off[k] + numel[k] rounded up to a multiple of
+ *     8.  Splitting a tensor at a multiple of 8 therefore changes nothing.
+ *
+ * E4M3 delayed scaling (the paper stores FP8 with scales but does not say
+ * how they are chosen): tensor k's stored weights decode as code * 2^e_t.  A
+ * step re-encodes with e_{t+1} = the smallest integer e with
+ * A_t <= 448 * 2^e (kept at e_t when A_t = 0; clamped to [-100, 100]), where
+ * A_t is the largest finite |w'| the previous step produced (or, before the
+ * first step, the largest |decoded stored weight|), and records A_{t+1}.
+ * The caller owns two device rings that hold this state:
+ *   fp8_exp  : int32[2 n],  e_t of tensor k at fp8_exp[(t mod 2) n + k];
+ *   fp8_amax : uint32[3 n], binary32 bits of A_t at fp8_amax[(t mod 3) n + k].
+ * Step t reads slot t, writes slot t+1 and clears amax slot t+2.
+ *
+ * Conventions for every entry point:
+ *   - returns MPADAM_OK (0) or a positive mpadam_status; never aborts or
+ *     throws across the ABI; mpadam_last_error() then holds a message (per
+ *     host thread);
+ *   - `stream` is a cudaStream_t (NULL = legacy default stream);
+ *   - device pointers are addresses in the current CUDA context's device;
+ *     all tensor memory is owned by the caller; the library owns only the
+ *     metadata it allocates in mpadam_create and frees in mpadam_destroy;
+ *   - calls on one state are not thread-safe and must all be issued to the
+ *     same stream (or ordered by the caller).
+ */
+#ifndef MPADAM_H
+#define MPADAM_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+struct CUstream_st; /* cudaStream_t is `struct CUstream_st *` */
+
+typedef enum {
+  MPADAM_OK = 0,
+  MPADAM_EINVAL = 1,       /* bad argument; nothing was launched */
+  MPADAM_EALLOC = 2,       /* a device or pinned host allocation failed */
+  MPADAM_ECUDA = 3,        /* a CUDA runtime call or launch failed */
+  MPADAM_EUNSUPPORTED = 4  /* valid request this build does not implement */
+} mpadam_status;
+
+typedef enum { MPADAM_F32 = 0, MPADAM_BF16 = 1, MPADAM_E4M3 = 2 } mpadam_dtype;
+typedef enum { MPADAM_ROUND_NEAREST = 0, MPADAM_ROUND_STOCHASTIC = 1 } mpadam_rounding;
+
+/* One parameter tensor (Algorithm 1's state per parameter: w, mu, nu, nu_e),
+ * a contiguous 1-D view of `numel` elements in caller-owned device memory.
+ * w has the config's weight_dtype; m, v, ve its moment_dtype.  Pointers must
+ * be aligned to their element size (may be NULL only when numel == 0).
+ * Tensors whose pointers are all 32-byte aligned take the vectorised path;
+ * others are correct but slower. */
+typedef struct {
+  void* w;
+  void* m;
+  void* v;
+  void* ve;
+  int64_t numel;
+} mpadam_tensor;
+
+/* Hyper-parameters (Algorithm 1 "Inputs", Algorithm 2 options).
+ * Valid ranges (else MPADAM_EINVAL): lr_add, lr_mul >= 0 and finite;
+ * 0 <= beta1, beta2 < 1; eps > 0, tau > 0 finite; rmax_pos > 0 finite;
+ * 0 < rmax_neg < 1; g_max, dmult_max, w_max > 0 (+INFINITY switches the
+ * option off); wd_add >= 0 finite (0 = off). */
+typedef struct {
+  float lr_add;            /* eta_a */
+  float lr_mul;            /* eta_m */
+  float beta1, beta2;
+  float eps;               /* epsilon of both denominators */
+  float tau;               /* rho = max(|w|, tau) */
+  float rmax_pos;          /* u_m <= rmax_pos (Algorithm 2: 0.75) */
+  float rmax_neg;          /* u_m >= -rmax_neg (Algorithm 2: 0.75 - eps0) */
+  float g_max;             /* |n| <= g_max */
+  float dmult_max;         /* |log2(1 + u_m)| <= dmult_max */
+  float w_max;             /* |w'| <= w_max */
+  float wd_add;            /* lambda: u_a -= eta_a lambda w (AdamW-style) */
+  int32_t bias_correction; /* 1: Algorithm 1's mu-hat, nu-hat; 0: Algorithm 2 */
+  int32_t rounding;        /* mpadam_rounding of the weight store */
+  uint64_t seed;           /* Philox key of stochastic rounding */
+  int32_t weight_dtype;    /* MPADAM_BF16 or MPADAM_E4M3 */
+  int32_t grad_dtype;      /* MPADAM_F32 or MPADAM_BF16 */
+  int32_t moment_dtype;    /* MPADAM_F32 or MPADAM_BF16 (stored nearest-even) */
+  int32_t reserved;        /* must be 0 */
+} mpadam_config;
+
+typedef struct mpadam_state mpadam_state;
+
+/* Build the fused step for a tensor list (Algorithm 1 "State").  Copies
+ * `tensors` (the caller may free the array), validates, lays out the global
+ * element index, allocates and uploads device metadata (synchronously, on the
+ * current device).  fp8_exp / fp8_amax: the caller-owned device rings
+ * described above, required for E4M3 weights, NULL otherwise.  n may be 0.
+ * Errors: EINVAL (arguments), EALLOC, ECUDA.  On error *out is NULL. */
+int32_t mpadam_create(const mpadam_tensor* tensors, int32_t n, const mpadam_config* cfg,
+                      int32_t* fp8_exp, uint32_t* fp8_amax, mpadam_state** out);
+
+/* E4M3 only: seed the scale state before `first_step` (t0 >= 1).  Writes
+ * init_exp (host array of n exponents in [-100, 100], the exponents the
+ * stored weights are currently encoded with) into both fp8_exp slots, clears
+ * all fp8_amax slots and writes A_t0 = largest |decoded stored weight| of
+ * each tensor into slot t0 mod 3, on `stream`.  Errors: EINVAL, ECUDA. */
+int32_t mpadam_fp8_init(mpadam_state* s, const int32_t* init_exp, int64_t first_step,
+                        struct CUstream_st* stream);
+
+/* One M+Adam step t (>= 1) over every tensor, asynchronously on `stream`.
+ * grads: host array of n device pointers, grads[k] holding numel[k]
+ * gradients of grad_dtype (read only).  The pointer table is re-uploaded
+ * only when it differs from the previous call's.  The same (inputs, t, seed)
+ * reproduce the same bits, so a resumed run calls with the step it stopped
+ * at.  Errors: EINVAL (t < 1, NULL/misaligned grads), ECUDA (launch). */
+int32_t mpadam_step(mpadam_state* s, const void* const* grads, int64_t step,
+                    struct CUstream_st* stream);
+
+/* The same step with gradients and weights in host memory: copies
+ * host_grads[k] (numel[k] gradients each) to library-owned device staging,
+ * runs mpadam_step, and copies every updated weight tensor back to
+ * host_w_out[k] (numel[k] weights of weight_dtype each), all on `stream`.
+ * For overlap the host buffers should be pinned.  When host_grads[k] (or
+ * host_w_out[k] and the device weights) follow the global-index layout of
+ * one flat buffer, a single copy moves them all.  The first call allocates
+ * the staging buffer.  Errors: EINVAL, EALLOC, ECUDA. */
+int32_t mpadam_step_host(mpadam_state* s, const void* const* host_grads, void* const* host_w_out,
+                         int64_t step, struct CUstream_st* stream);
+
+/* Frees the library's metadata (synchronises the device first).  NULL is a
+ * no-op.  Never touches caller-owned tensors. */
+int32_t mpadam_destroy(mpadam_state* s);
+
+/* Message of the last non-OK status returned on this host thread. */
+const char* mpadam_last_error(void);
+
+/* Layout queries: *offset = global index of tensor k's first element;
+ * *length = total length of the padded global index space. */
+int32_t mpadam_global_offset(const mpadam_state* s, int32_t k, int64_t* offset);
+int32_t mpadam_global_length(const mpadam_state* s, int64_t* length);
+
+/* Launch shape: ctas = number of CTAs of the step kernel (0 restores the
+ * default, one full wave at the kernel's occupancy).  Results do not depend
+ * on it.  mpadam_launch_info reports the current grid and threads per CTA. */
+int32_t mpadam_set_grid(mpadam_state* s, int32_t ctas);
+int32_t mpadam_launch_info(const mpadam_state* s, int32_t* ctas, int32_t* threads);
+
+/* Diagnostics: the random bits the step draws.  Writes into out (device,
+ * uint32[n]) the lane of global element indices first, ..., first + n - 1 at
+ * step `step` for weight storage `weight_dtype` (16-bit lanes for BF16,
+ * 32-bit for E4M3), on `stream`.  Errors: EINVAL, ECUDA. */
+int32_t mpadam_rng_lanes(uint64_t seed, int64_t step, int32_t weight_dtype, int64_t first,
+                         int64_t n, uint32_t* out, struct CUstream_st* stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* MPADAM_H */

@@ -1,0 +1,562 @@
+// mpadam_api.cu -- host side of the C ABI declared in include/mpadam.h, plus
+// the two small auxiliary kernels (E4M3 scale-state seeding, random-lane
+// dump).  The fused step kernel itself lives in step_kernel.cuh.
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <new>
+#include <string>
+#include <vector>
+
+#include "mpadam.h"
+#include "step_args.h"
+#include "step_kernel.cuh"
+
+using mpadam::StepArgs;
+using mpadam::StepScalars;
+using mpadam::TensorDesc;
+
+namespace {
+
+thread_local std::string g_last_error;
+
+int32_t fail(int32_t code, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof buf, fmt, ap);
+  va_end(ap);
+  g_last_error = buf;
+  return code;
+}
+
+int32_t cuda_fail(cudaError_t e, const char* what) {
+  return fail(MPADAM_ECUDA, "%s: %s (%s)", what, cudaGetErrorString(e), cudaGetErrorName(e));
+}
+
+size_t elem_size(int32_t dt) { return dt == MPADAM_F32 ? 4 : (dt == MPADAM_BF16 ? 2 : 1); }
+
+bool is_aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+// Per-step binary32 scalars of the canonical update, from binary64.
+float toward_zero(double x) {
+  float f = static_cast<float>(x);
+  if (x > 0.0 && static_cast<double>(f) > x) f = std::nextafter(f, 0.0f);
+  if (x < 0.0 && static_cast<double>(f) < x) f = std::nextafter(f, 0.0f);
+  return f;
+}
+
+void make_scalars(const mpadam_config& c, int64_t t, StepScalars* s) {
+  double bc1 = 1.0, bc2 = 1.0;
+  if (c.bias_correction) {
+    bc1 = 1.0 - std::pow(static_cast<double>(c.beta1), static_cast<double>(t));
+    bc2 = 1.0 - std::pow(static_cast<double>(c.beta2), static_cast<double>(t));
+  }
+  s->b1 = c.beta1;
+  s->b2 = c.beta2;
+  s->omb1 = static_cast<float>(1.0 - static_cast<double>(c.beta1));
+  s->omb2 = static_cast<float>(1.0 - static_cast<double>(c.beta2));
+  s->ka = static_cast<float>(-static_cast<double>(c.lr_add) / bc1);
+  s->c2 = static_cast<float>(1.0 / std::sqrt(bc2));
+  s->km = -c.lr_mul;
+  s->ln2 = static_cast<float>(0.693147180559945309417232121458);
+  s->eps = c.eps;
+  s->tau = c.tau;
+  const double d = static_cast<double>(c.dmult_max);
+  s->hi = toward_zero(std::fmin(static_cast<double>(c.rmax_pos), std::exp2(d) - 1.0));
+  s->lo = toward_zero(std::fmax(-static_cast<double>(c.rmax_neg), std::exp2(-d) - 1.0));
+  s->gmax_on = std::isfinite(c.g_max) ? 1 : 0;
+  s->gmax = s->gmax_on ? c.g_max : 0.0f;
+  s->wmax_on = std::isfinite(c.w_max) ? 1 : 0;
+  s->wmax = s->wmax_on ? c.w_max : 0.0f;
+  s->wd_on = c.wd_add != 0.0f ? 1 : 0;
+  s->kwd = static_cast<float>(static_cast<double>(c.lr_add) * static_cast<double>(c.wd_add));
+  s->pad = 0;
+}
+
+int32_t check_config(const mpadam_config* c) {
+  if (!c) return fail(MPADAM_EINVAL, "config is NULL");
+  if (c->weight_dtype != MPADAM_BF16 && c->weight_dtype != MPADAM_E4M3)
+    return fail(MPADAM_EINVAL, "weight_dtype must be MPADAM_BF16 or MPADAM_E4M3 (got %d)", c->weight_dtype);
+  if (c->grad_dtype != MPADAM_F32 && c->grad_dtype != MPADAM_BF16)
+    return fail(MPADAM_EINVAL, "grad_dtype must be MPADAM_F32 or MPADAM_BF16 (got %d)", c->grad_dtype);
+  if (c->moment_dtype != MPADAM_F32 && c->moment_dtype != MPADAM_BF16)
+    return fail(MPADAM_EINVAL, "moment_dtype must be MPADAM_F32 or MPADAM_BF16 (got %d)", c->moment_dtype);
+  if (c->rounding != MPADAM_ROUND_NEAREST && c->rounding != MPADAM_ROUND_STOCHASTIC)
+    return fail(MPADAM_EINVAL, "rounding must be nearest (0) or stochastic (1) (got %d)", c->rounding);
+  if (c->bias_correction != 0 && c->bias_correction != 1)
+    return fail(MPADAM_EINVAL, "bias_correction must be 0 or 1");
+  if (c->reserved != 0) return fail(MPADAM_EINVAL, "reserved must be 0");
+  auto fin_nonneg = [](float x) { return std::isfinite(x) && x >= 0.0f; };
+  auto fin_pos = [](float x) { return std::isfinite(x) && x > 0.0f; };
+  if (!fin_nonneg(c->lr_add)) return fail(MPADAM_EINVAL, "lr_add must be finite and >= 0");
+  if (!fin_nonneg(c->lr_mul)) return fail(MPADAM_EINVAL, "lr_mul must be finite and >= 0");
+  if (!(c->beta1 >= 0.0f && c->beta1 < 1.0f)) return fail(MPADAM_EINVAL, "beta1 must be in [0, 1)");
+  if (!(c->beta2 >= 0.0f && c->beta2 < 1.0f)) return fail(MPADAM_EINVAL, "beta2 must be in [0, 1)");
+  if (!fin_pos(c->eps)) return fail(MPADAM_EINVAL, "eps must be finite and > 0");
+  if (!fin_pos(c->tau)) return fail(MPADAM_EINVAL, "tau must be finite and > 0");
+  if (!fin_pos(c->rmax_pos)) return fail(MPADAM_EINVAL, "rmax_pos must be finite and > 0");
+  if (!(fin_pos(c->rmax_neg) && c->rmax_neg < 1.0f)) return fail(MPADAM_EINVAL, "rmax_neg must be in (0, 1)");
+  if (!(c->g_max > 0.0f)) return fail(MPADAM_EINVAL, "g_max must be > 0 (+inf = off)");
+  if (!(c->dmult_max > 0.0f)) return fail(MPADAM_EINVAL, "dmult_max must be > 0 (+inf = off)");
+  if (!(c->w_max > 0.0f)) return fail(MPADAM_EINVAL, "w_max must be > 0 (+inf = off)");
+  if (!fin_nonneg(c->wd_add)) return fail(MPADAM_EINVAL, "wd_add must be finite and >= 0");
+  return MPADAM_OK;
+}
+
+// ---------------------------------------------------------------------------
+// Auxiliary kernels
+// ---------------------------------------------------------------------------
+
+// Largest |decoded stored E4M3 weight| of each tensor -> fp8_amax[slot], over
+// the same per-CTA group ranges as the step kernel.
+__global__ void __launch_bounds__(mpadam::kThreads) fp8_amax_kernel(const __grid_constant__ StepArgs a,
+                                                                    int32_t exp_slot, int32_t amax_slot) {
+  const int64_t G = a.total_groups;
+  const int64_t g_begin = (int64_t)blockIdx.x * G / gridDim.x;
+  const int64_t g_end = ((int64_t)blockIdx.x + 1) * G / gridDim.x;
+  if (g_begin >= g_end) return;
+  const int n = a.n_tensors;
+  for (int k = a.cta_first[blockIdx.x]; k < n; ++k) {
+    const TensorDesc d = a.desc[k];
+    const int64_t t0 = d.goff >> 3;
+    const int64_t t1 = t0 + ((d.numel + 7) >> 3);
+    if (t0 >= g_end) break;
+    const int64_t lo = g_begin > t0 ? g_begin : t0;
+    const int64_t hi = g_end < t1 ? g_end : t1;
+    if (lo >= hi) continue;
+    uint32_t mag = 0;
+    const uint8_t* q = static_cast<const uint8_t*>(d.w);
+    for (int64_t gi = lo + threadIdx.x; gi < hi; gi += mpadam::kThreads) {
+      const int64_t e0 = (gi - t0) * mpadam::kGroup;
+      const int64_t left = d.numel - e0;
+      const int valid = left < mpadam::kGroup ? (int)left : mpadam::kGroup;
+      for (int j = 0; j < valid; ++j) {
+        const uint32_t c = q[e0 + j] & 0x7Fu;
+        if (c != 0x7Fu) mag = max(mag, c);  // E4M3 magnitude order = code order
+      }
+    }
+    const uint32_t wmag = __reduce_max_sync(0xFFFFFFFFu, mag);
+    if ((threadIdx.x & 31) == 0 && wmag != 0u) {
+      const int32_t e = a.fp8_exp[(int64_t)exp_slot * n + k];
+      const float v = __fmul_rn(mpadam::e4m3_value(wmag), mpadam::pow2f(e));
+      atomicMax(&a.fp8_amax[(int64_t)amax_slot * n + k], __float_as_uint(v));
+    }
+  }
+}
+
+__global__ void rng_lanes_kernel(uint32_t k0, uint32_t k1, uint32_t t_lo, uint32_t t_hi, int bf16,
+                                 uint64_t first, int64_t n, uint32_t* out) {
+  for (int64_t k = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; k < n;
+       k += (int64_t)gridDim.x * blockDim.x) {
+    const uint64_t i = first + (uint64_t)k;
+    const uint64_t blk = bf16 ? (i >> 3) : (i >> 2);
+    const uint4 r = mpadam::philox4x32_10((uint32_t)blk, (uint32_t)(blk >> 32), t_lo, t_hi, k0, k1);
+    const uint32_t lane = bf16 ? (uint32_t)(i & 7) : (uint32_t)(i & 3);
+    const uint32_t word_idx = bf16 ? (lane >> 1) : lane;
+    const uint32_t word = word_idx == 0 ? r.x : (word_idx == 1 ? r.y : (word_idx == 2 ? r.z : r.w));
+    out[k] = bf16 ? ((lane & 1) ? (word >> 16) : (word & 0xFFFFu)) : word;
+  }
+}
+
+}  // namespace
+
+// ---------------------------------------------------------------------------
+// State
+// ---------------------------------------------------------------------------
+struct mpadam_state {
+  int32_t n = 0;
+  mpadam_config cfg{};
+  std::vector<int64_t> numel, goff;
+  std::vector<void*> w;
+  int64_t length = 0;  // padded global index space
+  int64_t groups = 0;
+  int device = 0;
+  int sm_count = 0;
+  const void* kernel = nullptr;
+  int32_t default_grid = 0;
+  int32_t grid = 0;
+  TensorDesc* d_desc = nullptr;
+  const void** d_grads = nullptr;
+  int32_t* d_cta_first = nullptr;
+  int32_t cta_cap = 0;
+  const void** h_grads = nullptr;  // pinned staging of the grad pointer table
+  std::vector<const void*> last_grads;
+  bool grads_uploaded = false;
+  cudaEvent_t upload_done = nullptr;
+  bool upload_pending = false;
+  int32_t* fp8_exp = nullptr;
+  uint32_t* fp8_amax = nullptr;
+  char* d_gstage = nullptr;  // mpadam_step_host gradient staging (global-index layout)
+  std::vector<const void*> stage_ptrs;
+};
+
+namespace {
+
+void release(mpadam_state* s) {
+  if (!s) return;
+  if (s->d_desc) cudaFree(s->d_desc);
+  if (s->d_grads) cudaFree(const_cast<void**>(s->d_grads));
+  if (s->d_cta_first) cudaFree(s->d_cta_first);
+  if (s->d_gstage) cudaFree(s->d_gstage);
+  if (s->h_grads) cudaFreeHost(const_cast<void**>(s->h_grads));
+  if (s->upload_done) cudaEventDestroy(s->upload_done);
+  delete s;
+}
+
+// First tensor whose group range ends after each CTA's first group.
+std::vector<int32_t> cta_first_table(const mpadam_state* s, int32_t grid) {
+  std::vector<int32_t> first(grid);
+  int32_t k = 0;
+  for (int32_t b = 0; b < grid; ++b) {
+    const int64_t gb = (int64_t)b * s->groups / grid;
+    while (k < s->n && (s->goff[k] / 8 + (s->numel[k] + 7) / 8) <= gb) ++k;
+    first[b] = k;
+  }
+  return first;
+}
+
+int32_t upload_cta_table(mpadam_state* s, int32_t grid) {
+  if (grid > s->cta_cap) {
+    if (s->d_cta_first) cudaFree(s->d_cta_first);
+    s->d_cta_first = nullptr;
+    s->cta_cap = 0;
+    if (cudaMalloc(&s->d_cta_first, sizeof(int32_t) * grid) != cudaSuccess)
+      return fail(MPADAM_EALLOC, "cudaMalloc of %d CTA entries failed", grid);
+    s->cta_cap = grid;
+  }
+  std::vector<int32_t> first = cta_first_table(s, grid);
+  cudaError_t e = cudaMemcpy(s->d_cta_first, first.data(), sizeof(int32_t) * grid, cudaMemcpyHostToDevice);
+  if (e != cudaSuccess) return cuda_fail(e, "upload of the CTA table");
+  s->grid = grid;
+  return MPADAM_OK;
+}
+
+StepArgs base_args(const mpadam_state* s) {
+  StepArgs a;
+  std::memset(&a, 0, sizeof a);
+  a.desc = s->d_desc;
+  a.grads = s->d_grads;
+  a.cta_first = s->d_cta_first;
+  a.total_groups = s->groups;
+  a.n_tensors = s->n;
+  a.key0 = (uint32_t)s->cfg.seed;
+  a.key1 = (uint32_t)(s->cfg.seed >> 32);
+  a.fp8_exp = s->fp8_exp;
+  a.fp8_amax = s->fp8_amax;
+  return a;
+}
+
+int32_t check_device(const mpadam_state* s) {
+  int dev = -1;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+  if (dev != s->device)
+    return fail(MPADAM_EINVAL, "current device %d differs from the state's device %d", dev, s->device);
+  return MPADAM_OK;
+}
+
+}  // namespace
+
+// ---------------------------------------------------------------------------
+// C ABI
+// ---------------------------------------------------------------------------
+extern "C" {
+
+const char* mpadam_last_error(void) { return g_last_error.c_str(); }
+
+int32_t mpadam_create(const mpadam_tensor* tensors, int32_t n, const mpadam_config* cfg,
+                      int32_t* fp8_exp, uint32_t* fp8_amax, mpadam_state** out) {
+  if (!out) return fail(MPADAM_EINVAL, "out is NULL");
+  *out = nullptr;
+  if (n < 0) return fail(MPADAM_EINVAL, "n must be >= 0 (got %d)", n);
+  if (n > 0 && !tensors) return fail(MPADAM_EINVAL, "tensors is NULL");
+  int32_t rc = check_config(cfg);
+  if (rc) return rc;
+  const size_t wsz = elem_size(cfg->weight_dtype), msz = elem_size(cfg->moment_dtype);
+  if (cfg->weight_dtype == MPADAM_E4M3) {
+    if (!fp8_exp || !fp8_amax) return fail(MPADAM_EINVAL, "E4M3 weights need the fp8_exp and fp8_amax rings");
+    if (!is_aligned(fp8_exp, 4) || !is_aligned(fp8_amax, 4))
+      return fail(MPADAM_EINVAL, "fp8_exp / fp8_amax must be 4-byte aligned");
+  }
+  int64_t off = 0;
+  for (int32_t k = 0; k < n; ++k) {
+    const mpadam_tensor& t = tensors[k];
+    if (t.numel < 0) return fail(MPADAM_EINVAL, "tensor %d: numel < 0", k);
+    if (t.numel > 0) {
+      if (!t.w || !t.m || !t.v || !t.ve) return fail(MPADAM_EINVAL, "tensor %d: NULL pointer", k);
+      if (!is_aligned(t.w, wsz) || !is_aligned(t.m, msz) || !is_aligned(t.v, msz) || !is_aligned(t.ve, msz))
+        return fail(MPADAM_EINVAL, "tensor %d: pointer not aligned to its element size", k);
+    }
+    if (t.numel > (int64_t(1) << 56) || off > (int64_t(1) << 58))
+      return fail(MPADAM_EINVAL, "tensor %d: element index space too large", k);
+    off = (off + t.numel + 7) / 8 * 8;
+  }
+
+  mpadam_state* s = new (std::nothrow) mpadam_state();
+  if (!s) return fail(MPADAM_EALLOC, "host allocation failed");
+  try {
+    s->n = n;
+    s->cfg = *cfg;
+    s->numel.resize(n);
+    s->goff.resize(n);
+    s->w.resize(n);
+    s->last_grads.assign(n, nullptr);
+    std::vector<TensorDesc> desc(n);
+    int64_t o = 0;
+    for (int32_t k = 0; k < n; ++k) {
+      s->numel[k] = tensors[k].numel;
+      s->goff[k] = o;
+      s->w[k] = tensors[k].w;
+      desc[k] = TensorDesc{tensors[k].w, tensors[k].m, tensors[k].v, tensors[k].ve,
+                           tensors[k].numel, o, 0, 0};
+      o = (o + tensors[k].numel + 7) / 8 * 8;
+    }
+    s->length = o;
+    s->groups = o / 8;
+    s->fp8_exp = fp8_exp;
+    s->fp8_amax = fp8_amax;
+    s->kernel = cfg->weight_dtype == MPADAM_BF16
+                    ? mpadam::step_kernel_bf16(cfg->grad_dtype, cfg->moment_dtype, cfg->rounding)
+                    : mpadam::step_kernel_e4m3(cfg->grad_dtype, cfg->moment_dtype, cfg->rounding);
+    if (!s->kernel) { release(s); return fail(MPADAM_EUNSUPPORTED, "no kernel for these formats"); }
+
+    cudaError_t e = cudaGetDevice(&s->device);
+    if (e != cudaSuccess) { release(s); return cuda_fail(e, "cudaGetDevice"); }
+    e = cudaDeviceGetAttribute(&s->sm_count, cudaDevAttrMultiProcessorCount, s->device);
+    if (e != cudaSuccess) { release(s); return cuda_fail(e, "cudaDeviceGetAttribute"); }
+    int per_sm = 0;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, s->kernel, mpadam::kThreads, 0);
+    if (e != cudaSuccess) { release(s); return cuda_fail(e, "occupancy query"); }
+    if (per_sm < 1) { release(s); return fail(MPADAM_ECUDA, "step kernel cannot be resident"); }
+    s->default_grid = per_sm * s->sm_count;
+
+    const size_t nn = n > 0 ? (size_t)n : 1;
+    if (cudaMalloc(&s->d_desc, sizeof(TensorDesc) * nn) != cudaSuccess ||
+        cudaMalloc(reinterpret_cast<void**>(&s->d_grads), sizeof(void*) * nn) != cudaSuccess ||
+        cudaMallocHost(reinterpret_cast<void**>(&s->h_grads), sizeof(void*) * nn) != cudaSuccess) {
+      release(s);
+      return fail(MPADAM_EALLOC, "allocation of the tensor tables failed");
+    }
+    e = cudaEventCreateWithFlags(&s->upload_done, cudaEventDisableTiming);
+    if (e != cudaSuccess) { release(s); return cuda_fail(e, "cudaEventCreate"); }
+    if (n > 0) {
+      e = cudaMemcpy(s->d_desc, desc.data(), sizeof(TensorDesc) * n, cudaMemcpyHostToDevice);
+      if (e != cudaSuccess) { release(s); return cuda_fail(e, "upload of the tensor table"); }
+    }
+    rc = upload_cta_table(s, s->default_grid);
+    if (rc) { release(s); return rc; }
+  } catch (const std::bad_alloc&) {
+    release(s);
+    return fail(MPADAM_EALLOC, "host allocation failed");
+  }
+  *out = s;
+  return MPADAM_OK;
+}
+
+int32_t mpadam_destroy(mpadam_state* s) {
+  if (!s) return MPADAM_OK;
+  release(s);
+  return MPADAM_OK;
+}
+
+int32_t mpadam_global_offset(const mpadam_state* s, int32_t k, int64_t* offset) {
+  if (!s || !offset) return fail(MPADAM_EINVAL, "NULL argument");
+  if (k < 0 || k >= s->n) return fail(MPADAM_EINVAL, "tensor index %d out of range [0, %d)", k, s->n);
+  *offset = s->goff[k];
+  return MPADAM_OK;
+}
+
+int32_t mpadam_global_length(const mpadam_state* s, int64_t* length) {
+  if (!s || !length) return fail(MPADAM_EINVAL, "NULL argument");
+  *length = s->length;
+  return MPADAM_OK;
+}
+
+int32_t mpadam_set_grid(mpadam_state* s, int32_t ctas) {
+  if (!s) return fail(MPADAM_EINVAL, "state is NULL");
+  if (ctas < 0 || ctas > (1 << 20)) return fail(MPADAM_EINVAL, "ctas must be in [0, 2^20]");
+  int32_t rc = check_device(s);
+  if (rc) return rc;
+  cudaError_t e = cudaDeviceSynchronize();  // the old table may be in use
+  if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceSynchronize");
+  return upload_cta_table(s, ctas == 0 ? s->default_grid : ctas);
+}
+
+int32_t mpadam_launch_info(const mpadam_state* s, int32_t* ctas, int32_t* threads) {
+  if (!s || !ctas || !threads) return fail(MPADAM_EINVAL, "NULL argument");
+  *ctas = s->grid;
+  *threads = mpadam::kThreads;
+  return MPADAM_OK;
+}
+
+int32_t mpadam_step(mpadam_state* s, const void* const* grads, int64_t step, cudaStream_t stream) {
+  if (!s) return fail(MPADAM_EINVAL, "state is NULL");
+  if (step < 1) return fail(MPADAM_EINVAL, "step must be >= 1 (got %lld)", (long long)step);
+  if (s->n == 0 || s->groups == 0) return MPADAM_OK;
+  if (!grads) return fail(MPADAM_EINVAL, "grads is NULL");
+  const size_t gsz = elem_size(s->cfg.grad_dtype);
+  for (int32_t k = 0; k < s->n; ++k) {
+    if (s->numel[k] == 0) continue;
+    if (!grads[k]) return fail(MPADAM_EINVAL, "grads[%d] is NULL", k);
+    if (!is_aligned(grads[k], gsz)) return fail(MPADAM_EINVAL, "grads[%d] not aligned to its element size", k);
+  }
+  int32_t rc = check_device(s);
+  if (rc) return rc;
+
+  cudaError_t e;
+  if (!s->grads_uploaded || std::memcmp(s->last_grads.data(), grads, sizeof(void*) * s->n) != 0) {
+    if (s->upload_pending) {  // the pinned table may still be read by the last copy
+      e = cudaEventSynchronize(s->upload_done);
+      if (e != cudaSuccess) return cuda_fail(e, "cudaEventSynchronize");
+    }
+    std::memcpy(s->h_grads, grads, sizeof(void*) * s->n);
+    e = cudaMemcpyAsync(s->d_grads, s->h_grads, sizeof(void*) * s->n, cudaMemcpyHostToDevice, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "upload of the gradient table");
+    e = cudaEventRecord(s->upload_done, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
+    s->upload_pending = true;
+    std::memcpy(s->last_grads.data(), grads, sizeof(void*) * s->n);
+    s->grads_uploaded = true;
+  }
+
+  StepArgs a = base_args(s);
+  make_scalars(s->cfg, step, &a.s);
+  a.t_lo = (uint32_t)(uint64_t)step;
+  a.t_hi = (uint32_t)((uint64_t)step >> 32);
+  a.e_cur_slot = (int32_t)(step % 2);
+  a.e_next_slot = (int32_t)((step + 1) % 2);
+  a.a_cur_slot = (int32_t)(step % 3);
+  a.a_next_slot = (int32_t)((step + 1) % 3);
+  a.a_zero_slot = (int32_t)((step + 2) % 3);
+  void* params[] = {&a};
+  e = cudaLaunchKernel(s->kernel, dim3(s->grid), dim3(mpadam::kThreads), params, 0, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "launch of the step kernel");
+  return MPADAM_OK;
+}
+
+int32_t mpadam_fp8_init(mpadam_state* s, const int32_t* init_exp, int64_t first_step, cudaStream_t stream) {
+  if (!s) return fail(MPADAM_EINVAL, "state is NULL");
+  if (s->cfg.weight_dtype != MPADAM_E4M3) return fail(MPADAM_EINVAL, "fp8_init needs E4M3 weights");
+  if (first_step < 1) return fail(MPADAM_EINVAL, "first_step must be >= 1");
+  if (s->n == 0) return MPADAM_OK;
+  if (!init_exp) return fail(MPADAM_EINVAL, "init_exp is NULL");
+  for (int32_t k = 0; k < s->n; ++k)
+    if (init_exp[k] < -100 || init_exp[k] > 100)
+      return fail(MPADAM_EINVAL, "init_exp[%d] = %d outside [-100, 100]", k, init_exp[k]);
+  int32_t rc = check_device(s);
+  if (rc) return rc;
+  std::vector<int32_t> both(2 * (size_t)s->n);
+  std::copy(init_exp, init_exp + s->n, both.begin());
+  std::copy(init_exp, init_exp + s->n, both.begin() + s->n);
+  cudaError_t e = cudaMemcpyAsync(s->fp8_exp, both.data(), sizeof(int32_t) * both.size(),
+                                  cudaMemcpyHostToDevice, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "upload of the initial exponents");
+  e = cudaStreamSynchronize(stream);  // `both` is pageable and about to go away
+  if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
+  e = cudaMemsetAsync(s->fp8_amax, 0, sizeof(uint32_t) * 3 * (size_t)s->n, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "clearing fp8_amax");
+  if (s->groups == 0) return MPADAM_OK;
+  StepArgs a = base_args(s);
+  int32_t exp_slot = (int32_t)(first_step % 2), amax_slot = (int32_t)(first_step % 3);
+  void* params[] = {&a, &exp_slot, &amax_slot};
+  e = cudaLaunchKernel(reinterpret_cast<const void*>(&fp8_amax_kernel), dim3(s->grid),
+                       dim3(mpadam::kThreads), params, 0, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "launch of the amax kernel");
+  return MPADAM_OK;
+}
+
+int32_t mpadam_rng_lanes(uint64_t seed, int64_t step, int32_t weight_dtype, int64_t first, int64_t n,
+                         uint32_t* out, cudaStream_t stream) {
+  if (step < 0) return fail(MPADAM_EINVAL, "step must be >= 0");
+  if (weight_dtype != MPADAM_BF16 && weight_dtype != MPADAM_E4M3)
+    return fail(MPADAM_EINVAL, "weight_dtype must be MPADAM_BF16 or MPADAM_E4M3");
+  if (first < 0 || n < 0) return fail(MPADAM_EINVAL, "first and n must be >= 0");
+  if (n == 0) return MPADAM_OK;
+  if (!out || !is_aligned(out, 4)) return fail(MPADAM_EINVAL, "out is NULL or misaligned");
+  const int64_t blocks = std::min<int64_t>((n + 255) / 256, 4096);
+  rng_lanes_kernel<<<(unsigned)blocks, 256, 0, stream>>>((uint32_t)seed, (uint32_t)(seed >> 32),
+                                                         (uint32_t)(uint64_t)step,
+                                                         (uint32_t)((uint64_t)step >> 32),
+                                                         weight_dtype == MPADAM_BF16 ? 1 : 0,
+                                                         (uint64_t)first, n, out);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(e, "launch of the rng kernel");
+  return MPADAM_OK;
+}
+
+int32_t mpadam_step_host(mpadam_state* s, const void* const* host_grads, void* const* host_w_out,
+                         int64_t step, cudaStream_t stream) {
+  if (!s) return fail(MPADAM_EINVAL, "state is NULL");
+  if (step < 1) return fail(MPADAM_EINVAL, "step must be >= 1");
+  if (s->n == 0 || s->groups == 0) return MPADAM_OK;
+  if (!host_grads || !host_w_out) return fail(MPADAM_EINVAL, "host_grads / host_w_out is NULL");
+  for (int32_t k = 0; k < s->n; ++k)
+    if (s->numel[k] > 0 && (!host_grads[k] || !host_w_out[k]))
+      return fail(MPADAM_EINVAL, "host buffer %d is NULL", k);
+  int32_t rc = check_device(s);
+  if (rc) return rc;
+  const size_t gsz = elem_size(s->cfg.grad_dtype), wsz = elem_size(s->cfg.weight_dtype);
+  cudaError_t e;
+  if (!s->d_gstage) {
+    if (cudaMalloc(&s->d_gstage, (size_t)s->length * gsz) != cudaSuccess)
+      return fail(MPADAM_EALLOC, "cudaMalloc of %lld bytes of gradient staging failed",
+                  (long long)((size_t)s->length * gsz));
+    s->stage_ptrs.resize(s->n);
+    for (int32_t k = 0; k < s->n; ++k) s->stage_ptrs[k] = s->d_gstage + (size_t)s->goff[k] * gsz;
+  }
+  // Does a set of per-tensor pointers follow one flat buffer in global-index layout?
+  auto flat_base = [&](const void* const* p, size_t esz, const char** base) {
+    const char* b = nullptr;
+    for (int32_t k = 0; k < s->n; ++k) {
+      if (s->numel[k] == 0) continue;
+      const char* c = static_cast<const char*>(p[k]) - (size_t)s->goff[k] * esz;
+      if (!b) b = c;
+      else if (c != b) return false;
+    }
+    *base = b;
+    return b != nullptr;
+  };
+  int32_t first = 0, last = s->n - 1;
+  while (first < s->n && s->numel[first] == 0) ++first;
+  while (last >= 0 && s->numel[last] == 0) --last;
+  if (first > last) return MPADAM_OK;
+  const size_t lo_e = (size_t)s->goff[first], hi_e = (size_t)(s->goff[last] + s->numel[last]);
+
+  const char* hb = nullptr;
+  if (flat_base(host_grads, gsz, &hb)) {
+    e = cudaMemcpyAsync(s->d_gstage + lo_e * gsz, hb + lo_e * gsz, (hi_e - lo_e) * gsz,
+                        cudaMemcpyHostToDevice, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "gradient upload");
+  } else {
+    for (int32_t k = 0; k < s->n; ++k) {
+      if (s->numel[k] == 0) continue;
+      e = cudaMemcpyAsync(const_cast<void*>(s->stage_ptrs[k]), host_grads[k], (size_t)s->numel[k] * gsz,
+                          cudaMemcpyHostToDevice, stream);
+      if (e != cudaSuccess) return cuda_fail(e, "gradient upload");
+    }
+  }
+  rc = mpadam_step(s, s->stage_ptrs.data(), step, stream);
+  if (rc) return rc;
+  const char* dw = nullptr;
+  const char* hw = nullptr;
+  if (flat_base(const_cast<const void* const*>(reinterpret_cast<void* const*>(s->w.data())), wsz, &dw) &&
+      flat_base(const_cast<const void* const*>(host_w_out), wsz, &hw)) {
+    e = cudaMemcpyAsync(const_cast<char*>(hw) + lo_e * wsz, dw + lo_e * wsz, (hi_e - lo_e) * wsz,
+                        cudaMemcpyDeviceToHost, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "weight download");
+  } else {
+    for (int32_t k = 0; k < s->n; ++k) {
+      if (s->numel[k] == 0) continue;
+      e = cudaMemcpyAsync(host_w_out[k], s->w[k], (size_t)s->numel[k] * wsz, cudaMemcpyDeviceToHost, stream);
+      if (e != cudaSuccess) return cuda_fail(e, "weight download");
+    }
+  }
+  return MPADAM_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,143 @@
+"""Shared machinery of the GPU parity tests and the smoke check: run the CUDA
+step (through the C ABI) and the oracle on the same seeded inputs and compare
+every stored bit.
+
+Tolerance: the library and the oracle follow the same binary32 operation
+sequence, so stored weights, moments and E4M3 scale state must agree bit for
+bit (NaN compares equal to NaN).  That is stricter than the bar of the
+method's parity contract (weights within 1 storage ulp on at most 1e-4 of
+elements where rounding is stochastic, binary32 moments within relative
+1e-5); `contract_ok` checks that weaker bar too, for reporting.
+"""
+from __future__ import annotations
+
+import math
+from typing import Dict, List, Optional
+
+import numpy as np
+import torch
+
+import oracle
+import workloads as W
+from paper_2607_10611_gb300.optimizer import MPAdam
+
+ODT = {"f32": oracle.F32, "bf16": oracle.BF16, "e4m3": oracle.E4M3}
+HP_KEYS = ("lr_add", "lr_mul", "beta1", "beta2", "eps", "tau", "rmax_pos", "rmax_neg", "g_max",
+           "dmult_max", "w_max", "wd_add", "bias_correction")
+
+
+def oracle_hparams(wl: W.Workload, hp: Dict):
+    kw = {k: v for k, v in hp.items() if k in HP_KEYS}
+    return oracle.hparams(stochastic=1 if wl.rounding == "stochastic" else 0, seed=wl.seed, **kw)
+
+
+def host_tensors(mt: W.Materialized) -> List[dict]:
+    return [dict(w=W.to_numpy_bits(mt.w[k]), g=W.to_numpy_bits(mt.g[k]), m=W.to_numpy_bits(mt.m[k]),
+                 v=W.to_numpy_bits(mt.v[k]), ve=W.to_numpy_bits(mt.ve[k])) for k in range(len(mt.w))]
+
+
+def device_copy(mt: W.Materialized, layout: str = "separate", misalign: int = 0) -> Dict[str, list]:
+    """Copy a CPU-materialised workload to cuda:0.  misalign > 0 shifts every
+    tensor by that many elements inside a larger allocation (vector path off)."""
+    out = {}
+    for key in ("w", "g", "m", "v", "ve"):
+        src = getattr(mt, key)
+        if layout == "flat" and mt.flat:
+            base = mt.flat[key].to("cuda")
+            out[key] = [base[o:o + t.numel()] for o, t in zip(mt.offsets, src)]
+        elif misalign:
+            views = []
+            for t in src:
+                buf = torch.zeros(t.numel() + misalign, dtype=t.dtype, device="cuda")
+                v = buf[misalign:]
+                v.copy_(t)
+                views.append(v)
+            out[key] = views
+        else:
+            out[key] = [t.to("cuda") for t in src]
+    return out
+
+
+def bits_equal(a: np.ndarray, b: np.ndarray) -> np.ndarray:
+    """Element-wise equality of stored bit patterns, any NaN equal to any NaN."""
+    eq = a.view(a.dtype) == b.view(b.dtype)
+    if a.dtype == np.float32:
+        ua, ub = a.view(np.uint32), b.view(np.uint32)
+        eq = (ua == ub) | (np.isnan(a) & np.isnan(b))
+    return eq
+
+
+def mismatches(got: np.ndarray, want: np.ndarray) -> int:
+    return int((~bits_equal(got, want)).sum())
+
+
+def contract_ok(got_w, want_w, got_m, want_m, wdt: str) -> bool:
+    """The method's parity bar (weaker than bit-exact)."""
+    bad = ~bits_equal(got_w, want_w)
+    if bad.any():
+        if wdt == "bf16":
+            d = np.abs(got_w[bad].astype(np.int64) - want_w[bad].astype(np.int64))
+        else:
+            d = np.abs((got_w[bad] & 0x7F).astype(np.int64) - (want_w[bad] & 0x7F).astype(np.int64))
+        if d.max() > 1 or bad.mean() > 1e-4:
+            return False
+    if got_m.dtype == np.float32:
+        ok = bits_equal(got_m, want_m) | (np.abs(got_m - want_m) <= 1e-5 * np.abs(want_m))
+        return bool(ok.all())
+    return bool(bits_equal(got_m, want_m).all())
+
+
+class Run:
+    """A GPU optimizer and an oracle twin over the same workload."""
+
+    def __init__(self, wl: W.Workload, *, warm: bool = False, layout: str = "separate",
+                 misalign: int = 0, hp: Optional[Dict] = None, mt: Optional[W.Materialized] = None):
+        self.wl = wl
+        self.hp = dict(hp or {})
+        self.mt = mt if mt is not None else W.materialize(wl, "cpu", layout=layout, warm_state=warm)
+        self.host = host_tensors(self.mt)
+        self.dev = device_copy(self.mt, layout, misalign)
+        self.ohp = oracle_hparams(wl, self.hp)
+        gkw = {k: v for k, v in self.hp.items() if k in HP_KEYS}
+        self.opt = MPAdam(self.dev["w"], self.dev["m"], self.dev["v"], self.dev["ve"],
+                          weight_dtype=wl.weight_dtype, grad_dtype=wl.grad_dtype,
+                          moment_dtype=wl.moment_dtype, rounding=wl.rounding, seed=wl.seed,
+                          fp8_exp=self.mt.fp8_exp, **gkw)
+        self.fp8 = oracle.fp8_init(self.host, self.mt.fp8_exp) if wl.weight_dtype == "e4m3" else None
+        self.wdt, self.gdt, self.mdt = ODT[wl.weight_dtype], ODT[wl.grad_dtype], ODT[wl.moment_dtype]
+
+    def step(self, t: int):
+        self.opt.step(self.dev["g"], t)
+        oracle.step(self.host, wdt=self.wdt, gdt=self.gdt, mdt=self.mdt, hp=self.ohp, t=t,
+                    fp8_state=self.fp8)
+        torch.cuda.synchronize()
+
+    def compare(self, t_next: int) -> Dict[str, int]:
+        """Mismatch counts per array (and the E4M3 scale state read for step t_next)."""
+        res = {"w": 0, "m": 0, "v": 0, "ve": 0, "elements": 0, "contract_ok": True}
+        for k in range(len(self.host)):
+            h = self.host[k]
+            res["elements"] += h["w"].size
+            gw = W.to_numpy_bits(self.dev["w"][k])
+            gm = W.to_numpy_bits(self.dev["m"][k])
+            res["w"] += mismatches(gw, h["w"])
+            res["m"] += mismatches(gm, h["m"])
+            res["v"] += mismatches(W.to_numpy_bits(self.dev["v"][k]), h["v"])
+            res["ve"] += mismatches(W.to_numpy_bits(self.dev["ve"][k]), h["ve"])
+            if h["w"].size and not contract_ok(gw, h["w"], gm, h["m"], self.wl.weight_dtype):
+                res["contract_ok"] = False
+        if self.fp8 is not None:
+            exps = self.opt.fp8_exponents(t_next)
+            amax = self.opt.fp8_amax(t_next).cpu().numpy()
+            res["fp8_exp"] = sum(int(e != s[0]) for e, s in zip(exps, self.fp8))
+            res["fp8_amax"] = sum(int(np.float32(a).view(np.uint32) != np.float32(s[1]).view(np.uint32))
+                                  for a, s in zip(amax, self.fp8))
+        return res
+
+    def close(self):
+        self.opt.close()
+
+
+def assert_exact(res: Dict[str, int], what: str = ""):
+    bad = {k: v for k, v in res.items() if k not in ("elements", "contract_ok") and v}
+    assert not bad, f"{what}: mismatching elements {bad} of {res['elements']}"
