@@ -201,6 +201,31 @@ int32_t mpadam_launch_info(const mpadam_state* s, int32_t* ctas, int32_t* thread
 int32_t mpadam_rng_lanes(uint64_t seed, int64_t step, int32_t weight_dtype, int64_t first,
                          int64_t n, uint32_t* out, struct CUstream_st* stream);
 
+/* Allocation-free variant of mpadam_step (the paper has no counterpart: this
+ * is a deployment aid).  It is for callers that must not call cudaMalloc --
+ * for example a runtime whose device memory all belongs to its own caching
+ * allocator or memory pool, or a service that fixes its device-memory budget
+ * at start-up and may not allocate afterwards.  It takes the tensor list and
+ * config of mpadam_create plus the arguments of mpadam_step, keeps no state
+ * object, and calls no cudaMalloc, cudaFree or other allocating routine:
+ * the metadata the step kernel reads (tensor descriptors, gradient pointers,
+ * per-CTA start tensors, 606,208 bytes at most) lives in one file-scope
+ * device array that every GPU loading the library holds until the process
+ * exits.  Limits: at most 8192 tensors (larger lists: MPADAM_EINVAL; use
+ * mpadam_create).  The first call on a device looks up that array's device
+ * address (set-up, once per device, with that device current); make that
+ * first call before any stream capture.  Every call rewrites the array's
+ * tables completely before the step kernel reads them, so calls issued to
+ * one stream follow each other safely, but calls that overlap on the GPU
+ * (different streams, or several host threads without ordering) race on
+ * the shared array.  Results are bit-identical to mpadam_step on the same
+ * inputs.  E4M3 weights use the caller's fp8_exp / fp8_amax rings exactly as
+ * mpadam_step does (seed them with mpadam_fp8_init or equivalent values).
+ * Errors: EINVAL, EUNSUPPORTED, ECUDA. */
+int32_t mpadam_step_noalloc(const mpadam_tensor* tensors, int32_t n, const void* const* grads,
+                            const mpadam_config* cfg, int32_t* fp8_exp, uint32_t* fp8_amax,
+                            int64_t step, struct CUstream_st* stream);
+
 #ifdef __cplusplus
 }
 #endif

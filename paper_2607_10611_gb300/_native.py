@@ -21,7 +21,7 @@ ROUNDING = {"nearest": MPADAM_ROUND_NEAREST, "stochastic": MPADAM_ROUND_STOCHAST
 
 EXPORTED = ["mpadam_create", "mpadam_fp8_init", "mpadam_step", "mpadam_step_host", "mpadam_destroy",
             "mpadam_last_error", "mpadam_global_offset", "mpadam_global_length", "mpadam_set_grid",
-            "mpadam_launch_info", "mpadam_rng_lanes"]
+            "mpadam_launch_info", "mpadam_rng_lanes", "mpadam_step_noalloc"]
 
 
 class MPAdamError(RuntimeError):
@@ -92,6 +92,7 @@ def lib() -> ctypes.CDLL:
             "mpadam_set_grid": [P, i32],
             "mpadam_launch_info": [P, P, P],
             "mpadam_rng_lanes": [u64, i64, i32, i64, i64, P, P],
+            "mpadam_step_noalloc": [P, i32, P, P, P, P, i64, P],
         }
         for name, args in sig.items():
             f = getattr(L, name)
@@ -174,3 +175,13 @@ def mpadam_launch_info(state: int) -> tuple:
 def mpadam_rng_lanes(seed: int, step: int, weight_dtype: int, first: int, n: int, out: int,
                      stream: int = 0) -> None:
     _check(lib().mpadam_rng_lanes(seed, step, weight_dtype, first, n, out, stream or None))
+
+
+def mpadam_step_noalloc(tensors: Sequence[tuple], grads: Sequence[int], cfg: mpadam_config, step: int,
+                        fp8_exp: int = 0, fp8_amax: int = 0, stream: int = 0) -> None:
+    """Allocation-free step: tensors as for mpadam_create, grads as for mpadam_step."""
+    arr = (mpadam_tensor * max(1, len(tensors)))()
+    for i, (w, m, v, ve, n) in enumerate(tensors):
+        arr[i] = mpadam_tensor(w, m, v, ve, n)
+    _check(lib().mpadam_step_noalloc(arr, len(tensors), _ptr_array(grads), ctypes.byref(cfg),
+                                     fp8_exp or None, fp8_amax or None, step, stream or None))

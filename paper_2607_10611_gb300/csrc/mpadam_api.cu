@@ -8,6 +8,7 @@
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
+#include <mutex>
 #include <new>
 #include <string>
 #include <vector>
@@ -560,3 +561,195 @@ int32_t mpadam_step_host(mpadam_state* s, const void* const* host_grads, void* c
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// Allocation-free step (mpadam_step_noalloc)
+//
+// For callers that must not call cudaMalloc -- for example a runtime whose
+// device memory all belongs to its own caching allocator or memory pool, or
+// a service that fixes its device-memory budget at start-up.  The metadata
+// the step kernel reads (tensor descriptors, gradient pointers, per-CTA start
+// tensors) goes into one file-scope device array instead of memory the
+// library allocates.  Every GPU that loads the library holds the array until
+// the process exits.  The tables are written by small kernels that receive
+// them as kernel parameters, so no host staging buffer is needed either.
+// ---------------------------------------------------------------------------
+namespace {
+
+constexpr int32_t kNoAllocMaxTensors = 8192;
+constexpr int32_t kNoAllocMaxCtas = 4096;
+constexpr size_t kNoAllocScratchBytes =
+    sizeof(TensorDesc) * kNoAllocMaxTensors + sizeof(void*) * kNoAllocMaxTensors +
+    sizeof(int32_t) * kNoAllocMaxCtas;  // 606,208 bytes
+
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
+
+constexpr int32_t kFillChunk = 384;  // table entries per fill launch (27.7 KB of parameters)
+
+struct FillTensorArgs {
+  TensorDesc desc[kFillChunk];
+  const void* grads[kFillChunk];
+  TensorDesc* dst_desc;
+  const void** dst_grads;
+  int32_t count;
+};
+
+struct FillCtaArgs {
+  int32_t first[kNoAllocMaxCtas];
+  int32_t* dst;
+  int32_t count;
+};
+
+__global__ void noalloc_fill_tensors(const __grid_constant__ FillTensorArgs a) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < a.count) {
+    a.dst_desc[i] = a.desc[i];
+    a.dst_grads[i] = a.grads[i];
+  }
+}
+
+__global__ void noalloc_fill_ctas(const __grid_constant__ FillCtaArgs a) {
+  for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < a.count; i += gridDim.x * blockDim.x)
+    a.dst[i] = a.first[i];
+}
+
+// Per-device set-up: the scratch array's device address and the SM count.
+constexpr int kNoAllocMaxDevices = 64;
+std::mutex g_noalloc_mutex;
+unsigned char* g_noalloc_ptr[kNoAllocMaxDevices] = {};
+int g_noalloc_sms[kNoAllocMaxDevices] = {};
+
+int32_t noalloc_setup(int dev, unsigned char** scratch, int* sms) {
+  if (dev < 0 || dev >= kNoAllocMaxDevices) return fail(MPADAM_EUNSUPPORTED, "device %d beyond the set-up table", dev);
+  std::lock_guard<std::mutex> lock(g_noalloc_mutex);
+  if (!g_noalloc_ptr[dev]) {
+    void* p = nullptr;
+    cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);  // with `dev` current
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress of the scratch array");
+    int n_sm = 0;
+    e = cudaDeviceGetAttribute(&n_sm, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceGetAttribute");
+    g_noalloc_sms[dev] = n_sm;
+    g_noalloc_ptr[dev] = static_cast<unsigned char*>(p);
+  }
+  *scratch = g_noalloc_ptr[dev];
+  *sms = g_noalloc_sms[dev];
+  return MPADAM_OK;
+}
+
+}  // namespace
+
+extern "C" int32_t mpadam_step_noalloc(const mpadam_tensor* tensors, int32_t n, const void* const* grads,
+                                       const mpadam_config* cfg, int32_t* fp8_exp, uint32_t* fp8_amax,
+                                       int64_t step, cudaStream_t stream) {
+  if (n < 0) return fail(MPADAM_EINVAL, "n must be >= 0 (got %d)", n);
+  if (n > kNoAllocMaxTensors)
+    return fail(MPADAM_EINVAL, "mpadam_step_noalloc takes at most %d tensors (got %d); use mpadam_create",
+                kNoAllocMaxTensors, n);
+  if (n > 0 && (!tensors || !grads)) return fail(MPADAM_EINVAL, "tensors / grads is NULL");
+  if (step < 1) return fail(MPADAM_EINVAL, "step must be >= 1 (got %lld)", (long long)step);
+  int32_t rc = check_config(cfg);
+  if (rc) return rc;
+  const size_t wsz = elem_size(cfg->weight_dtype), msz = elem_size(cfg->moment_dtype),
+               gsz = elem_size(cfg->grad_dtype);
+  if (cfg->weight_dtype == MPADAM_E4M3 && (!fp8_exp || !fp8_amax || !is_aligned(fp8_exp, 4) || !is_aligned(fp8_amax, 4)))
+    return fail(MPADAM_EINVAL, "E4M3 weights need 4-byte aligned fp8_exp and fp8_amax rings");
+  int64_t total = 0;
+  for (int32_t k = 0; k < n; ++k) {
+    const mpadam_tensor& t = tensors[k];
+    if (t.numel < 0) return fail(MPADAM_EINVAL, "tensor %d: numel < 0", k);
+    if (t.numel > 0) {
+      if (!t.w || !t.m || !t.v || !t.ve || !grads[k]) return fail(MPADAM_EINVAL, "tensor %d: NULL pointer", k);
+      if (!is_aligned(t.w, wsz) || !is_aligned(t.m, msz) || !is_aligned(t.v, msz) || !is_aligned(t.ve, msz) ||
+          !is_aligned(grads[k], gsz))
+        return fail(MPADAM_EINVAL, "tensor %d: pointer not aligned to its element size", k);
+    }
+    if (t.numel > (int64_t(1) << 56) || total > (int64_t(1) << 58))
+      return fail(MPADAM_EINVAL, "tensor %d: element index space too large", k);
+    total = (total + t.numel + 7) / 8 * 8;
+  }
+  const int64_t groups = total / 8;
+  if (groups == 0) return MPADAM_OK;
+
+  int dev = -1;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+  unsigned char* scratch = nullptr;
+  int sms = 0;
+  rc = noalloc_setup(dev, &scratch, &sms);
+  if (rc) return rc;
+  const void* kernel = cfg->weight_dtype == MPADAM_BF16
+                           ? mpadam::step_kernel_bf16(cfg->grad_dtype, cfg->moment_dtype, cfg->rounding)
+                           : mpadam::step_kernel_e4m3(cfg->grad_dtype, cfg->moment_dtype, cfg->rounding);
+  if (!kernel) return fail(MPADAM_EUNSUPPORTED, "no kernel for these formats");
+  int per_sm = 0;
+  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, mpadam::kThreads, 0);
+  if (e != cudaSuccess) return cuda_fail(e, "occupancy query");
+  const int32_t grid = std::min<int32_t>(std::max(1, per_sm) * sms, kNoAllocMaxCtas);
+
+  TensorDesc* d_desc = reinterpret_cast<TensorDesc*>(scratch);
+  const void** d_grads = reinterpret_cast<const void**>(scratch + sizeof(TensorDesc) * kNoAllocMaxTensors);
+  int32_t* d_first = reinterpret_cast<int32_t*>(scratch + (sizeof(TensorDesc) + sizeof(void*)) * kNoAllocMaxTensors);
+
+  // tensor and gradient tables, in chunks passed as kernel parameters
+  FillTensorArgs fa;
+  int64_t off = 0;
+  for (int32_t k0 = 0; k0 < n; k0 += kFillChunk) {
+    const int32_t cnt = std::min(kFillChunk, n - k0);
+    for (int32_t i = 0; i < cnt; ++i) {
+      const mpadam_tensor& t = tensors[k0 + i];
+      fa.desc[i] = TensorDesc{t.w, t.m, t.v, t.ve, t.numel, off, 0, 0};
+      fa.grads[i] = grads[k0 + i];
+      off = (off + t.numel + 7) / 8 * 8;
+    }
+    fa.dst_desc = d_desc + k0;
+    fa.dst_grads = d_grads + k0;
+    fa.count = cnt;
+    noalloc_fill_tensors<<<(cnt + 127) / 128, 128, 0, stream>>>(fa);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return cuda_fail(e, "launch of the table fill kernel");
+  }
+  // first tensor of each CTA's group range
+  FillCtaArgs fc;
+  {
+    int32_t k = 0;
+    int64_t goff_k = 0;  // global offset of tensor k
+    for (int32_t b = 0; b < grid; ++b) {
+      const int64_t gb = (int64_t)b * groups / grid;
+      while (k < n && (goff_k / 8 + (tensors[k].numel + 7) / 8) <= gb) {
+        goff_k = (goff_k + tensors[k].numel + 7) / 8 * 8;
+        ++k;
+      }
+      fc.first[b] = k;
+    }
+  }
+  fc.dst = d_first;
+  fc.count = grid;
+  noalloc_fill_ctas<<<(grid + 255) / 256, 256, 0, stream>>>(fc);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return cuda_fail(e, "launch of the CTA table fill kernel");
+
+  StepArgs a;
+  std::memset(&a, 0, sizeof a);
+  a.desc = d_desc;
+  a.grads = d_grads;
+  a.cta_first = d_first;
+  a.total_groups = groups;
+  a.n_tensors = n;
+  a.key0 = (uint32_t)cfg->seed;
+  a.key1 = (uint32_t)(cfg->seed >> 32);
+  a.fp8_exp = fp8_exp;
+  a.fp8_amax = fp8_amax;
+  make_scalars(*cfg, step, &a.s);
+  a.t_lo = (uint32_t)(uint64_t)step;
+  a.t_hi = (uint32_t)((uint64_t)step >> 32);
+  a.e_cur_slot = (int32_t)(step % 2);
+  a.e_next_slot = (int32_t)((step + 1) % 2);
+  a.a_cur_slot = (int32_t)(step % 3);
+  a.a_next_slot = (int32_t)((step + 1) % 3);
+  a.a_zero_slot = (int32_t)((step + 2) % 3);
+  void* params[] = {&a};
+  e = cudaLaunchKernel(kernel, dim3(grid), dim3(mpadam::kThreads), params, 0, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "launch of the step kernel");
+  return MPADAM_OK;
+}
