@@ -282,11 +282,16 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--e2e-steps", type=int, default=3)
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    ap.add_argument("--max-params", type=int, default=0,
+                    help="truncate the list to its first N params (small profiling cases)")
     args = ap.parse_args()
     warmup = max(3, args.warmup)
 
     import workloads as W
     wl = W.CONFIGS[args.config]
+    if args.max_params:
+        wl, got = oracle_sample(wl, args.max_params)
+        wl = W.replace(wl, name=f"{wl.name}[:{got}]")
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
 

@@ -194,6 +194,12 @@ int32_t mpadam_global_length(const mpadam_state* s, int64_t* length);
 int32_t mpadam_set_grid(mpadam_state* s, int32_t ctas);
 int32_t mpadam_launch_info(const mpadam_state* s, int32_t* ctas, int32_t* threads);
 
+/* Device-side status of the steps issued so far: synchronises the device,
+ * returns in *code the error bits the step kernel recorded (0 = none; a
+ * non-zero value means a bounded wait inside the kernel gave up and that
+ * launch's results are incomplete) and clears them.  Errors: EINVAL, ECUDA. */
+int32_t mpadam_device_status(mpadam_state* s, int32_t* code);
+
 /* Diagnostics: the random bits the step draws.  Writes into out (device,
  * uint32[n]) the lane of global element indices first, ..., first + n - 1 at
  * step `step` for weight storage `weight_dtype` (16-bit lanes for BF16,

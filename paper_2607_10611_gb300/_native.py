@@ -21,7 +21,7 @@ ROUNDING = {"nearest": MPADAM_ROUND_NEAREST, "stochastic": MPADAM_ROUND_STOCHAST
 
 EXPORTED = ["mpadam_create", "mpadam_fp8_init", "mpadam_step", "mpadam_step_host", "mpadam_destroy",
             "mpadam_last_error", "mpadam_global_offset", "mpadam_global_length", "mpadam_set_grid",
-            "mpadam_launch_info", "mpadam_rng_lanes", "mpadam_step_noalloc"]
+            "mpadam_launch_info", "mpadam_rng_lanes", "mpadam_step_noalloc", "mpadam_device_status"]
 
 
 class MPAdamError(RuntimeError):
@@ -93,6 +93,7 @@ def lib() -> ctypes.CDLL:
             "mpadam_launch_info": [P, P, P],
             "mpadam_rng_lanes": [u64, i64, i32, i64, i64, P, P],
             "mpadam_step_noalloc": [P, i32, P, P, P, P, i64, P],
+            "mpadam_device_status": [P, P],
         }
         for name, args in sig.items():
             f = getattr(L, name)
@@ -170,6 +171,13 @@ def mpadam_launch_info(state: int) -> tuple:
     c, t = ctypes.c_int32(), ctypes.c_int32()
     _check(lib().mpadam_launch_info(state, ctypes.byref(c), ctypes.byref(t)))
     return c.value, t.value
+
+
+def mpadam_device_status(state: int) -> int:
+    """Synchronises; returns and clears the step kernel's device error bits."""
+    out = ctypes.c_int32()
+    _check(lib().mpadam_device_status(state, ctypes.byref(out)))
+    return out.value
 
 
 def mpadam_rng_lanes(seed: int, step: int, weight_dtype: int, first: int, n: int, out: int,

@@ -1,6 +1,7 @@
 // mpadam_api.cu -- host side of the C ABI declared in include/mpadam.h, plus
-// the two small auxiliary kernels (E4M3 scale-state seeding, random-lane
-// dump).  The fused step kernel itself lives in step_kernel.cuh.
+// the small auxiliary kernels (E4M3 scale-state seeding, random-lane dump,
+// table fills of the allocation-free step).  The fused step kernel itself
+// lives in step_kernel.cuh.
 #include <cuda_runtime.h>
 
 #include <algorithm>
@@ -76,7 +77,30 @@ void make_scalars(const mpadam_config& c, int64_t t, StepScalars* s) {
   s->wmax = s->wmax_on ? c.w_max : 0.0f;
   s->wd_on = c.wd_add != 0.0f ? 1 : 0;
   s->kwd = static_cast<float>(static_cast<double>(c.lr_add) * static_cast<double>(c.wd_add));
-  s->pad = 0;
+  s->cert_ok = (c.eps >= 0x1p-125f && c.tau >= 0x1p-125f) ? 1 : 0;
+}
+
+// Philox4x32-10 round keys: key + r * (0x9E3779B9, 0xBB67AE85), r = 0..9.
+void round_keys(uint64_t seed, uint32_t* rk0, uint32_t* rk1) {
+  uint32_t k0 = (uint32_t)seed, k1 = (uint32_t)(seed >> 32);
+  for (int r = 0; r < mpadam::kPhiloxRounds; ++r) {
+    rk0[r] = k0;
+    rk1[r] = k1;
+    k0 += 0x9E3779B9u;
+    k1 += 0xBB67AE85u;
+  }
+}
+
+// Shared-memory ring of the step kernel: one stage holds one tile of every
+// array (w | g | mu | nu | nu_e); as many stages as fit, 2 to kMaxStages.
+struct Geometry {
+  int32_t stages = 0, stage_bytes = 0, off_g = 0, off_m = 0, off_v = 0, off_ve = 0, dyn_smem = 0;
+};
+
+int32_t make_geometry(const mpadam_config& c, int dev, Geometry* g);
+
+bool kernel_options(const mpadam_config& c) {
+  return std::isfinite(c.g_max) || std::isfinite(c.w_max) || c.wd_add != 0.0f;
 }
 
 int32_t check_config(const mpadam_config* c) {
@@ -109,58 +133,94 @@ int32_t check_config(const mpadam_config* c) {
   return MPADAM_OK;
 }
 
+int32_t make_geometry(const mpadam_config& c, int dev, Geometry* g) {
+  const int32_t rw = mpadam::kTile * (int32_t)elem_size(c.weight_dtype);
+  const int32_t rg = mpadam::kTile * (int32_t)elem_size(c.grad_dtype);
+  const int32_t rm = mpadam::kTile * (int32_t)elem_size(c.moment_dtype);
+  g->off_g = rw;
+  g->off_m = rw + rg;
+  g->off_v = g->off_m + rm;
+  g->off_ve = g->off_v + rm;
+  g->stage_bytes = g->off_ve + rm;
+  int optin = 0;
+  cudaError_t e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceGetAttribute(MaxSharedMemoryPerBlockOptin)");
+  const int32_t budget = optin - 2048;  // static barriers and slack
+  g->stages = std::min<int32_t>(mpadam::kMaxStages, budget / g->stage_bytes);
+  if (g->stages < 2) return fail(MPADAM_EUNSUPPORTED, "device shared memory too small for the step pipeline");
+  g->dyn_smem = g->stages * g->stage_bytes;
+  return MPADAM_OK;
+}
+
 // ---------------------------------------------------------------------------
 // Auxiliary kernels
 // ---------------------------------------------------------------------------
 
 // Largest |decoded stored E4M3 weight| of each tensor -> fp8_amax[slot], over
-// the same per-CTA group ranges as the step kernel.
-__global__ void __launch_bounds__(mpadam::kThreads) fp8_amax_kernel(const __grid_constant__ StepArgs a,
-                                                                    int32_t exp_slot, int32_t amax_slot) {
-  const int64_t G = a.total_groups;
-  const int64_t g_begin = (int64_t)blockIdx.x * G / gridDim.x;
-  const int64_t g_end = ((int64_t)blockIdx.x + 1) * G / gridDim.x;
-  if (g_begin >= g_end) return;
+// the same per-CTA tile ranges as the step kernel (kConsumers threads; thread
+// c reads the 8 codes [8c, 8c + 8) of each tile).
+__global__ void __launch_bounds__(mpadam::kConsumers) fp8_amax_kernel(const __grid_constant__ StepArgs a,
+                                                                      int32_t exp_slot, int32_t amax_slot) {
+  const int64_t T = a.total_tiles;
+  const int64_t tb = (int64_t)blockIdx.x * T / gridDim.x;
+  const int64_t te = ((int64_t)blockIdx.x + 1) * T / gridDim.x;
+  if (tb >= te) return;
   const int n = a.n_tensors;
-  for (int k = a.cta_first[blockIdx.x]; k < n; ++k) {
-    const TensorDesc d = a.desc[k];
-    const int64_t t0 = d.goff >> 3;
-    const int64_t t1 = t0 + ((d.numel + 7) >> 3);
-    if (t0 >= g_end) break;
-    const int64_t lo = g_begin > t0 ? g_begin : t0;
-    const int64_t hi = g_end < t1 ? g_end : t1;
-    if (lo >= hi) continue;
-    uint32_t mag = 0;
+  int k = a.cta_first[blockIdx.x];
+  TensorDesc d = a.desc[k];
+  int64_t tiles = (d.numel + mpadam::kTile - 1) / mpadam::kTile;
+  uint32_t mag = 0;
+  for (int64_t t = tb; t < te; ++t) {
+    if (t >= d.tile_off + tiles) {
+      const uint32_t wmag = __reduce_max_sync(0xFFFFFFFFu, mag);
+      if ((threadIdx.x & 31) == 0 && wmag != 0u) {
+        const int32_t e = a.fp8_exp[(int64_t)exp_slot * n + k];
+        const float v = __fmul_rn(mpadam::e4m3_value(wmag), mpadam::pow2f(e));
+        atomicMax(&a.fp8_amax[(int64_t)amax_slot * n + k], __float_as_uint(v));
+      }
+      mag = 0;
+      do {
+        ++k;
+        d = a.desc[k];
+        tiles = (d.numel + mpadam::kTile - 1) / mpadam::kTile;
+      } while (t >= d.tile_off + tiles);
+    }
+    const int64_t e0 = (t - d.tile_off) * mpadam::kTile + mpadam::kGroup * (int64_t)threadIdx.x;
     const uint8_t* q = static_cast<const uint8_t*>(d.w);
-    for (int64_t gi = lo + threadIdx.x; gi < hi; gi += mpadam::kThreads) {
-      const int64_t e0 = (gi - t0) * mpadam::kGroup;
-      const int64_t left = d.numel - e0;
-      const int valid = left < mpadam::kGroup ? (int)left : mpadam::kGroup;
-      for (int j = 0; j < valid; ++j) {
+    for (int j = 0; j < mpadam::kGroup; ++j) {
+      if (e0 + j < d.numel) {
         const uint32_t c = q[e0 + j] & 0x7Fu;
         if (c != 0x7Fu) mag = max(mag, c);  // E4M3 magnitude order = code order
       }
     }
-    const uint32_t wmag = __reduce_max_sync(0xFFFFFFFFu, mag);
-    if ((threadIdx.x & 31) == 0 && wmag != 0u) {
-      const int32_t e = a.fp8_exp[(int64_t)exp_slot * n + k];
-      const float v = __fmul_rn(mpadam::e4m3_value(wmag), mpadam::pow2f(e));
-      atomicMax(&a.fp8_amax[(int64_t)amax_slot * n + k], __float_as_uint(v));
-    }
+  }
+  const uint32_t wmag = __reduce_max_sync(0xFFFFFFFFu, mag);
+  if ((threadIdx.x & 31) == 0 && wmag != 0u) {
+    const int32_t e = a.fp8_exp[(int64_t)exp_slot * n + k];
+    const float v = __fmul_rn(mpadam::e4m3_value(wmag), mpadam::pow2f(e));
+    atomicMax(&a.fp8_amax[(int64_t)amax_slot * n + k], __float_as_uint(v));
   }
 }
 
-__global__ void rng_lanes_kernel(uint32_t k0, uint32_t k1, uint32_t t_lo, uint32_t t_hi, int bf16,
-                                 uint64_t first, int64_t n, uint32_t* out) {
-  for (int64_t k = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; k < n;
+struct RngArgs {
+  uint32_t rk0[mpadam::kPhiloxRounds], rk1[mpadam::kPhiloxRounds];
+  uint32_t t_lo, t_hi;
+  int32_t bf16;
+  uint64_t first;
+  int64_t n;
+  uint32_t* out;
+};
+
+__global__ void rng_lanes_kernel(const __grid_constant__ RngArgs a) {
+  for (int64_t k = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; k < a.n;
        k += (int64_t)gridDim.x * blockDim.x) {
-    const uint64_t i = first + (uint64_t)k;
-    const uint64_t blk = bf16 ? (i >> 3) : (i >> 2);
-    const uint4 r = mpadam::philox4x32_10((uint32_t)blk, (uint32_t)(blk >> 32), t_lo, t_hi, k0, k1);
-    const uint32_t lane = bf16 ? (uint32_t)(i & 7) : (uint32_t)(i & 3);
-    const uint32_t word_idx = bf16 ? (lane >> 1) : lane;
+    const uint64_t i = a.first + (uint64_t)k;
+    const uint64_t blk = a.bf16 ? (i >> 3) : (i >> 2);
+    const uint4 r = mpadam::philox4x32_10((uint32_t)blk, (uint32_t)(blk >> 32), a.t_lo, a.t_hi, a.rk0, a.rk1);
+    const uint32_t lane = a.bf16 ? (uint32_t)(i & 7) : (uint32_t)(i & 3);
+    const uint32_t word_idx = a.bf16 ? (lane >> 1) : lane;
     const uint32_t word = word_idx == 0 ? r.x : (word_idx == 1 ? r.y : (word_idx == 2 ? r.z : r.w));
-    out[k] = bf16 ? ((lane & 1) ? (word >> 16) : (word & 0xFFFFu)) : word;
+    a.out[k] = a.bf16 ? ((lane & 1) ? (word >> 16) : (word & 0xFFFFu)) : word;
   }
 }
 
@@ -172,19 +232,21 @@ __global__ void rng_lanes_kernel(uint32_t k0, uint32_t k1, uint32_t t_lo, uint32
 struct mpadam_state {
   int32_t n = 0;
   mpadam_config cfg{};
-  std::vector<int64_t> numel, goff;
+  std::vector<int64_t> numel, goff, tile_off;
   std::vector<void*> w;
   int64_t length = 0;  // padded global index space
-  int64_t groups = 0;
+  int64_t tiles = 0;   // total tiles
   int device = 0;
   int sm_count = 0;
   const void* kernel = nullptr;
+  Geometry geo;
   int32_t default_grid = 0;
   int32_t grid = 0;
   TensorDesc* d_desc = nullptr;
   const void** d_grads = nullptr;
   int32_t* d_cta_first = nullptr;
   int32_t cta_cap = 0;
+  int32_t* d_err = nullptr;        // device error bits of the step kernel
   const void** h_grads = nullptr;  // pinned staging of the grad pointer table
   std::vector<const void*> last_grads;
   bool grads_uploaded = false;
@@ -203,22 +265,27 @@ void release(mpadam_state* s) {
   if (s->d_desc) cudaFree(s->d_desc);
   if (s->d_grads) cudaFree(const_cast<void**>(s->d_grads));
   if (s->d_cta_first) cudaFree(s->d_cta_first);
+  if (s->d_err) cudaFree(s->d_err);
   if (s->d_gstage) cudaFree(s->d_gstage);
   if (s->h_grads) cudaFreeHost(const_cast<void**>(s->h_grads));
   if (s->upload_done) cudaEventDestroy(s->upload_done);
   delete s;
 }
 
-// First tensor whose group range ends after each CTA's first group.
-std::vector<int32_t> cta_first_table(const mpadam_state* s, int32_t grid) {
-  std::vector<int32_t> first(grid);
+int64_t tiles_of(int64_t numel) { return (numel + mpadam::kTile - 1) / mpadam::kTile; }
+
+// Tensor holding each CTA's first tile (n when the CTA has no tiles).
+void cta_first_table(const int64_t* numel, int32_t n, int64_t total_tiles, int32_t grid, int32_t* first) {
   int32_t k = 0;
+  int64_t tile_off = 0;
   for (int32_t b = 0; b < grid; ++b) {
-    const int64_t gb = (int64_t)b * s->groups / grid;
-    while (k < s->n && (s->goff[k] / 8 + (s->numel[k] + 7) / 8) <= gb) ++k;
+    const int64_t tb = (int64_t)b * total_tiles / grid;
+    while (k < n && tile_off + tiles_of(numel[k]) <= tb) {
+      tile_off += tiles_of(numel[k]);
+      ++k;
+    }
     first[b] = k;
   }
-  return first;
 }
 
 int32_t upload_cta_table(mpadam_state* s, int32_t grid) {
@@ -230,26 +297,67 @@ int32_t upload_cta_table(mpadam_state* s, int32_t grid) {
       return fail(MPADAM_EALLOC, "cudaMalloc of %d CTA entries failed", grid);
     s->cta_cap = grid;
   }
-  std::vector<int32_t> first = cta_first_table(s, grid);
+  std::vector<int32_t> first(grid);
+  cta_first_table(s->numel.data(), s->n, s->tiles, grid, first.data());
   cudaError_t e = cudaMemcpy(s->d_cta_first, first.data(), sizeof(int32_t) * grid, cudaMemcpyHostToDevice);
   if (e != cudaSuccess) return cuda_fail(e, "upload of the CTA table");
   s->grid = grid;
   return MPADAM_OK;
 }
 
+void fill_common(StepArgs& a, const mpadam_config& cfg, const Geometry& geo, int64_t total_tiles, int32_t n,
+                 int32_t* fp8_exp, uint32_t* fp8_amax) {
+  std::memset(&a, 0, sizeof a);
+  a.total_tiles = total_tiles;
+  a.n_tensors = n;
+  a.stages = geo.stages;
+  a.stage_bytes = geo.stage_bytes;
+  a.off_g = geo.off_g;
+  a.off_m = geo.off_m;
+  a.off_v = geo.off_v;
+  a.off_ve = geo.off_ve;
+  round_keys(cfg.seed, a.rk0, a.rk1);
+  a.fp8_exp = fp8_exp;
+  a.fp8_amax = fp8_amax;
+}
+
+void fill_step(StepArgs& a, const mpadam_config& cfg, int64_t step) {
+  make_scalars(cfg, step, &a.s);
+  a.t_lo = (uint32_t)(uint64_t)step;
+  a.t_hi = (uint32_t)((uint64_t)step >> 32);
+  a.e_cur_slot = (int32_t)(step % 2);
+  a.e_next_slot = (int32_t)((step + 1) % 2);
+  a.a_cur_slot = (int32_t)(step % 3);
+  a.a_next_slot = (int32_t)((step + 1) % 3);
+  a.a_zero_slot = (int32_t)((step + 2) % 3);
+}
+
 StepArgs base_args(const mpadam_state* s) {
   StepArgs a;
-  std::memset(&a, 0, sizeof a);
+  fill_common(a, s->cfg, s->geo, s->tiles, s->n, s->fp8_exp, s->fp8_amax);
   a.desc = s->d_desc;
   a.grads = s->d_grads;
   a.cta_first = s->d_cta_first;
-  a.total_groups = s->groups;
-  a.n_tensors = s->n;
-  a.key0 = (uint32_t)s->cfg.seed;
-  a.key1 = (uint32_t)(s->cfg.seed >> 32);
-  a.fp8_exp = s->fp8_exp;
-  a.fp8_amax = s->fp8_amax;
+  a.err = s->d_err;
   return a;
+}
+
+const void* select_kernel(const mpadam_config& c) {
+  const int opt = kernel_options(c) ? 1 : 0;
+  return c.weight_dtype == MPADAM_BF16 ? mpadam::step_kernel_bf16(c.grad_dtype, c.moment_dtype, c.rounding, opt)
+                                       : mpadam::step_kernel_e4m3(c.grad_dtype, c.moment_dtype, c.rounding, opt);
+}
+
+// Opt the kernel into the ring's shared memory and size one full wave.
+int32_t prepare_kernel(const void* kernel, const Geometry& geo, int sms, int32_t* grid) {
+  cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, geo.dyn_smem);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaFuncSetAttribute(MaxDynamicSharedMemorySize)");
+  int per_sm = 0;
+  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, mpadam::kThreads, geo.dyn_smem);
+  if (e != cudaSuccess) return cuda_fail(e, "occupancy query");
+  if (per_sm < 1) return fail(MPADAM_ECUDA, "step kernel cannot be resident");
+  *grid = per_sm * sms;
+  return MPADAM_OK;
 }
 
 int32_t check_device(const mpadam_state* s) {
@@ -305,44 +413,46 @@ int32_t mpadam_create(const mpadam_tensor* tensors, int32_t n, const mpadam_conf
     s->cfg = *cfg;
     s->numel.resize(n);
     s->goff.resize(n);
+    s->tile_off.resize(n);
     s->w.resize(n);
     s->last_grads.assign(n, nullptr);
     std::vector<TensorDesc> desc(n);
-    int64_t o = 0;
+    int64_t o = 0, to = 0;
     for (int32_t k = 0; k < n; ++k) {
       s->numel[k] = tensors[k].numel;
       s->goff[k] = o;
+      s->tile_off[k] = to;
       s->w[k] = tensors[k].w;
-      desc[k] = TensorDesc{tensors[k].w, tensors[k].m, tensors[k].v, tensors[k].ve,
-                           tensors[k].numel, o, 0, 0};
+      desc[k] = TensorDesc{tensors[k].w, tensors[k].m, tensors[k].v, tensors[k].ve, tensors[k].numel, o, to, 0};
       o = (o + tensors[k].numel + 7) / 8 * 8;
+      to += tiles_of(tensors[k].numel);
     }
     s->length = o;
-    s->groups = o / 8;
+    s->tiles = to;
     s->fp8_exp = fp8_exp;
     s->fp8_amax = fp8_amax;
-    s->kernel = cfg->weight_dtype == MPADAM_BF16
-                    ? mpadam::step_kernel_bf16(cfg->grad_dtype, cfg->moment_dtype, cfg->rounding)
-                    : mpadam::step_kernel_e4m3(cfg->grad_dtype, cfg->moment_dtype, cfg->rounding);
+    s->kernel = select_kernel(*cfg);
     if (!s->kernel) { release(s); return fail(MPADAM_EUNSUPPORTED, "no kernel for these formats"); }
 
     cudaError_t e = cudaGetDevice(&s->device);
     if (e != cudaSuccess) { release(s); return cuda_fail(e, "cudaGetDevice"); }
     e = cudaDeviceGetAttribute(&s->sm_count, cudaDevAttrMultiProcessorCount, s->device);
     if (e != cudaSuccess) { release(s); return cuda_fail(e, "cudaDeviceGetAttribute"); }
-    int per_sm = 0;
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, s->kernel, mpadam::kThreads, 0);
-    if (e != cudaSuccess) { release(s); return cuda_fail(e, "occupancy query"); }
-    if (per_sm < 1) { release(s); return fail(MPADAM_ECUDA, "step kernel cannot be resident"); }
-    s->default_grid = per_sm * s->sm_count;
+    rc = make_geometry(*cfg, s->device, &s->geo);
+    if (rc) { release(s); return rc; }
+    rc = prepare_kernel(s->kernel, s->geo, s->sm_count, &s->default_grid);
+    if (rc) { release(s); return rc; }
 
     const size_t nn = n > 0 ? (size_t)n : 1;
     if (cudaMalloc(&s->d_desc, sizeof(TensorDesc) * nn) != cudaSuccess ||
         cudaMalloc(reinterpret_cast<void**>(&s->d_grads), sizeof(void*) * nn) != cudaSuccess ||
+        cudaMalloc(&s->d_err, sizeof(int32_t)) != cudaSuccess ||
         cudaMallocHost(reinterpret_cast<void**>(&s->h_grads), sizeof(void*) * nn) != cudaSuccess) {
       release(s);
       return fail(MPADAM_EALLOC, "allocation of the tensor tables failed");
     }
+    e = cudaMemset(s->d_err, 0, sizeof(int32_t));
+    if (e != cudaSuccess) { release(s); return cuda_fail(e, "clearing the error word"); }
     e = cudaEventCreateWithFlags(&s->upload_done, cudaEventDisableTiming);
     if (e != cudaSuccess) { release(s); return cuda_fail(e, "cudaEventCreate"); }
     if (n > 0) {
@@ -395,10 +505,23 @@ int32_t mpadam_launch_info(const mpadam_state* s, int32_t* ctas, int32_t* thread
   return MPADAM_OK;
 }
 
+int32_t mpadam_device_status(mpadam_state* s, int32_t* code) {
+  if (!s || !code) return fail(MPADAM_EINVAL, "NULL argument");
+  int32_t rc = check_device(s);
+  if (rc) return rc;
+  cudaError_t e = cudaDeviceSynchronize();
+  if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceSynchronize");
+  e = cudaMemcpy(code, s->d_err, sizeof(int32_t), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail(e, "reading the error word");
+  e = cudaMemset(s->d_err, 0, sizeof(int32_t));
+  if (e != cudaSuccess) return cuda_fail(e, "clearing the error word");
+  return MPADAM_OK;
+}
+
 int32_t mpadam_step(mpadam_state* s, const void* const* grads, int64_t step, cudaStream_t stream) {
   if (!s) return fail(MPADAM_EINVAL, "state is NULL");
   if (step < 1) return fail(MPADAM_EINVAL, "step must be >= 1 (got %lld)", (long long)step);
-  if (s->n == 0 || s->groups == 0) return MPADAM_OK;
+  if (s->n == 0 || s->tiles == 0) return MPADAM_OK;
   if (!grads) return fail(MPADAM_EINVAL, "grads is NULL");
   const size_t gsz = elem_size(s->cfg.grad_dtype);
   for (int32_t k = 0; k < s->n; ++k) {
@@ -426,16 +549,9 @@ int32_t mpadam_step(mpadam_state* s, const void* const* grads, int64_t step, cud
   }
 
   StepArgs a = base_args(s);
-  make_scalars(s->cfg, step, &a.s);
-  a.t_lo = (uint32_t)(uint64_t)step;
-  a.t_hi = (uint32_t)((uint64_t)step >> 32);
-  a.e_cur_slot = (int32_t)(step % 2);
-  a.e_next_slot = (int32_t)((step + 1) % 2);
-  a.a_cur_slot = (int32_t)(step % 3);
-  a.a_next_slot = (int32_t)((step + 1) % 3);
-  a.a_zero_slot = (int32_t)((step + 2) % 3);
+  fill_step(a, s->cfg, step);
   void* params[] = {&a};
-  e = cudaLaunchKernel(s->kernel, dim3(s->grid), dim3(mpadam::kThreads), params, 0, stream);
+  e = cudaLaunchKernel(s->kernel, dim3(s->grid), dim3(mpadam::kThreads), params, (size_t)s->geo.dyn_smem, stream);
   if (e != cudaSuccess) return cuda_fail(e, "launch of the step kernel");
   return MPADAM_OK;
 }
@@ -461,12 +577,12 @@ int32_t mpadam_fp8_init(mpadam_state* s, const int32_t* init_exp, int64_t first_
   if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
   e = cudaMemsetAsync(s->fp8_amax, 0, sizeof(uint32_t) * 3 * (size_t)s->n, stream);
   if (e != cudaSuccess) return cuda_fail(e, "clearing fp8_amax");
-  if (s->groups == 0) return MPADAM_OK;
+  if (s->tiles == 0) return MPADAM_OK;
   StepArgs a = base_args(s);
   int32_t exp_slot = (int32_t)(first_step % 2), amax_slot = (int32_t)(first_step % 3);
   void* params[] = {&a, &exp_slot, &amax_slot};
-  e = cudaLaunchKernel(reinterpret_cast<const void*>(&fp8_amax_kernel), dim3(s->grid),
-                       dim3(mpadam::kThreads), params, 0, stream);
+  e = cudaLaunchKernel(reinterpret_cast<const void*>(&fp8_amax_kernel), dim3(s->grid), dim3(mpadam::kConsumers),
+                       params, 0, stream);
   if (e != cudaSuccess) return cuda_fail(e, "launch of the amax kernel");
   return MPADAM_OK;
 }
@@ -479,12 +595,16 @@ int32_t mpadam_rng_lanes(uint64_t seed, int64_t step, int32_t weight_dtype, int6
   if (first < 0 || n < 0) return fail(MPADAM_EINVAL, "first and n must be >= 0");
   if (n == 0) return MPADAM_OK;
   if (!out || !is_aligned(out, 4)) return fail(MPADAM_EINVAL, "out is NULL or misaligned");
+  RngArgs a;
+  round_keys(seed, a.rk0, a.rk1);
+  a.t_lo = (uint32_t)(uint64_t)step;
+  a.t_hi = (uint32_t)((uint64_t)step >> 32);
+  a.bf16 = weight_dtype == MPADAM_BF16 ? 1 : 0;
+  a.first = (uint64_t)first;
+  a.n = n;
+  a.out = out;
   const int64_t blocks = std::min<int64_t>((n + 255) / 256, 4096);
-  rng_lanes_kernel<<<(unsigned)blocks, 256, 0, stream>>>((uint32_t)seed, (uint32_t)(seed >> 32),
-                                                         (uint32_t)(uint64_t)step,
-                                                         (uint32_t)((uint64_t)step >> 32),
-                                                         weight_dtype == MPADAM_BF16 ? 1 : 0,
-                                                         (uint64_t)first, n, out);
+  rng_lanes_kernel<<<(unsigned)blocks, 256, 0, stream>>>(a);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return cuda_fail(e, "launch of the rng kernel");
   return MPADAM_OK;
@@ -494,7 +614,7 @@ int32_t mpadam_step_host(mpadam_state* s, const void* const* host_grads, void* c
                          int64_t step, cudaStream_t stream) {
   if (!s) return fail(MPADAM_EINVAL, "state is NULL");
   if (step < 1) return fail(MPADAM_EINVAL, "step must be >= 1");
-  if (s->n == 0 || s->groups == 0) return MPADAM_OK;
+  if (s->n == 0 || s->tiles == 0) return MPADAM_OK;
   if (!host_grads || !host_w_out) return fail(MPADAM_EINVAL, "host_grads / host_w_out is NULL");
   for (int32_t k = 0; k < s->n; ++k)
     if (s->numel[k] > 0 && (!host_grads[k] || !host_w_out[k]))
@@ -654,7 +774,7 @@ extern "C" int32_t mpadam_step_noalloc(const mpadam_tensor* tensors, int32_t n, 
                gsz = elem_size(cfg->grad_dtype);
   if (cfg->weight_dtype == MPADAM_E4M3 && (!fp8_exp || !fp8_amax || !is_aligned(fp8_exp, 4) || !is_aligned(fp8_amax, 4)))
     return fail(MPADAM_EINVAL, "E4M3 weights need 4-byte aligned fp8_exp and fp8_amax rings");
-  int64_t total = 0;
+  int64_t total = 0, total_tiles = 0;
   for (int32_t k = 0; k < n; ++k) {
     const mpadam_tensor& t = tensors[k];
     if (t.numel < 0) return fail(MPADAM_EINVAL, "tensor %d: numel < 0", k);
@@ -667,9 +787,9 @@ extern "C" int32_t mpadam_step_noalloc(const mpadam_tensor* tensors, int32_t n, 
     if (t.numel > (int64_t(1) << 56) || total > (int64_t(1) << 58))
       return fail(MPADAM_EINVAL, "tensor %d: element index space too large", k);
     total = (total + t.numel + 7) / 8 * 8;
+    total_tiles += tiles_of(t.numel);
   }
-  const int64_t groups = total / 8;
-  if (groups == 0) return MPADAM_OK;
+  if (total_tiles == 0) return MPADAM_OK;
 
   int dev = -1;
   cudaError_t e = cudaGetDevice(&dev);
@@ -678,14 +798,15 @@ extern "C" int32_t mpadam_step_noalloc(const mpadam_tensor* tensors, int32_t n, 
   int sms = 0;
   rc = noalloc_setup(dev, &scratch, &sms);
   if (rc) return rc;
-  const void* kernel = cfg->weight_dtype == MPADAM_BF16
-                           ? mpadam::step_kernel_bf16(cfg->grad_dtype, cfg->moment_dtype, cfg->rounding)
-                           : mpadam::step_kernel_e4m3(cfg->grad_dtype, cfg->moment_dtype, cfg->rounding);
+  const void* kernel = select_kernel(*cfg);
   if (!kernel) return fail(MPADAM_EUNSUPPORTED, "no kernel for these formats");
-  int per_sm = 0;
-  e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, mpadam::kThreads, 0);
-  if (e != cudaSuccess) return cuda_fail(e, "occupancy query");
-  const int32_t grid = std::min<int32_t>(std::max(1, per_sm) * sms, kNoAllocMaxCtas);
+  Geometry geo;
+  rc = make_geometry(*cfg, dev, &geo);
+  if (rc) return rc;
+  int32_t grid = 0;
+  rc = prepare_kernel(kernel, geo, sms, &grid);
+  if (rc) return rc;
+  grid = std::min(grid, kNoAllocMaxCtas);
 
   TensorDesc* d_desc = reinterpret_cast<TensorDesc*>(scratch);
   const void** d_grads = reinterpret_cast<const void**>(scratch + sizeof(TensorDesc) * kNoAllocMaxTensors);
@@ -693,14 +814,15 @@ extern "C" int32_t mpadam_step_noalloc(const mpadam_tensor* tensors, int32_t n, 
 
   // tensor and gradient tables, in chunks passed as kernel parameters
   FillTensorArgs fa;
-  int64_t off = 0;
+  int64_t off = 0, toff = 0;
   for (int32_t k0 = 0; k0 < n; k0 += kFillChunk) {
     const int32_t cnt = std::min(kFillChunk, n - k0);
     for (int32_t i = 0; i < cnt; ++i) {
       const mpadam_tensor& t = tensors[k0 + i];
-      fa.desc[i] = TensorDesc{t.w, t.m, t.v, t.ve, t.numel, off, 0, 0};
+      fa.desc[i] = TensorDesc{t.w, t.m, t.v, t.ve, t.numel, off, toff, 0};
       fa.grads[i] = grads[k0 + i];
       off = (off + t.numel + 7) / 8 * 8;
+      toff += tiles_of(t.numel);
     }
     fa.dst_desc = d_desc + k0;
     fa.dst_grads = d_grads + k0;
@@ -709,15 +831,15 @@ extern "C" int32_t mpadam_step_noalloc(const mpadam_tensor* tensors, int32_t n, 
     e = cudaGetLastError();
     if (e != cudaSuccess) return cuda_fail(e, "launch of the table fill kernel");
   }
-  // first tensor of each CTA's group range
+  // tensor holding each CTA's first tile
   FillCtaArgs fc;
   {
     int32_t k = 0;
-    int64_t goff_k = 0;  // global offset of tensor k
+    int64_t tile_off = 0;
     for (int32_t b = 0; b < grid; ++b) {
-      const int64_t gb = (int64_t)b * groups / grid;
-      while (k < n && (goff_k / 8 + (tensors[k].numel + 7) / 8) <= gb) {
-        goff_k = (goff_k + tensors[k].numel + 7) / 8 * 8;
+      const int64_t tb = (int64_t)b * total_tiles / grid;
+      while (k < n && tile_off + tiles_of(tensors[k].numel) <= tb) {
+        tile_off += tiles_of(tensors[k].numel);
         ++k;
       }
       fc.first[b] = k;
@@ -730,26 +852,14 @@ extern "C" int32_t mpadam_step_noalloc(const mpadam_tensor* tensors, int32_t n, 
   if (e != cudaSuccess) return cuda_fail(e, "launch of the CTA table fill kernel");
 
   StepArgs a;
-  std::memset(&a, 0, sizeof a);
+  fill_common(a, *cfg, geo, total_tiles, n, fp8_exp, fp8_amax);
   a.desc = d_desc;
   a.grads = d_grads;
   a.cta_first = d_first;
-  a.total_groups = groups;
-  a.n_tensors = n;
-  a.key0 = (uint32_t)cfg->seed;
-  a.key1 = (uint32_t)(cfg->seed >> 32);
-  a.fp8_exp = fp8_exp;
-  a.fp8_amax = fp8_amax;
-  make_scalars(*cfg, step, &a.s);
-  a.t_lo = (uint32_t)(uint64_t)step;
-  a.t_hi = (uint32_t)((uint64_t)step >> 32);
-  a.e_cur_slot = (int32_t)(step % 2);
-  a.e_next_slot = (int32_t)((step + 1) % 2);
-  a.a_cur_slot = (int32_t)(step % 3);
-  a.a_next_slot = (int32_t)((step + 1) % 3);
-  a.a_zero_slot = (int32_t)((step + 2) % 3);
+  a.err = nullptr;
+  fill_step(a, *cfg, step);
   void* params[] = {&a};
-  e = cudaLaunchKernel(kernel, dim3(grid), dim3(mpadam::kThreads), params, 0, stream);
+  e = cudaLaunchKernel(kernel, dim3(grid), dim3(mpadam::kThreads), params, (size_t)geo.dyn_smem, stream);
   if (e != cudaSuccess) return cuda_fail(e, "launch of the step kernel");
   return MPADAM_OK;
 }

@@ -1,17 +1,31 @@
 // step_kernel.cuh -- the fused M+Adam step kernel for sm_103a (GB300).
 //
-// One launch = one pass over every element: each thread takes groups of 8
-// consecutive elements, loads w, g, mu, nu, nu_e with one coalesced vector
-// load per array (256-bit for binary32 arrays, 128-bit for BF16, 64-bit for
-// E4M3 weights), runs the canonical binary32 update (Algorithm 1 with the
-// Algorithm 2 options, arxiv 2607.10611), rounds w into its storage format
-// (nearest-even or Philox-keyed stochastic rounding) and stores everything
-// back with one vector store per array.  The path is HBM-bound streaming:
-// no shared-memory staging, no tensor cores (nothing here is a contraction).
+// One launch = one pass over every element of the tensor list.  Each CTA
+// (one per SM) is a producer/consumer pipeline over its range of tiles:
+//   - one producer warp (one elected lane) streams each tile's slice of every
+//     array -- weights w, gradients g and the moments mu, nu, nu_e, each one
+//     contiguous run of bytes -- into a multi-stage shared-memory ring with
+//     1-D TMA bulk copies (cp.async.bulk ... mbarrier::complete_tx), evict-
+//     first in L2 since every byte is used once;
+//   - fifteen consumer warps wait on the stage's mbarrier, read their 8
+//     elements from shared memory, run the canonical binary32 update
+//     (Algorithm 1 with the Algorithm 2 options, arxiv 2607.10611), round the
+//     weight into its storage format (nearest-even, or stochastic with
+//     Philox4x32-10 bits) and store w, mu, nu, nu_e straight back to HBM with
+//     vector stores (256-bit for binary32 arrays), then release the stage.
+// Memory latency is hidden by the ring, not by occupancy, so the consumers'
+// instruction stream is the only other limit.  Tensor tails that are not a
+// whole number of 16-byte chunks, and tensors whose pointers are not 16-byte
+// aligned, are read by the consumers directly from global memory with the
+// same arithmetic.  No tensor cores: nothing here is a contraction.
 //
 // Numerics: every floating-point operation is an explicit round-to-nearest
-// intrinsic (__fmul_rn, __fadd_rn, __fmaf_rn, __fdiv_rn, __fsqrt_rn), so the
-// build flags cannot contract or approximate anything.
+// intrinsic (__fmul_rn, __fadd_rn, __fmaf_rn, __fdiv_rn, __fsqrt_rn), so build
+// flags cannot contract or approximate anything.
+//
+// Every wait on an mbarrier is bounded; a wait that gives up sets a bit in
+// *err, the producer waits (again bounded) for its own copies in flight, and
+// the CTA returns.
 #pragma once
 
 #include <cstdint>
@@ -21,10 +35,10 @@
 
 namespace mpadam {
 
+constexpr uint32_t kSpinLimit = 1u << 22;  // mbarrier try_wait attempts before giving up (seconds)
+
 // ---------------------------------------------------------------------------
-// Global memory access: streaming vector loads/stores (no L1 allocation; each
-// byte is touched exactly once).  Gradients are read-only for the whole
-// launch and use the non-coherent path.
+// Global memory: streaming vector loads/stores (no L1 allocation).
 // ---------------------------------------------------------------------------
 __device__ __forceinline__ void ld8(const void* p, uint32_t (&r)[8]) {
   asm("ld.global.L1::no_allocate.v8.u32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
@@ -72,25 +86,84 @@ __device__ __forceinline__ void st2(void* p, const uint32_t (&r)[2]) {
 }
 
 // ---------------------------------------------------------------------------
-// Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11): ten rounds; each round
-// takes the 64-bit products of words 0 and 2 with the two multipliers, feeds
-// the high halves (xored with words 3 / 1 and the round key) to the other
-// lane and the low halves straight through; the key steps by the Weyl pair.
+// Shared memory, mbarriers and the TMA bulk copy
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t smem_addr(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ void lds4(uint32_t addr, uint32_t (&r)[4]) {
+  asm volatile("ld.shared.v4.u32 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(addr));
+}
+__device__ __forceinline__ void lds2(uint32_t addr, uint32_t (&r)[2]) {
+  asm volatile("ld.shared.v2.u32 {%0,%1}, [%2];" : "=r"(r[0]), "=r"(r[1]) : "r"(addr));
+}
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_init_fence() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.release.cta.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.release.cta.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+               : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.acquire.cta.shared::cta.b64 p, [%1], %2;\n"
+      " selp.u32 %0, 1, 0, p;\n}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+// Wait until the phase with the given parity has completed; false after
+// kSpinLimit attempts.
+__device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity) {
+  for (uint32_t i = 0; i < kSpinLimit; ++i)
+    if (mbar_try_wait(bar, parity)) return true;
+  return false;
+}
+__device__ __forceinline__ uint64_t evict_first_policy() {
+  uint64_t pol;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(pol));
+  return pol;
+}
+// 1-D bulk copy global -> shared, completing `bytes` of transaction on `bar`.
+// Source and destination 16-byte aligned, bytes a multiple of 16.
+__device__ __forceinline__ void tma_load(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar,
+                                         uint64_t pol) {
+  asm volatile(
+      "cp.async.bulk.shared::cta.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], %4;" ::"r"(dst),
+      "l"(src), "r"(bytes), "r"(bar), "l"(pol)
+      : "memory");
+}
+
+// ---------------------------------------------------------------------------
+// Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11) with precomputed round
+// keys rk[r] = key + r * (Weyl constants): each round takes the 64-bit
+// products of words 0 and 2 with the two multipliers, feeds the high halves
+// (xored with words 3 / 1 and the round key) across and the low halves
+// straight through.
 // ---------------------------------------------------------------------------
 __device__ __forceinline__ uint4 philox4x32_10(uint32_t x0, uint32_t x1, uint32_t x2, uint32_t x3,
-                                               uint32_t k0, uint32_t k1) {
+                                               const uint32_t (&rk0)[kPhiloxRounds],
+                                               const uint32_t (&rk1)[kPhiloxRounds]) {
 #pragma unroll
-  for (int r = 0; r < 10; ++r) {
-    const uint32_t a_lo = 0xD2511F53u * x0;
-    const uint32_t a_hi = __umulhi(0xD2511F53u, x0);
-    const uint32_t b_lo = 0xCD9E8D57u * x2;
-    const uint32_t b_hi = __umulhi(0xCD9E8D57u, x2);
-    x0 = b_hi ^ x1 ^ k0;
-    x1 = b_lo;
-    x2 = a_hi ^ x3 ^ k1;
-    x3 = a_lo;
-    k0 += 0x9E3779B9u;
-    k1 += 0xBB67AE85u;
+  for (int r = 0; r < kPhiloxRounds; ++r) {
+    const uint64_t pa = static_cast<uint64_t>(x0) * 0xD2511F53u;
+    const uint64_t pb = static_cast<uint64_t>(x2) * 0xCD9E8D57u;
+    const uint32_t y0 = static_cast<uint32_t>(pb >> 32) ^ x1 ^ rk0[r];
+    const uint32_t y2 = static_cast<uint32_t>(pa >> 32) ^ x3 ^ rk1[r];
+    x1 = static_cast<uint32_t>(pb);
+    x3 = static_cast<uint32_t>(pa);
+    x0 = y0;
+    x2 = y2;
   }
   return make_uint4(x0, x1, x2, x3);
 }
@@ -102,26 +175,99 @@ struct Upd {
   float wn, m, v, ve;
 };
 
-__device__ __forceinline__ Upd madam_update(const StepScalars& s, float w, float g, float m,
-                                            float v, float ve) {
+template <bool OPT>
+__device__ __forceinline__ Upd madam_update(const StepScalars& s, float w, float g, float m, float v,
+                                            float ve) {
   Upd o;
   // additive branch (Adam moments, bias correction folded into ka and c2)
   o.m = __fmaf_rn(s.b1, m, __fmul_rn(s.omb1, g));
   o.v = __fmaf_rn(s.b2, v, __fmul_rn(s.omb2, __fmul_rn(g, g)));
   float ua = __fdiv_rn(__fmul_rn(s.ka, o.m), __fmaf_rn(__fsqrt_rn(o.v), s.c2, s.eps));
-  if (s.wd_on) ua = __fsub_rn(ua, __fmul_rn(s.kwd, w));
+  if (OPT && s.wd_on) ua = __fsub_rn(ua, __fmul_rn(s.kwd, w));
   // multiplicative branch: exponent gradient, its second moment, proposal
   const float ge = __fmul_rn(__fmul_rn(s.ln2, w), g);
   o.ve = __fmaf_rn(s.b2, ve, __fmul_rn(s.omb2, __fmul_rn(ge, ge)));
   float n = __fdiv_rn(ge, __fmaf_rn(__fsqrt_rn(o.ve), s.c2, s.eps));
-  if (s.gmax_on) n = fmaxf(-s.gmax, fminf(n, s.gmax));
+  if (OPT && s.gmax_on) n = fmaxf(-s.gmax, fminf(n, s.gmax));
   float um = __fdiv_rn(__fmul_rn(s.km, n), fmaxf(fabsf(w), s.tau));
   um = fmaxf(s.lo, fminf(um, s.hi));
   // combine: w + w u_m + u_a
   float wn = __fadd_rn(__fmaf_rn(w, um, w), ua);
-  if (s.wmax_on) wn = fmaxf(-s.wmax, fminf(wn, s.wmax));
+  if (OPT && s.wmax_on) wn = fmaxf(-s.wmax, fminf(wn, s.wmax));
   o.wn = wn;
   return o;
+}
+
+// ---------------------------------------------------------------------------
+// Certified fast update (Ziv's rounding test: A. Ziv, "Fast evaluation of
+// elementary mathematical functions with correctly rounded last bit", ACM
+// TOMS 17(3), 1991).  The moments are computed exactly as above; the two
+// square roots and three divisions of the weight update use the hardware
+// approximations sqrt.approx.f32 and div.approx.f32 (__fdividef; CUDA
+// documents at most 2 ulp for divisors in [2^-126, 2^126]).  With every
+// approximate result assumed within 2^-19 relative of the correctly rounded
+// one -- 8x the documented bound -- the fast weight wn' differs from the
+// canonical wn by at most
+//     eps = (|w u_m'| + |u_a'|) 2^-17 + (|w + w u_m'| + |wn'|) 2^-22 + 2^-140
+// (the relative errors propagate through the divisions, the clamp is
+// 1-Lipschitz, and each of the two final roundings adds at most one ulp; the
+// constants carry a further factor-of-two margin).  The caller stores the
+// encoding of wn' only when encoding wn' - eps (rounded down) and wn' + eps
+// (rounded up) gives the same code: every encoder here is monotone, so the
+// canonical wn, which lies in between, has that code too.  Otherwise the
+// element is recomputed with the exact sequence (madam_wn_exact).  Results
+// are therefore identical to the canonical sequence bit for bit; the test
+// only decides how much work that takes.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ float sqrt_approx(float x) {
+  float y;
+  asm("sqrt.approx.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+struct CertUpd {
+  float wn, lo, hi;  // fast weight and the interval holding the canonical one
+  float m, v, ve;    // exact moments
+  bool ok;           // divisors in the documented range and wn' finite
+};
+
+__device__ __forceinline__ CertUpd madam_update_cert(const StepScalars& s, float w, float g, float m, float v,
+                                                     float ve) {
+  CertUpd o;
+  o.m = __fmaf_rn(s.b1, m, __fmul_rn(s.omb1, g));
+  o.v = __fmaf_rn(s.b2, v, __fmul_rn(s.omb2, __fmul_rn(g, g)));
+  const float ge = __fmul_rn(__fmul_rn(s.ln2, w), g);
+  o.ve = __fmaf_rn(s.b2, ve, __fmul_rn(s.omb2, __fmul_rn(ge, ge)));
+  const float den_a = __fmaf_rn(sqrt_approx(o.v), s.c2, s.eps);
+  const float ua = __fdividef(__fmul_rn(s.ka, o.m), den_a);
+  const float den_e = __fmaf_rn(sqrt_approx(o.ve), s.c2, s.eps);
+  const float n = __fdividef(ge, den_e);
+  const float rho = fmaxf(fabsf(w), s.tau);
+  float um = __fdividef(__fmul_rn(s.km, n), rho);
+  um = fmaxf(s.lo, fminf(um, s.hi));
+  const float t = __fmaf_rn(w, um, w);
+  o.wn = __fadd_rn(t, ua);
+  const float e = __fmaf_rn(__fadd_rn(fabsf(__fmul_rn(w, um)), fabsf(ua)), 7.62939453125e-06f /* 2^-17 */,
+                            __fmaf_rn(__fadd_rn(fabsf(t), fabsf(o.wn)), 2.384185791015625e-07f /* 2^-22 */,
+                                      7.174648137343064e-43f /* 2^-140 */));
+  o.lo = __fsub_rd(o.wn, e);
+  o.hi = __fadd_ru(o.wn, e);
+  // divisors must stay below 2^125 (their lower bounds eps, tau >= 2^-125 are
+  // checked on the host), and wn' must be finite
+  o.ok = fmaxf(fmaxf(den_a, den_e), rho) <= 4.253529586511731e+37f /* 2^125 */ && fabsf(o.wn) < INFINITY;
+  return o;
+}
+
+// The weight of the canonical sequence from the already updated (exact)
+// moments: the exact fallback of the certified path.
+static __device__ __noinline__ float madam_wn_exact(const StepScalars& s, float w, float g, float m1, float v1,
+                                             float ve1) {
+  const float ua = __fdiv_rn(__fmul_rn(s.ka, m1), __fmaf_rn(__fsqrt_rn(v1), s.c2, s.eps));
+  const float ge = __fmul_rn(__fmul_rn(s.ln2, w), g);
+  const float n = __fdiv_rn(ge, __fmaf_rn(__fsqrt_rn(ve1), s.c2, s.eps));
+  float um = __fdiv_rn(__fmul_rn(s.km, n), fmaxf(fabsf(w), s.tau));
+  um = fmaxf(s.lo, fminf(um, s.hi));
+  return __fadd_rn(__fmaf_rn(w, um, w), ua);
 }
 
 // ---------------------------------------------------------------------------
@@ -137,10 +283,9 @@ __device__ __forceinline__ uint32_t bf16x2_rn(float lo, float hi) {
   return d;
 }
 
-// Stochastic BF16 of x given the complement of its 16 random bits in the low
-// half of `nr`: adding 0xFFFF - R carries into the kept half exactly when
-// R < (low half of x), i.e. with probability (low half) / 2^16.  Returns the
-// 32-bit sum whose high half is the result.
+// Stochastic BF16 of x given the complement of its 16 random bits (0xFFFF -
+// R): the sum carries into the kept half exactly when R < (low half of x),
+// i.e. with probability (low half) / 2^16.  The result is the high half.
 __device__ __forceinline__ uint32_t bf16_sr_sum(float x, uint32_t nr16) {
   const uint32_t sum = __float_as_uint(x) + nr16;
   return (x != x) ? 0x7FFF0000u : sum;
@@ -193,181 +338,234 @@ __device__ __forceinline__ uint32_t e4m3_encode(float x, uint32_t r) {
 // bits, finite and >= 0); keep e_cur when A = 0; clamp to [-100, 100].
 __device__ __forceinline__ int32_t fp8_next_exponent(uint32_t a_bits, int32_t e_cur) {
   if (a_bits == 0u) return e_cur;
-  const int32_t ef = (int32_t)(a_bits >> 23);
+  const int32_t ef = static_cast<int32_t>(a_bits >> 23);
   int32_t k = -100;
   if (ef != 0) k = ef - 127 - 8 + ((a_bits & 0x7FFFFFu) > 0x600000u ? 1 : 0);
   return k < -100 ? -100 : (k > 100 ? 100 : k);
 }
 
-__device__ __forceinline__ float pow2f(int32_t e) { return __uint_as_float((uint32_t)(e + 127) << 23); }
+__device__ __forceinline__ float pow2f(int32_t e) {
+  return __uint_as_float(static_cast<uint32_t>(e + 127) << 23);
+}
+
+__device__ __forceinline__ bool aligned(const void* p, uintptr_t bytes) {
+  return (reinterpret_cast<uintptr_t>(p) & (bytes - 1)) == 0;
+}
+
+// Bytes of a tile's slice of one array that the TMA stages: the largest
+// multiple of 16 within the tile, or nothing when the array's base pointer is
+// not 16-byte aligned (tile starts are then misaligned too).
+__device__ __forceinline__ uint32_t staged_bytes(const void* base, int count, int esize) {
+  return aligned(base, 16) ? (static_cast<uint32_t>(count * esize) & ~15u) : 0u;
+}
 
 // ---------------------------------------------------------------------------
-// One group of 8 elements.  FULL: all 8 valid and every pointer aligned for
-// vector access; otherwise element-wise loads/stores of the `valid` leading
-// elements.
+// Group loads: 8 consecutive elements from shared memory (staged) or global.
 // ---------------------------------------------------------------------------
-template <int WD, int GD, int MD, bool SR, bool FULL>
-__device__ __forceinline__ void process_group(const StepArgs& a, const TensorDesc& d,
-                                              const void* gp, int64_t e0, int valid, int64_t gi,
-                                              float dec_scale, float enc_scale,
-                                              uint32_t& amax_bits) {
-  float w[8], g[8], m[8], v[8], ve[8];
-  // ---- loads -------------------------------------------------------------
-  if (FULL) {
-    if (WD == kBF16) {
-      uint32_t r[4];
-      ld4(static_cast<const uint16_t*>(d.w) + e0, r);
+template <bool RO>
+__device__ __forceinline__ void get_bf16(float (&x)[8], bool staged, uint32_t saddr, const void* g,
+                                         int64_t e0, int valid, bool vec) {
+  if (staged || (vec && valid == kGroup)) {
+    uint32_t r[4];
+    if (staged) lds4(saddr, r);
+    else if (RO) ld4_ro(static_cast<const uint16_t*>(g) + e0, r);
+    else ld4(static_cast<const uint16_t*>(g) + e0, r);
 #pragma unroll
-      for (int i = 0; i < 4; ++i) { w[2 * i] = bf16_lo(r[i]); w[2 * i + 1] = bf16_hi(r[i]); }
-    } else {
-      uint32_t r[2];
-      ld2(static_cast<const uint8_t*>(d.w) + e0, r);
-#pragma unroll
-      for (int j = 0; j < 8; ++j)
-        w[j] = __fmul_rn(e4m3_value((r[j >> 2] >> (8 * (j & 3))) & 0xFFu), dec_scale);
-    }
-    if (GD == kF32) {
-      uint32_t r[8];
-      ld8_ro(static_cast<const float*>(gp) + e0, r);
-#pragma unroll
-      for (int j = 0; j < 8; ++j) g[j] = __uint_as_float(r[j]);
-    } else {
-      uint32_t r[4];
-      ld4_ro(static_cast<const uint16_t*>(gp) + e0, r);
-#pragma unroll
-      for (int i = 0; i < 4; ++i) { g[2 * i] = bf16_lo(r[i]); g[2 * i + 1] = bf16_hi(r[i]); }
-    }
-    if (MD == kF32) {
-      uint32_t rm[8], rv[8], re[8];
-      ld8(static_cast<const float*>(d.m) + e0, rm);
-      ld8(static_cast<const float*>(d.v) + e0, rv);
-      ld8(static_cast<const float*>(d.ve) + e0, re);
-#pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        m[j] = __uint_as_float(rm[j]); v[j] = __uint_as_float(rv[j]); ve[j] = __uint_as_float(re[j]);
-      }
-    } else {
-      uint32_t rm[4], rv[4], re[4];
-      ld4(static_cast<const uint16_t*>(d.m) + e0, rm);
-      ld4(static_cast<const uint16_t*>(d.v) + e0, rv);
-      ld4(static_cast<const uint16_t*>(d.ve) + e0, re);
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        m[2 * i] = bf16_lo(rm[i]); m[2 * i + 1] = bf16_hi(rm[i]);
-        v[2 * i] = bf16_lo(rv[i]); v[2 * i + 1] = bf16_hi(rv[i]);
-        ve[2 * i] = bf16_lo(re[i]); ve[2 * i + 1] = bf16_hi(re[i]);
-      }
-    }
+    for (int i = 0; i < 4; ++i) { x[2 * i] = bf16_lo(r[i]); x[2 * i + 1] = bf16_hi(r[i]); }
   } else {
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      w[j] = g[j] = m[j] = v[j] = ve[j] = 0.0f;
-      if (j < valid) {
-        const int64_t e = e0 + j;
-        if (WD == kBF16) w[j] = __uint_as_float((uint32_t)static_cast<const uint16_t*>(d.w)[e] << 16);
-        else w[j] = __fmul_rn(e4m3_value(static_cast<const uint8_t*>(d.w)[e]), dec_scale);
-        if (GD == kF32) g[j] = static_cast<const float*>(gp)[e];
-        else g[j] = __uint_as_float((uint32_t)static_cast<const uint16_t*>(gp)[e] << 16);
-        if (MD == kF32) {
-          m[j] = static_cast<const float*>(d.m)[e];
-          v[j] = static_cast<const float*>(d.v)[e];
-          ve[j] = static_cast<const float*>(d.ve)[e];
-        } else {
-          m[j] = __uint_as_float((uint32_t)static_cast<const uint16_t*>(d.m)[e] << 16);
-          v[j] = __uint_as_float((uint32_t)static_cast<const uint16_t*>(d.v)[e] << 16);
-          ve[j] = __uint_as_float((uint32_t)static_cast<const uint16_t*>(d.ve)[e] << 16);
-        }
-      }
-    }
+    for (int j = 0; j < kGroup; ++j)
+      x[j] = j < valid ? __uint_as_float(static_cast<uint32_t>(static_cast<const uint16_t*>(g)[e0 + j]) << 16)
+                       : 0.0f;
   }
+}
 
-  // ---- random bits (one Philox block per 8 BF16 lanes / 4 E4M3 lanes) ----
+template <bool RO>
+__device__ __forceinline__ void get_f32(float (&x)[8], bool staged, uint32_t saddr, const void* g,
+                                        int64_t e0, int valid, bool vec) {
+  if (staged) {
+    uint32_t a[4], b[4];
+    lds4(saddr, a);
+    lds4(saddr + 16, b);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) { x[i] = __uint_as_float(a[i]); x[4 + i] = __uint_as_float(b[i]); }
+  } else if (vec && valid == kGroup) {
+    uint32_t r[8];
+    if (RO) ld8_ro(static_cast<const float*>(g) + e0, r);
+    else ld8(static_cast<const float*>(g) + e0, r);
+#pragma unroll
+    for (int j = 0; j < kGroup; ++j) x[j] = __uint_as_float(r[j]);
+  } else {
+#pragma unroll
+    for (int j = 0; j < kGroup; ++j) x[j] = j < valid ? static_cast<const float*>(g)[e0 + j] : 0.0f;
+  }
+}
+
+__device__ __forceinline__ void get_e4m3(float (&x)[8], bool staged, uint32_t saddr, const void* g,
+                                         int64_t e0, int valid, bool vec, float scale) {
+  if (staged || (vec && valid == kGroup)) {
+    uint32_t r[2];
+    if (staged) lds2(saddr, r);
+    else ld2(static_cast<const uint8_t*>(g) + e0, r);
+#pragma unroll
+    for (int j = 0; j < kGroup; ++j) x[j] = __fmul_rn(e4m3_value((r[j >> 2] >> (8 * (j & 3))) & 0xFFu), scale);
+  } else {
+#pragma unroll
+    for (int j = 0; j < kGroup; ++j)
+      x[j] = j < valid ? __fmul_rn(e4m3_value(static_cast<const uint8_t*>(g)[e0 + j]), scale) : 0.0f;
+  }
+}
+
+// Group stores (vector when whole and aligned, else element by element).
+__device__ __forceinline__ void put_bf16(const uint32_t (&o)[4], void* g, int64_t e0, int valid, bool vec) {
+  if (vec && valid == kGroup) {
+    st4(static_cast<uint16_t*>(g) + e0, o);
+  } else {
+#pragma unroll
+    for (int j = 0; j < kGroup; ++j)
+      if (j < valid)
+        static_cast<uint16_t*>(g)[e0 + j] =
+            static_cast<uint16_t>((j & 1) ? (o[j >> 1] >> 16) : (o[j >> 1] & 0xFFFFu));
+  }
+}
+__device__ __forceinline__ void put_f32(const float (&x)[8], void* g, int64_t e0, int valid, bool vec) {
+  if (vec && valid == kGroup) {
+    uint32_t o[8];
+#pragma unroll
+    for (int j = 0; j < kGroup; ++j) o[j] = __float_as_uint(x[j]);
+    st8(static_cast<float*>(g) + e0, o);
+  } else {
+#pragma unroll
+    for (int j = 0; j < kGroup; ++j)
+      if (j < valid) static_cast<float*>(g)[e0 + j] = x[j];
+  }
+}
+__device__ __forceinline__ void put_e4m3(const uint32_t (&o)[2], void* g, int64_t e0, int valid, bool vec) {
+  if (vec && valid == kGroup) {
+    st2(static_cast<uint8_t*>(g) + e0, o);
+  } else {
+#pragma unroll
+    for (int j = 0; j < kGroup; ++j)
+      if (j < valid) static_cast<uint8_t*>(g)[e0 + j] = static_cast<uint8_t>(o[j >> 2] >> (8 * (j & 3)));
+  }
+}
+
+__host__ __device__ constexpr int esize_of(int dt) { return dt == kF32 ? 4 : (dt == kBF16 ? 2 : 1); }
+
+// Per-tensor values the consumers keep while walking a tensor's tiles.
+struct TensorCtx {
+  TensorDesc d;
+  const void* g;
+  int64_t tiles;
+  bool vec;            // all pointers aligned for vector access by whole groups
+  bool fast;           // whole tiles are fully staged and stored with vector stores
+  float dec_scale, enc_scale;
+};
+
+template <int WD, int GD, int MD>
+__device__ __forceinline__ void load_tensor(const StepArgs& a, int k, TensorCtx& c) {
+  c.d = a.desc[k];
+  c.g = a.grads[k];
+  c.tiles = (c.d.numel + kTile - 1) / kTile;
+  c.vec = aligned(c.d.w, WD == kBF16 ? 16 : 8) && aligned(c.g, GD == kF32 ? 32 : 16) &&
+          aligned(c.d.m, MD == kF32 ? 32 : 16) && aligned(c.d.v, MD == kF32 ? 32 : 16) &&
+          aligned(c.d.ve, MD == kF32 ? 32 : 16);
+  c.fast = c.vec && aligned(c.d.w, 16) && aligned(c.g, 16) && aligned(c.d.m, 16) && aligned(c.d.v, 16) &&
+           aligned(c.d.ve, 16);
+  c.dec_scale = c.enc_scale = 1.0f;
+}
+
+// Update 8 loaded elements and store them (vector stores when `vec` and
+// whole, else element by element).
+template <int WD, int GD, int MD, bool SR, bool OPT>
+__device__ __forceinline__ void finish_group(const StepArgs& a, const TensorCtx& x, int64_t e0, int valid,
+                                             float (&w)[8], float (&g)[8], float (&m)[8], float (&v)[8],
+                                             float (&ve)[8], uint32_t& amax_bits) {
+  // random bits: one Philox block per 8 BF16 lanes, two per 8 E4M3 lanes
   uint32_t rnd[8];
   if (SR) {
+    const uint64_t gi = static_cast<uint64_t>(x.d.goff + e0) >> 3;  // global group index
     if (WD == kBF16) {
-      const uint4 r = philox4x32_10((uint32_t)gi, (uint32_t)((uint64_t)gi >> 32), a.t_lo, a.t_hi,
-                                    a.key0, a.key1);
-      // complemented 16-bit lanes, ready for the carry trick
+      const uint4 r = philox4x32_10(static_cast<uint32_t>(gi), static_cast<uint32_t>(gi >> 32), a.t_lo,
+                                    a.t_hi, a.rk0, a.rk1);
       rnd[0] = ~r.x & 0xFFFFu; rnd[1] = ~r.x >> 16;
       rnd[2] = ~r.y & 0xFFFFu; rnd[3] = ~r.y >> 16;
       rnd[4] = ~r.z & 0xFFFFu; rnd[5] = ~r.z >> 16;
       rnd[6] = ~r.w & 0xFFFFu; rnd[7] = ~r.w >> 16;
     } else {
-      const uint64_t b0 = 2ull * (uint64_t)gi;
-      const uint4 r0 = philox4x32_10((uint32_t)b0, (uint32_t)(b0 >> 32), a.t_lo, a.t_hi, a.key0, a.key1);
-      const uint64_t b1 = b0 + 1ull;
-      const uint4 r1 = philox4x32_10((uint32_t)b1, (uint32_t)(b1 >> 32), a.t_lo, a.t_hi, a.key0, a.key1);
+      const uint64_t b0 = 2ull * gi, b1 = b0 + 1ull;
+      const uint4 r0 = philox4x32_10(static_cast<uint32_t>(b0), static_cast<uint32_t>(b0 >> 32), a.t_lo,
+                                     a.t_hi, a.rk0, a.rk1);
+      const uint4 r1 = philox4x32_10(static_cast<uint32_t>(b1), static_cast<uint32_t>(b1 >> 32), a.t_lo,
+                                     a.t_hi, a.rk0, a.rk1);
       rnd[0] = r0.x; rnd[1] = r0.y; rnd[2] = r0.z; rnd[3] = r0.w;
       rnd[4] = r1.x; rnd[5] = r1.y; rnd[6] = r1.z; rnd[7] = r1.w;
     }
   }
 
-  // ---- update ------------------------------------------------------------
+  if (WD == kBF16 && !OPT && a.s.cert_ok) {  // certified fast path (see madam_update_cert)
+    uint32_t out[8];
+    uint32_t redo = 0u;
+#pragma unroll
+    for (int j = 0; j < kGroup; ++j) {
+      const CertUpd u = madam_update_cert(a.s, w[j], g[j], m[j], v[j], ve[j]);
+      bool same;
+      if (SR) {
+        const uint32_t slo = __float_as_uint(u.lo) + rnd[j], shi = __float_as_uint(u.hi) + rnd[j];
+        same = ((slo ^ shi) >> 16) == 0u;
+        out[j] = slo >> 16;
+      } else {
+        const uint32_t pair = bf16x2_rn(u.lo, u.hi);
+        same = ((pair ^ (pair >> 16)) & 0xFFFFu) == 0u;
+        out[j] = pair & 0xFFFFu;
+      }
+      if (!(u.ok && same)) redo |= 1u << j;
+      m[j] = u.m; v[j] = u.v; ve[j] = u.ve;
+    }
+    if (redo) {  // rare: encode the canonical weight of the undecided elements
+#pragma unroll
+      for (int j = 0; j < kGroup; ++j) {
+        if ((redo >> j) & 1u) {
+          const float xe = madam_wn_exact(a.s, w[j], g[j], m[j], v[j], ve[j]);
+          out[j] = SR ? (bf16_sr_sum(xe, rnd[j]) >> 16) : (bf16x2_rn(xe, xe) & 0xFFFFu);
+        }
+      }
+    }
+    uint32_t ow[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) ow[i] = out[2 * i] | (out[2 * i + 1] << 16);
+    put_bf16(ow, x.d.w, e0, valid, x.vec);
+  } else {
   float wn[8];
 #pragma unroll
-  for (int j = 0; j < 8; ++j) {
-    const Upd u = madam_update(a.s, w[j], g[j], m[j], v[j], ve[j]);
+  for (int j = 0; j < kGroup; ++j) {
+    const Upd u = madam_update<OPT>(a.s, w[j], g[j], m[j], v[j], ve[j]);
     wn[j] = u.wn; m[j] = u.m; v[j] = u.v; ve[j] = u.ve;
   }
 
-  // ---- encode + store ------------------------------------------------------
   if (WD == kBF16) {
     uint32_t ow[4];
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
-      if (SR) {
-        const uint32_t s0 = bf16_sr_sum(wn[2 * i], rnd[2 * i]);
-        const uint32_t s1 = bf16_sr_sum(wn[2 * i + 1], rnd[2 * i + 1]);
-        ow[i] = __byte_perm(s0, s1, 0x7632);
-      } else {
-        ow[i] = bf16x2_rn(wn[2 * i], wn[2 * i + 1]);
-      }
+      if (SR) ow[i] = __byte_perm(bf16_sr_sum(wn[2 * i], rnd[2 * i]), bf16_sr_sum(wn[2 * i + 1], rnd[2 * i + 1]), 0x7632);
+      else ow[i] = bf16x2_rn(wn[2 * i], wn[2 * i + 1]);
     }
-    if (FULL) {
-      st4(static_cast<uint16_t*>(d.w) + e0, ow);
-    } else {
-#pragma unroll
-      for (int j = 0; j < 8; ++j)
-        if (j < valid)
-          static_cast<uint16_t*>(d.w)[e0 + j] = (uint16_t)((j & 1) ? (ow[j >> 1] >> 16) : (ow[j >> 1] & 0xFFFFu));
-    }
+    put_bf16(ow, x.d.w, e0, valid, x.vec);
   } else {
     uint32_t ow[2] = {0u, 0u};
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
+    for (int j = 0; j < kGroup; ++j) {
       const uint32_t wb = __float_as_uint(wn[j]) & 0x7FFFFFFFu;
-      if ((FULL || j < valid) && wb < 0x7F800000u) amax_bits = max(amax_bits, wb);
-      const uint32_t c = e4m3_encode<SR>(__fmul_rn(wn[j], enc_scale), SR ? rnd[j] : 0u);
-      ow[j >> 2] |= c << (8 * (j & 3));
+      if (j < valid && wb < 0x7F800000u) amax_bits = max(amax_bits, wb);
+      ow[j >> 2] |= e4m3_encode<SR>(__fmul_rn(wn[j], x.enc_scale), SR ? rnd[j] : 0u) << (8 * (j & 3));
     }
-    if (FULL) {
-      st2(static_cast<uint8_t*>(d.w) + e0, ow);
-    } else {
-#pragma unroll
-      for (int j = 0; j < 8; ++j)
-        if (j < valid) static_cast<uint8_t*>(d.w)[e0 + j] = (uint8_t)(ow[j >> 2] >> (8 * (j & 3)));
-    }
+    put_e4m3(ow, x.d.w, e0, valid, x.vec);
   }
-
+  }
   if (MD == kF32) {
-    if (FULL) {
-      uint32_t om[8], ov[8], oe[8];
-#pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        om[j] = __float_as_uint(m[j]); ov[j] = __float_as_uint(v[j]); oe[j] = __float_as_uint(ve[j]);
-      }
-      st8(static_cast<float*>(d.m) + e0, om);
-      st8(static_cast<float*>(d.v) + e0, ov);
-      st8(static_cast<float*>(d.ve) + e0, oe);
-    } else {
-#pragma unroll
-      for (int j = 0; j < 8; ++j)
-        if (j < valid) {
-          static_cast<float*>(d.m)[e0 + j] = m[j];
-          static_cast<float*>(d.v)[e0 + j] = v[j];
-          static_cast<float*>(d.ve)[e0 + j] = ve[j];
-        }
-    }
+    put_f32(m, x.d.m, e0, valid, x.vec);
+    put_f32(v, x.d.v, e0, valid, x.vec);
+    put_f32(ve, x.d.ve, e0, valid, x.vec);
   } else {
     uint32_t om[4], ov[4], oe[4];
 #pragma unroll
@@ -376,81 +574,200 @@ __device__ __forceinline__ void process_group(const StepArgs& a, const TensorDes
       ov[i] = bf16x2_rn(v[2 * i], v[2 * i + 1]);
       oe[i] = bf16x2_rn(ve[2 * i], ve[2 * i + 1]);
     }
-    if (FULL) {
-      st4(static_cast<uint16_t*>(d.m) + e0, om);
-      st4(static_cast<uint16_t*>(d.v) + e0, ov);
-      st4(static_cast<uint16_t*>(d.ve) + e0, oe);
-    } else {
-#pragma unroll
-      for (int j = 0; j < 8; ++j)
-        if (j < valid) {
-          const int sh = (j & 1) ? 16 : 0;
-          static_cast<uint16_t*>(d.m)[e0 + j] = (uint16_t)(om[j >> 1] >> sh);
-          static_cast<uint16_t*>(d.v)[e0 + j] = (uint16_t)(ov[j >> 1] >> sh);
-          static_cast<uint16_t*>(d.ve)[e0 + j] = (uint16_t)(oe[j >> 1] >> sh);
-        }
-    }
+    put_bf16(om, x.d.m, e0, valid, x.vec);
+    put_bf16(ov, x.d.v, e0, valid, x.vec);
+    put_bf16(oe, x.d.ve, e0, valid, x.vec);
   }
 }
 
-__device__ __forceinline__ bool aligned(const void* p, uintptr_t bytes) {
-  return (reinterpret_cast<uintptr_t>(p) & (bytes - 1)) == 0;
+// One group of a partial tile, or of a tensor whose arrays are not all staged
+// or aligned: loads each array from the stage when its bytes were staged, else
+// from global memory; kept out of line so the whole-tile path stays lean.
+template <int WD, int GD, int MD, bool SR, bool OPT>
+__device__ __noinline__ void general_group(const StepArgs& a, const TensorCtx& x, int64_t tile_e0, int count,
+                                           int c, uint32_t st, uint32_t& amax_bits) {
+  constexpr int WS = esize_of(WD), GS = esize_of(GD), MS = esize_of(MD);
+  if (kGroup * c >= count) return;
+  const int valid = count - kGroup * c < kGroup ? count - kGroup * c : kGroup;
+  const int64_t e0 = tile_e0 + kGroup * c;
+  const uint32_t end = static_cast<uint32_t>(kGroup * (c + 1));  // elements through this group
+  float w[8], g[8], m[8], v[8], ve[8];
+  if (WD == kBF16)
+    get_bf16<false>(w, end * WS <= staged_bytes(x.d.w, count, WS), st + kGroup * WS * c, x.d.w, e0, valid, x.vec);
+  else
+    get_e4m3(w, end * WS <= staged_bytes(x.d.w, count, WS), st + kGroup * WS * c, x.d.w, e0, valid, x.vec,
+             x.dec_scale);
+  const bool g_st = end * GS <= staged_bytes(x.g, count, GS);
+  if (GD == kF32) get_f32<true>(g, g_st, st + a.off_g + kGroup * GS * c, x.g, e0, valid, x.vec);
+  else get_bf16<true>(g, g_st, st + a.off_g + kGroup * GS * c, x.g, e0, valid, x.vec);
+  const bool m_st = end * MS <= staged_bytes(x.d.m, count, MS);
+  const bool v_st = end * MS <= staged_bytes(x.d.v, count, MS);
+  const bool e_st = end * MS <= staged_bytes(x.d.ve, count, MS);
+  if (MD == kF32) {
+    get_f32<false>(m, m_st, st + a.off_m + kGroup * MS * c, x.d.m, e0, valid, x.vec);
+    get_f32<false>(v, v_st, st + a.off_v + kGroup * MS * c, x.d.v, e0, valid, x.vec);
+    get_f32<false>(ve, e_st, st + a.off_ve + kGroup * MS * c, x.d.ve, e0, valid, x.vec);
+  } else {
+    get_bf16<false>(m, m_st, st + a.off_m + kGroup * MS * c, x.d.m, e0, valid, x.vec);
+    get_bf16<false>(v, v_st, st + a.off_v + kGroup * MS * c, x.d.v, e0, valid, x.vec);
+    get_bf16<false>(ve, e_st, st + a.off_ve + kGroup * MS * c, x.d.ve, e0, valid, x.vec);
+  }
+  finish_group<WD, GD, MD, SR, OPT>(a, x, e0, valid, w, g, m, v, ve, amax_bits);
 }
 
 // ---------------------------------------------------------------------------
-// The persistent step kernel: one CTA per slice of the global group range.
+// The step kernel.
 // ---------------------------------------------------------------------------
-template <int WD, int GD, int MD, bool SR>
-__global__ void __launch_bounds__(kThreads) step_kernel(const __grid_constant__ StepArgs a) {
-  const int64_t G = a.total_groups;
-  const int64_t g_begin = (int64_t)blockIdx.x * G / gridDim.x;
-  const int64_t g_end = ((int64_t)blockIdx.x + 1) * G / gridDim.x;
-  if (g_begin >= g_end) return;
-  const int n = a.n_tensors;
+template <int WD, int GD, int MD, bool SR, bool OPT>
+__global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant__ StepArgs a) {
+  constexpr int WS = esize_of(WD), GS = esize_of(GD), MS = esize_of(MD);
+  extern __shared__ __align__(128) uint8_t smem[];
+  __shared__ __align__(8) uint64_t full_bar[kMaxStages];
+  __shared__ __align__(8) uint64_t empty_bar[kMaxStages];
 
-  for (int k = a.cta_first[blockIdx.x]; k < n; ++k) {
-    const TensorDesc d = a.desc[k];
-    const int64_t t0 = d.goff >> 3;
-    const int64_t t1 = t0 + ((d.numel + 7) >> 3);
-    if (t0 >= g_end) break;
-    const int64_t lo = g_begin > t0 ? g_begin : t0;
-    const int64_t hi = g_end < t1 ? g_end : t1;
-    if (lo >= hi) continue;
+  const int tid = threadIdx.x;
+  const int warp = tid >> 5, lane = tid & 31;
+  const int S = a.stages;
+  if (tid == 0) {
+    for (int s = 0; s < S; ++s) {
+      mbar_init(smem_addr(&full_bar[s]), 1);
+      mbar_init(smem_addr(&empty_bar[s]), kConsumerWarps);
+    }
+    mbar_init_fence();
+  }
+  __syncthreads();
+
+  const int64_t T = a.total_tiles;
+  const int64_t tb = static_cast<int64_t>(blockIdx.x) * T / gridDim.x;
+  const int64_t te = (static_cast<int64_t>(blockIdx.x) + 1) * T / gridDim.x;
+  if (tb >= te) return;
+  const uint32_t smem0 = smem_addr(smem);
+
+  // ------------------------------------------------------------ producer --
+  if (warp == kConsumerWarps) {
+    if (lane != 0) return;
+    const uint64_t pol = evict_first_policy();
+    int k = a.cta_first[blockIdx.x];
+    TensorDesc d = a.desc[k];
     const void* gp = a.grads[k];
-
-    const bool vec = aligned(d.w, WD == kBF16 ? 16 : 8) && aligned(gp, GD == kF32 ? 32 : 16) &&
-                     aligned(d.m, MD == kF32 ? 32 : 16) && aligned(d.v, MD == kF32 ? 32 : 16) &&
-                     aligned(d.ve, MD == kF32 ? 32 : 16);
-
-    float dec_scale = 1.0f, enc_scale = 1.0f;
-    if (WD == kE4M3) {
-      const int32_t e_cur = a.fp8_exp[(int64_t)a.e_cur_slot * n + k];
-      const uint32_t a_cur = a.fp8_amax[(int64_t)a.a_cur_slot * n + k];
-      const int32_t e_next = fp8_next_exponent(a_cur, e_cur);
-      dec_scale = pow2f(e_cur);
-      enc_scale = pow2f(-e_next);
-      if (lo == t0 && threadIdx.x == 0) {  // the CTA holding the tensor's first group
-        a.fp8_exp[(int64_t)a.e_next_slot * n + k] = e_next;
-        a.fp8_amax[(int64_t)a.a_zero_slot * n + k] = 0u;
+    int64_t tiles = (d.numel + kTile - 1) / kTile;
+    int s = 0;
+    uint32_t use = 0;
+    int64_t issued = 0;
+    bool failed = false;
+    for (int64_t t = tb; t < te; ++t) {
+      while (t >= d.tile_off + tiles) {
+        ++k;
+        d = a.desc[k];
+        gp = a.grads[k];
+        tiles = (d.numel + kTile - 1) / kTile;
+      }
+      if (use > 0 && !mbar_wait(smem_addr(&empty_bar[s]), (use - 1) & 1u)) {
+        if (a.err) atomicOr(a.err, kErrEmptyWait);
+        failed = true;
+        break;
+      }
+      const int64_t e0 = (t - d.tile_off) * kTile;
+      const int count = static_cast<int>(d.numel - e0 < kTile ? d.numel - e0 : kTile);
+      const uint32_t nw = staged_bytes(d.w, count, WS), ng = staged_bytes(gp, count, GS);
+      const uint32_t nm = staged_bytes(d.m, count, MS), nv = staged_bytes(d.v, count, MS);
+      const uint32_t nve = staged_bytes(d.ve, count, MS);
+      const uint32_t bar = smem_addr(&full_bar[s]);
+      const uint32_t st = smem0 + static_cast<uint32_t>(s * a.stage_bytes);
+      mbar_arrive_expect_tx(bar, nw + ng + nm + nv + nve);
+      if (nw) tma_load(st, static_cast<const uint8_t*>(d.w) + e0 * WS, nw, bar, pol);
+      if (ng) tma_load(st + a.off_g, static_cast<const uint8_t*>(gp) + e0 * GS, ng, bar, pol);
+      if (nm) tma_load(st + a.off_m, static_cast<const uint8_t*>(d.m) + e0 * MS, nm, bar, pol);
+      if (nv) tma_load(st + a.off_v, static_cast<const uint8_t*>(d.v) + e0 * MS, nv, bar, pol);
+      if (nve) tma_load(st + a.off_ve, static_cast<const uint8_t*>(d.ve) + e0 * MS, nve, bar, pol);
+      ++issued;
+      if (++s == S) { s = 0; ++use; }
+    }
+    if (failed) {  // wait (bounded) for this CTA's copies still in flight, then leave
+      const int64_t last = issued < S ? issued : S;
+      for (int64_t i = 1; i <= last; ++i) {
+        const int64_t it = issued - i;
+        if (!mbar_wait(smem_addr(&full_bar[it % S]), static_cast<uint32_t>((it / S) & 1)) && a.err)
+          atomicOr(a.err, kErrDrainWait);
       }
     }
+    return;
+  }
 
-    uint32_t amax_bits = 0u;
-    for (int64_t gi = lo + threadIdx.x; gi < hi; gi += kThreads) {
-      const int64_t e0 = (gi - t0) * kGroup;
-      const int64_t left = d.numel - e0;
-      const int valid = left < kGroup ? (int)left : kGroup;
-      if (vec && valid == kGroup)
-        process_group<WD, GD, MD, SR, true>(a, d, gp, e0, valid, gi, dec_scale, enc_scale, amax_bits);
-      else
-        process_group<WD, GD, MD, SR, false>(a, d, gp, e0, valid, gi, dec_scale, enc_scale, amax_bits);
+  // ----------------------------------------------------------- consumers --
+  const int c = tid;  // consumer index, owns elements [8c, 8c + 8) of every tile
+  const int n = a.n_tensors;
+  int k = a.cta_first[blockIdx.x];
+  TensorCtx x;
+  load_tensor<WD, GD, MD>(a, k, x);
+  int32_t e_next = 0;
+  if (WD == kE4M3) {
+    const int32_t e_cur = a.fp8_exp[static_cast<int64_t>(a.e_cur_slot) * n + k];
+    e_next = fp8_next_exponent(a.fp8_amax[static_cast<int64_t>(a.a_cur_slot) * n + k], e_cur);
+    x.dec_scale = pow2f(e_cur);
+    x.enc_scale = pow2f(-e_next);
+  }
+  uint32_t amax_bits = 0u;
+  int s = 0;
+  uint32_t use = 0;
+  for (int64_t t = tb; t < te; ++t) {
+    if (t >= x.d.tile_off + x.tiles) {  // next tensor: flush this one's E4M3 amax
+      if (WD == kE4M3) {
+        const uint32_t wmax = __reduce_max_sync(0xFFFFFFFFu, amax_bits);
+        if (lane == 0 && wmax != 0u) atomicMax(&a.fp8_amax[static_cast<int64_t>(a.a_next_slot) * n + k], wmax);
+        amax_bits = 0u;
+      }
+      do { ++k; load_tensor<WD, GD, MD>(a, k, x); } while (t >= x.d.tile_off + x.tiles);
+      if (WD == kE4M3) {
+        const int32_t e_cur = a.fp8_exp[static_cast<int64_t>(a.e_cur_slot) * n + k];
+        e_next = fp8_next_exponent(a.fp8_amax[static_cast<int64_t>(a.a_cur_slot) * n + k], e_cur);
+        x.dec_scale = pow2f(e_cur);
+        x.enc_scale = pow2f(-e_next);
+      }
     }
-
-    if (WD == kE4M3) {
-      const uint32_t wmax = __reduce_max_sync(0xFFFFFFFFu, amax_bits);
-      if ((threadIdx.x & 31) == 0 && wmax != 0u)
-        atomicMax(&a.fp8_amax[(int64_t)a.a_next_slot * n + k], wmax);
+    const int64_t tile_e0 = (t - x.d.tile_off) * kTile;
+    if (WD == kE4M3 && tile_e0 == 0 && c == 0) {  // the CTA holding the tensor's first tile
+      a.fp8_exp[static_cast<int64_t>(a.e_next_slot) * n + k] = e_next;
+      a.fp8_amax[static_cast<int64_t>(a.a_zero_slot) * n + k] = 0u;
     }
+    if (!__all_sync(0xFFFFFFFFu, mbar_wait(smem_addr(&full_bar[s]), use & 1u))) {  // warp-uniform give-up
+      if (a.err && lane == 0) atomicOr(a.err, kErrFullWait);
+      return;
+    }
+    const int count = static_cast<int>(x.d.numel - tile_e0 < kTile ? x.d.numel - tile_e0 : kTile);
+    if (count == kTile && x.fast) {  // whole tile, every array staged: straight-line group
+      const uint32_t st = smem0 + static_cast<uint32_t>(s * a.stage_bytes);
+      const int64_t e0 = tile_e0 + kGroup * c;
+      float w[8], g[8], m[8], v[8], ve[8];
+      if (WD == kBF16) get_bf16<false>(w, true, st + kGroup * WS * c, x.d.w, e0, kGroup, true);
+      else get_e4m3(w, true, st + kGroup * WS * c, x.d.w, e0, kGroup, true, x.dec_scale);
+      if (GD == kF32) get_f32<true>(g, true, st + a.off_g + kGroup * GS * c, x.g, e0, kGroup, true);
+      else get_bf16<true>(g, true, st + a.off_g + kGroup * GS * c, x.g, e0, kGroup, true);
+      if (MD == kF32) {
+        get_f32<false>(m, true, st + a.off_m + kGroup * MS * c, x.d.m, e0, kGroup, true);
+        get_f32<false>(v, true, st + a.off_v + kGroup * MS * c, x.d.v, e0, kGroup, true);
+        get_f32<false>(ve, true, st + a.off_ve + kGroup * MS * c, x.d.ve, e0, kGroup, true);
+      } else {
+        get_bf16<false>(m, true, st + a.off_m + kGroup * MS * c, x.d.m, e0, kGroup, true);
+        get_bf16<false>(v, true, st + a.off_v + kGroup * MS * c, x.d.v, e0, kGroup, true);
+        get_bf16<false>(ve, true, st + a.off_ve + kGroup * MS * c, x.d.ve, e0, kGroup, true);
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_addr(&empty_bar[s]));
+      finish_group<WD, GD, MD, SR, OPT>(a, x, e0, kGroup, w, g, m, v, ve, amax_bits);
+      if (++s == S) { s = 0; ++use; }
+      continue;
+    }
+    // partial tile or unstaged arrays: element-wise fallback, out of line
+    general_group<WD, GD, MD, SR, OPT>(a, x, tile_e0, count, c, smem0 + static_cast<uint32_t>(s * a.stage_bytes),
+                                       amax_bits);
+    __syncwarp();
+    if (lane == 0) mbar_arrive(smem_addr(&empty_bar[s]));
+    if (++s == S) { s = 0; ++use; }
+  }
+  if (WD == kE4M3) {
+    const uint32_t wmax = __reduce_max_sync(0xFFFFFFFFu, amax_bits);
+    if (lane == 0 && wmax != 0u) atomicMax(&a.fp8_amax[static_cast<int64_t>(a.a_next_slot) * n + k], wmax);
   }
 }
 

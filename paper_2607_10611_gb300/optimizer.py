@@ -75,6 +75,10 @@ class MPAdam:
     def global_offsets(self) -> List[int]:
         return [N.mpadam_global_offset(self.state, k) for k in range(self.n)]
 
+    def device_status(self) -> int:
+        """Device error bits of the steps so far (0 = none); synchronises."""
+        return N.mpadam_device_status(self.state)
+
     def set_grid(self, ctas: int):
         N.mpadam_set_grid(self.state, ctas)
 

@@ -111,6 +111,8 @@ class Run:
         oracle.step(self.host, wdt=self.wdt, gdt=self.gdt, mdt=self.mdt, hp=self.ohp, t=t,
                     fp8_state=self.fp8)
         torch.cuda.synchronize()
+        assert self.opt.device_status() == 0, "a bounded wait in the step kernel gave up"
+
 
     def compare(self, t_next: int) -> Dict[str, int]:
         """Mismatch counts per array (and the E4M3 scale state read for step t_next)."""
