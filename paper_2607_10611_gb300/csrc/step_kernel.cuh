@@ -29,6 +29,7 @@
 #pragma once
 
 #include <cstdint>
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 
 #include "step_args.h"
@@ -304,6 +305,48 @@ __device__ __forceinline__ float e4m3_value(uint32_t c) {
   return (c & 0x80u) ? -val : val;
 }
 
+// Eight E4M3 codes (bytes of r[0], r[1], lowest byte first) -> binary32.
+// E4M3 -> FP16 -> FP32 are both widening conversions, so this is exact
+// (NaN codes give NaN).
+__device__ __forceinline__ void e4m3x8_to_f32(const uint32_t (&r)[2], float (&x)[8]) {
+#pragma unroll
+  for (int i = 0; i < 2; ++i) {
+    uint32_t h01, h23;
+    asm("{\n .reg .b16 lo, hi;\n mov.b32 {lo, hi}, %2;\n"
+        " cvt.rn.f16x2.e4m3x2 %0, lo;\n cvt.rn.f16x2.e4m3x2 %1, hi;\n}"
+        : "=r"(h01), "=r"(h23)
+        : "r"(r[i]));
+    const float2 f01 = __half22float2(*reinterpret_cast<const __half2*>(&h01));
+    const float2 f23 = __half22float2(*reinterpret_cast<const __half2*>(&h23));
+    x[4 * i + 0] = f01.x;
+    x[4 * i + 1] = f01.y;
+    x[4 * i + 2] = f23.x;
+    x[4 * i + 3] = f23.y;
+  }
+}
+
+// Both ends of a bound interval (already scaled by 2^-e, outward rounded)
+// encoded at once in the E4M3 normal range: code of the lower end, and
+// whether the upper end has the same code.  Anything outside [2^-6, 448),
+// or a sign change, reports `same` = false (the caller then takes the exact
+// path, whose full encoder handles subnormals, saturation and NaN).
+template <bool SR>
+__device__ __forceinline__ uint32_t e4m3_pair_normal(float xlo, float xhi, uint32_t r, bool& same) {
+  const uint32_t blo = __float_as_uint(xlo), bhi = __float_as_uint(xhi);
+  const uint32_t alo = blo & 0x7FFFFFFFu, ahi = bhi & 0x7FFFFFFFu;
+  uint32_t clo, chi;
+  if (SR) {
+    clo = (alo >> 20) + (r < (alo << 12) ? 1u : 0u);
+    chi = (ahi >> 20) + (r < (ahi << 12) ? 1u : 0u);
+  } else {  // nearest, ties to even: carry out of (rem + 0x7FFFF + lsb)
+    clo = (alo >> 20) + (((alo & 0xFFFFFu) + 0x7FFFFu + ((alo >> 20) & 1u)) >> 20);
+    chi = (ahi >> 20) + (((ahi & 0xFFFFFu) + 0x7FFFFu + ((ahi >> 20) & 1u)) >> 20);
+  }
+  same = clo == chi && ((blo ^ bhi) >> 31) == 0u && (alo - 0x3C800000u) < (0x43E00000u - 0x3C800000u) &&
+         (ahi - 0x3C800000u) < (0x43E00000u - 0x3C800000u);
+  return ((blo >> 24) & 0x80u) | (clo - 960u);
+}
+
 // binary32 (already scaled by 2^-e) -> E4M3 code, saturating at +-448.
 template <bool SR>
 __device__ __forceinline__ uint32_t e4m3_encode(float x, uint32_t r) {
@@ -407,8 +450,9 @@ __device__ __forceinline__ void get_e4m3(float (&x)[8], bool staged, uint32_t sa
     uint32_t r[2];
     if (staged) lds2(saddr, r);
     else ld2(static_cast<const uint8_t*>(g) + e0, r);
+    e4m3x8_to_f32(r, x);
 #pragma unroll
-    for (int j = 0; j < kGroup; ++j) x[j] = __fmul_rn(e4m3_value((r[j >> 2] >> (8 * (j & 3))) & 0xFFu), scale);
+    for (int j = 0; j < kGroup; ++j) x[j] = __fmul_rn(x[j], scale);
   } else {
 #pragma unroll
     for (int j = 0; j < kGroup; ++j)
@@ -535,6 +579,38 @@ __device__ __forceinline__ void finish_group(const StepArgs& a, const TensorCtx&
 #pragma unroll
     for (int i = 0; i < 4; ++i) ow[i] = out[2 * i] | (out[2 * i + 1] << 16);
     put_bf16(ow, x.d.w, e0, valid, x.vec);
+  } else if (WD == kE4M3 && !OPT && a.s.cert_ok) {
+    // Certified fast path for E4M3: both ends of the bound are scaled by 2^-e
+    // with outward rounding and encoded; the largest |w'| must be exact, so an
+    // element whose bound reaches this thread's running maximum (of exact
+    // values) is recomputed as well -- no other element can be the maximum.
+    uint32_t code[8];
+    uint32_t redo = 0u;
+    const float amax_f = __uint_as_float(amax_bits);
+#pragma unroll
+    for (int j = 0; j < kGroup; ++j) {
+      const CertUpd u = madam_update_cert(a.s, w[j], g[j], m[j], v[j], ve[j]);
+      bool same;
+      code[j] = e4m3_pair_normal<SR>(__fmul_rd(u.lo, x.enc_scale), __fmul_ru(u.hi, x.enc_scale),
+                                     SR ? rnd[j] : 0u, same);
+      if (!(u.ok && same) || fmaxf(fabsf(u.lo), fabsf(u.hi)) >= amax_f) redo |= 1u << j;
+      m[j] = u.m; v[j] = u.v; ve[j] = u.ve;
+    }
+    if (redo) {  // rare: the canonical weight of undecided elements and maximum candidates
+#pragma unroll
+      for (int j = 0; j < kGroup; ++j) {
+        if ((redo >> j) & 1u) {
+          const float xe = madam_wn_exact(a.s, w[j], g[j], m[j], v[j], ve[j]);
+          const uint32_t wb = __float_as_uint(xe) & 0x7FFFFFFFu;
+          if (j < valid && wb < 0x7F800000u) amax_bits = max(amax_bits, wb);
+          code[j] = e4m3_encode<SR>(__fmul_rn(xe, x.enc_scale), SR ? rnd[j] : 0u);
+        }
+      }
+    }
+    uint32_t ow[2];
+    ow[0] = code[0] | (code[1] << 8) | (code[2] << 16) | (code[3] << 24);
+    ow[1] = code[4] | (code[5] << 8) | (code[6] << 16) | (code[7] << 24);
+    put_e4m3(ow, x.d.w, e0, valid, x.vec);
   } else {
   float wn[8];
 #pragma unroll
