@@ -263,7 +263,8 @@ def summarize(wl, res, n_gpus, peak, peak_kind):
                      "frac": round(achieved / peak, 4), "traffic": recorded_traffic(wl.name),
                      "peak_source": peak_kind, "bytes_per_param": bpp,
                      "kernel": "mpadam::step_kernel", "launch_ms_avg": round(avg_launch, 4),
-                     "launch_ms_min": round(launch[0], 4), "launch_ms_max": round(launch[-1], 4)},
+                     "launch_ms_min": round(launch[0], 4), "launch_ms_max": round(launch[-1], 4),
+                     "launch_ms_first_last": [round(res["launch_ms"][0], 4), round(res["launch_ms"][-1], 4)]},
     }
     if "e2e_ms" in res:
         out["e2e"] = {"value": n_gpus * n / (res["e2e_ms"] * 1e-3) / 1e9, "unit": UNIT,

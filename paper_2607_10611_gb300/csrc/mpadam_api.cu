@@ -77,7 +77,7 @@ void make_scalars(const mpadam_config& c, int64_t t, StepScalars* s) {
   s->wmax = s->wmax_on ? c.w_max : 0.0f;
   s->wd_on = c.wd_add != 0.0f ? 1 : 0;
   s->kwd = static_cast<float>(static_cast<double>(c.lr_add) * static_cast<double>(c.wd_add));
-  s->cert_ok = (c.eps >= 0x1p-125f && c.tau >= 0x1p-125f) ? 1 : 0;
+  s->cert_ok = (c.eps >= 0x1p-28f && c.tau >= 0x1p-125f && s->c2 <= 0x1p14f && c.lr_mul <= 4.0f) ? 1 : 0;
 }
 
 // Philox4x32-10 round keys: key + r * (0x9E3779B9, 0xBB67AE85), r = 0..9.

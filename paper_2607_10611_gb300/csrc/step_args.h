@@ -61,7 +61,7 @@ struct StepScalars {
   float gmax, wmax;  // active when gmax_on / wmax_on
   float kwd;         // eta_a * lambda, active when wd_on
   int32_t gmax_on, wmax_on, wd_on;
-  int32_t cert_ok;   // eps, tau >= 2^-125: the certified fast path may be used
+  int32_t cert_ok;   // eps >= 2^-28, tau >= 2^-125, c2 <= 2^14, eta_m <= 4: certified fast path allowed
 };
 
 struct StepArgs {

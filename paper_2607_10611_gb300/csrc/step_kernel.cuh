@@ -204,15 +204,23 @@ __device__ __forceinline__ Upd madam_update(const StepScalars& s, float w, float
 // elementary mathematical functions with correctly rounded last bit", ACM
 // TOMS 17(3), 1991).  The moments are computed exactly as above; the two
 // square roots and three divisions of the weight update use the hardware
-// approximations sqrt.approx.f32 and div.approx.f32 (__fdividef; CUDA
-// documents at most 2 ulp for divisors in [2^-126, 2^126]).  With every
-// approximate result assumed within 2^-19 relative of the correctly rounded
-// one -- 8x the documented bound -- the fast weight wn' differs from the
-// canonical wn by at most
-//     eps = (|w u_m'| + |u_a'|) 2^-17 + (|w + w u_m'| + |wn'|) 2^-22 + 2^-140
+// approximations sqrt.approx{.ftz}.f32 and div.approx{.ftz}.f32 (CUDA
+// documents at most 2 ulp for approximate division with divisors in
+// [2^-126, 2^126]).
+// With every approximate result assumed within 2^-19 relative of the
+// correctly rounded one -- 8x the documented bound -- plus an absolute 2^-126
+// for an operand or result flushed from the subnormal range, the fast weight
+// wn' differs from the canonical wn by at most
+//     eps = (|w u_m'| + |u_a'|) 2^-17 + (|w + w u_m'| + |wn'|) 2^-22 + 2^-96
 // (the relative errors propagate through the divisions, the clamp is
-// 1-Lipschitz, and each of the two final roundings adds at most one ulp; the
-// constants carry a further factor-of-two margin).  The caller stores the
+// 1-Lipschitz, each of the two final roundings adds at most one ulp, and the
+// constants carry a further factor-of-two margin).  Flushing stays inside
+// the 2^-96 term and the relative terms when eps >= 2^-28, c2 <= 2^14 and
+// eta_m <= 4: a subnormal numerator of u_a or of n moves them by at most
+// 2^-126 / eps <= 2^-98 (and w u_m by at most eta_m 2^-98); a subnormal
+// nu or nu_e moves its denominator by at most c2 2^-63 <= 2^-21 eps; a
+// flushed u_m moves w u_m by at most |w| 2^-126.  The host enables this path
+// only under those conditions (cert_ok); divisors are checked in range here.  The caller stores the
 // encoding of wn' only when encoding wn' - eps (rounded down) and wn' + eps
 // (rounded up) gives the same code: every encoder here is monotone, so the
 // canonical wn, which lies in between, has that code too.  Otherwise the
@@ -220,10 +228,22 @@ __device__ __forceinline__ Upd madam_update(const StepScalars& s, float w, float
 // are therefore identical to the canonical sequence bit for bit; the test
 // only decides how much work that takes.
 // ---------------------------------------------------------------------------
+// FTZ selects the flushing forms.  Both forms are covered by the same bound
+// (flushing is the larger error); which one runs is a measured choice per
+// storage format: the flushing forms for BF16 weights, the others for E4M3.
+template <bool FTZ>
 __device__ __forceinline__ float sqrt_approx(float x) {
   float y;
-  asm("sqrt.approx.f32 %0, %1;" : "=f"(y) : "f"(x));
+  if (FTZ) asm("sqrt.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  else asm("sqrt.approx.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
+}
+template <bool FTZ>
+__device__ __forceinline__ float div_approx(float a, float b) {
+  float q;
+  if (FTZ) asm("div.approx.ftz.f32 %0, %1, %2;" : "=f"(q) : "f"(a), "f"(b));
+  else asm("div.approx.f32 %0, %1, %2;" : "=f"(q) : "f"(a), "f"(b));
+  return q;
 }
 
 struct CertUpd {
@@ -232,6 +252,7 @@ struct CertUpd {
   bool ok;           // divisors in the documented range and wn' finite
 };
 
+template <bool FTZ>
 __device__ __forceinline__ CertUpd madam_update_cert(const StepScalars& s, float w, float g, float m, float v,
                                                      float ve) {
   CertUpd o;
@@ -239,18 +260,18 @@ __device__ __forceinline__ CertUpd madam_update_cert(const StepScalars& s, float
   o.v = __fmaf_rn(s.b2, v, __fmul_rn(s.omb2, __fmul_rn(g, g)));
   const float ge = __fmul_rn(__fmul_rn(s.ln2, w), g);
   o.ve = __fmaf_rn(s.b2, ve, __fmul_rn(s.omb2, __fmul_rn(ge, ge)));
-  const float den_a = __fmaf_rn(sqrt_approx(o.v), s.c2, s.eps);
-  const float ua = __fdividef(__fmul_rn(s.ka, o.m), den_a);
-  const float den_e = __fmaf_rn(sqrt_approx(o.ve), s.c2, s.eps);
-  const float n = __fdividef(ge, den_e);
+  const float den_a = __fmaf_rn(sqrt_approx<FTZ>(o.v), s.c2, s.eps);
+  const float ua = div_approx<FTZ>(__fmul_rn(s.ka, o.m), den_a);
+  const float den_e = __fmaf_rn(sqrt_approx<FTZ>(o.ve), s.c2, s.eps);
+  const float n = div_approx<FTZ>(ge, den_e);
   const float rho = fmaxf(fabsf(w), s.tau);
-  float um = __fdividef(__fmul_rn(s.km, n), rho);
+  float um = div_approx<FTZ>(__fmul_rn(s.km, n), rho);
   um = fmaxf(s.lo, fminf(um, s.hi));
   const float t = __fmaf_rn(w, um, w);
   o.wn = __fadd_rn(t, ua);
   const float e = __fmaf_rn(__fadd_rn(fabsf(__fmul_rn(w, um)), fabsf(ua)), 7.62939453125e-06f /* 2^-17 */,
                             __fmaf_rn(__fadd_rn(fabsf(t), fabsf(o.wn)), 2.384185791015625e-07f /* 2^-22 */,
-                                      7.174648137343064e-43f /* 2^-140 */));
+                                      1.2621774483536189e-29f /* 2^-96 */));
   o.lo = __fsub_rd(o.wn, e);
   o.hi = __fadd_ru(o.wn, e);
   // divisors must stay below 2^125 (their lower bounds eps, tau >= 2^-125 are
@@ -552,7 +573,7 @@ __device__ __forceinline__ void finish_group(const StepArgs& a, const TensorCtx&
     uint32_t redo = 0u;
 #pragma unroll
     for (int j = 0; j < kGroup; ++j) {
-      const CertUpd u = madam_update_cert(a.s, w[j], g[j], m[j], v[j], ve[j]);
+      const CertUpd u = madam_update_cert<true>(a.s, w[j], g[j], m[j], v[j], ve[j]);
       bool same;
       if (SR) {
         const uint32_t slo = __float_as_uint(u.lo) + rnd[j], shi = __float_as_uint(u.hi) + rnd[j];
@@ -589,7 +610,7 @@ __device__ __forceinline__ void finish_group(const StepArgs& a, const TensorCtx&
     const float amax_f = __uint_as_float(amax_bits);
 #pragma unroll
     for (int j = 0; j < kGroup; ++j) {
-      const CertUpd u = madam_update_cert(a.s, w[j], g[j], m[j], v[j], ve[j]);
+      const CertUpd u = madam_update_cert<false>(a.s, w[j], g[j], m[j], v[j], ve[j]);
       bool same;
       code[j] = e4m3_pair_normal<SR>(__fmul_rd(u.lo, x.enc_scale), __fmul_ru(u.hi, x.enc_scale),
                                      SR ? rnd[j] : 0u, same);

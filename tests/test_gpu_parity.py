@@ -101,6 +101,8 @@ def test_flat_layout_matches():
     dict(g_max=0.7), dict(w_max=0.03), dict(wd_add=0.1), dict(dmult_max=0.02),
     dict(bias_correction=0), dict(lr_mul=0.0), dict(lr_add=0.0), dict(lr_mul=0.5, lr_add=0.05),
     dict(g_max=0.5, w_max=0.05, wd_add=0.01, dmult_max=0.1, rmax_neg=0.6, rmax_pos=0.5, tau=1e-3),
+    # outside the certified fast path's conditions: the exact sequence runs throughout
+    dict(eps=1e-10), dict(lr_mul=5.0), dict(beta2=0.9999999),
 ])
 @pytest.mark.parametrize("name", ["gpt2_124m", "llama_1p5b"])
 def test_algorithm2_options(hp, name):
