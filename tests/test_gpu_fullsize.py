@@ -1,0 +1,180 @@
+"""Parity at the full workload sizes, in the launch configuration bench.py
+times (default grid, flat layout, inputs drawn on the GPU).
+
+- flat_1m: every element, all 10 steps, against the oracle.
+- the four large lists: about a million sampled elements per step (random
+  positions plus each tensor's first and last elements), run through the
+  oracle one by one with their global indices.  Step 2 continues from the
+  oracle's own step-1 results on those elements (which equal the GPU's bit
+  for bit, checked first), so no oracle input ever comes from the CUDA path.
+- llama_1p5b (E4M3): the scale state depends on whole tensors, so step 1 is
+  checked on samples with the amax the oracle computes from the stored codes,
+  and two steps are checked on whole tensors (norm gains, a 4M matrix, the
+  final norm), where the oracle also reproduces the recorded amax.
+"""
+import gc
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import workloads as W
+
+pytestmark = pytest.mark.gpu
+
+ODT = {"f32": oracle.F32, "bf16": oracle.BF16, "e4m3": oracle.E4M3}
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    from paper_2607_10611_gb300 import build
+    build()
+
+
+def _bits(t: torch.Tensor) -> np.ndarray:
+    t = t.cpu()
+    if t.dtype == torch.bfloat16:
+        return t.view(torch.int16).numpy().view(np.uint16).copy()
+    return t.numpy().copy()
+
+
+def _free():
+    gc.collect()
+    torch.cuda.synchronize()
+    torch.cuda.empty_cache()
+
+
+def _setup(wl):
+    from paper_2607_10611_gb300.optimizer import MPAdam
+    mt = W.materialize(wl, "cuda", layout="flat")
+    opt = MPAdam(mt.w, mt.m, mt.v, mt.ve, weight_dtype=wl.weight_dtype, grad_dtype=wl.grad_dtype,
+                 moment_dtype=wl.moment_dtype, rounding=wl.rounding, seed=wl.seed, fp8_exp=mt.fp8_exp)
+    return mt, opt
+
+
+def _sample_positions(mt, n_random, seed):
+    rng = np.random.default_rng(seed)
+    numels = np.array([t.numel() for t in mt.w], dtype=np.int64)
+    offs = np.array(mt.offsets, dtype=np.int64)
+    heads = np.concatenate([offs[k] + np.arange(min(4, n)) for k, n in enumerate(numels) if n])
+    tails = np.concatenate([offs[k] + np.arange(max(0, n - 4), n) for k, n in enumerate(numels) if n])
+    # random elements, weighted by size, mapped into the padded global space
+    cum = np.cumsum(numels)
+    flat = rng.integers(0, cum[-1], n_random)
+    k = np.searchsorted(cum, flat, side="right")
+    within = flat - np.concatenate([[0], cum[:-1]])[k]
+    pos = np.unique(np.concatenate([heads, tails, offs[k] + within]))
+    tens = np.searchsorted(offs, pos, side="right") - 1
+    return pos, tens
+
+
+def _gather(mt, pos):
+    p = torch.from_numpy(pos).to("cuda")
+    return {key: _bits(mt.flat[key].index_select(0, p)) for key in ("w", "g", "m", "v", "ve")}
+
+
+def _oracle_step(wl, host, pos, t, hp, e_cur=0, e_next=0):
+    oracle.step_elements(hp, t, ODT[wl.weight_dtype], ODT[wl.grad_dtype], ODT[wl.moment_dtype],
+                         host["w"], host["g"], host["m"], host["v"], host["ve"], gidx=pos,
+                         e_cur=e_cur, e_next=e_next)
+
+
+def _assert_same(got, want, what):
+    for key in ("w", "m", "v", "ve"):
+        a, b = got[key], want[key]
+        eq = a.view(a.dtype) == b.view(b.dtype)
+        if a.dtype == np.float32:
+            eq = (a.view(np.uint32) == b.view(np.uint32)) | (np.isnan(a) & np.isnan(b))
+        bad = int((~eq).sum())
+        assert bad == 0, f"{what}: {bad} of {a.size} sampled {key} differ"
+
+
+def test_flat_1m_every_element_all_steps():
+    wl = W.CONFIGS["flat_1m"]
+    mt, opt = _setup(wl)
+    hp = oracle.hparams(stochastic=0, seed=wl.seed)
+    pos = np.arange(mt.w[0].numel(), dtype=np.int64)
+    host = _gather(mt, pos)
+    for t in range(1, wl.steps + 1):
+        opt.step(mt.g, t)
+        _oracle_step(wl, host, pos, t, hp)
+        _assert_same(_gather(mt, pos), host, f"flat_1m step {t}")
+    assert opt.device_status() == 0
+    opt.close()
+    del mt, opt
+    _free()
+
+
+@pytest.mark.parametrize("name,rounding", [("gpt2_124m", None), ("llama_7b", None),
+                                           ("ragged_20k", "nearest"), ("ragged_20k", "stochastic")])
+def test_large_bf16_lists_sampled_two_steps(name, rounding):
+    wl = W.CONFIGS[name]
+    if rounding:
+        wl = W.replace(wl, rounding=rounding)
+    mt, opt = _setup(wl)
+    hp = oracle.hparams(stochastic=1 if wl.rounding == "stochastic" else 0, seed=wl.seed)
+    pos, _ = _sample_positions(mt, 1_000_000, seed=7)
+    host = _gather(mt, pos)
+    for t in (1, 2):
+        opt.step(mt.g, t)
+        _oracle_step(wl, host, pos, t, hp)
+        _assert_same(_gather(mt, pos), host, f"{name} step {t}")
+    assert opt.device_status() == 0
+    opt.close()
+    del mt, opt
+    _free()
+
+
+def test_llama_1p5b_e4m3():
+    wl = W.CONFIGS["llama_1p5b"]
+    mt, opt = _setup(wl)
+    hp = oracle.hparams(stochastic=1, seed=wl.seed)
+    n = len(mt.w)
+    # the oracle's own scale state before step 1: largest |decoded stored weight|
+    st = [[mt.fp8_exp[k], oracle.e4m3_amax(_bits(mt.w[k]), mt.fp8_exp[k])] for k in range(n)]
+    a_gpu = opt.fp8_amax(1).cpu().numpy()
+    assert all(np.float32(a_gpu[k]) == np.float32(st[k][1]) for k in range(n))
+
+    # whole tensors for two steps: two norm gains, one 2048x2048 matrix, the final norm
+    whole = [1 + 7, 1 + 1, 1 + 9 * 3 + 7, n - 2]
+    whole_host = {k: {key: _bits(getattr(mt, key)[k]) for key in ("w", "g", "m", "v", "ve")} for k in whole}
+    whole_state = {k: list(st[k]) for k in whole}
+
+    # sampled elements over every tensor, step 1
+    pos, tens = _sample_positions(mt, 1_000_000, seed=11)
+    host = _gather(mt, pos)
+    opt.step(mt.g, 1)
+    torch.cuda.synchronize()
+    for k in np.unique(tens):
+        sel = tens == k
+        sub = {key: np.ascontiguousarray(host[key][sel]) for key in host}
+        e_next = oracle.fp8_next_exponent(st[k][1], st[k][0])
+        _oracle_step(wl, sub, pos[sel], 1, hp, e_cur=st[k][0], e_next=e_next)
+        for key in host:
+            host[key][sel] = sub[key]
+    _assert_same(_gather(mt, pos), host, "llama_1p5b step 1 (sampled)")
+
+    # whole tensors: step 1 then step 2, including the recorded scale state
+    for t in (1, 2):
+        if t == 2:
+            opt.step(mt.g, 2)
+            torch.cuda.synchronize()
+        exps = opt.fp8_exponents(t + 1)
+        amax = opt.fp8_amax(t + 1).cpu().numpy()
+        for k in whole:
+            h = whole_host[k]
+            e_cur, a_cur = whole_state[k]
+            e_next = oracle.fp8_next_exponent(a_cur, e_cur)
+            a_next = oracle.step_elements(hp, t, oracle.E4M3, ODT[wl.grad_dtype], ODT[wl.moment_dtype],
+                                          h["w"], h["g"], h["m"], h["v"], h["ve"], gidx0=mt.offsets[k],
+                                          e_cur=e_cur, e_next=e_next)
+            whole_state[k] = [e_next, a_next]
+            got = {key: _bits(getattr(mt, key)[k]) for key in ("w", "m", "v", "ve")}
+            _assert_same(got, h, f"llama_1p5b tensor {k} step {t}")
+            assert exps[k] == e_next
+            assert np.float32(amax[k]).view(np.uint32) == np.float32(a_next).view(np.uint32)
+    assert opt.device_status() == 0
+    opt.close()
+    del mt, opt
+    _free()
