@@ -279,9 +279,9 @@ def main():
     ap.add_argument("--steps", type=int, default=50)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--config", default="llama_7b")
-    ap.add_argument("--secondary", default="llama_1p5b", help="'' to skip")
+    ap.add_argument("--secondary", default="llama_1p5b,gpt2_124m,ragged_20k", help="'' to skip")
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--e2e-steps", type=int, default=3)
+    ap.add_argument("--e2e-steps", type=int, default=5)
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--max-params", type=int, default=0,
                     help="truncate the list to its first N params (small profiling cases)")

@@ -167,12 +167,19 @@ int32_t mpadam_step(mpadam_state* s, const void* const* grads, int64_t step,
 
 /* The same step with gradients and weights in host memory: copies
  * host_grads[k] (numel[k] gradients each) to library-owned device staging,
- * runs mpadam_step, and copies every updated weight tensor back to
- * host_w_out[k] (numel[k] weights of weight_dtype each), all on `stream`.
- * For overlap the host buffers should be pinned.  When host_grads[k] (or
- * host_w_out[k] and the device weights) follow the global-index layout of
- * one flat buffer, a single copy moves them all.  The first call allocates
- * the staging buffer.  Errors: EINVAL, EALLOC, ECUDA. */
+ * runs the step, and copies every updated weight tensor back to
+ * host_w_out[k] (numel[k] weights of weight_dtype each).  The host buffers
+ * should be pinned.  When host_grads, host_w_out and the device weights each
+ * follow the global-index layout of one flat allocation (pointer k = base +
+ * off[k] * element size), the step is pipelined in up to 8 chunks of whole
+ * tiles: chunk c's gradients upload on an internal stream while chunk c-1 is
+ * stepped on `stream` and chunk c-2's weights download on a second internal
+ * stream (copies cover each chunk's whole global-index range, padding
+ * included); otherwise the copies are one per tensor, before and after the
+ * step.  Either way the work is ordered after earlier work on `stream`, and
+ * `stream` completes only after the last download.  The first call allocates
+ * the staging buffer and the pipeline's streams and events.
+ * Errors: EINVAL, EALLOC, ECUDA. */
 int32_t mpadam_step_host(mpadam_state* s, const void* const* host_grads, void* const* host_w_out,
                          int64_t step, struct CUstream_st* stream);
 

@@ -162,8 +162,8 @@ int32_t make_geometry(const mpadam_config& c, int dev, Geometry* g) {
 __global__ void __launch_bounds__(mpadam::kConsumers) fp8_amax_kernel(const __grid_constant__ StepArgs a,
                                                                       int32_t exp_slot, int32_t amax_slot) {
   const int64_t T = a.total_tiles;
-  const int64_t tb = (int64_t)blockIdx.x * T / gridDim.x;
-  const int64_t te = ((int64_t)blockIdx.x + 1) * T / gridDim.x;
+  const int64_t tb = a.tile_base + (int64_t)blockIdx.x * T / gridDim.x;
+  const int64_t te = a.tile_base + ((int64_t)blockIdx.x + 1) * T / gridDim.x;
   if (tb >= te) return;
   const int n = a.n_tensors;
   int k = a.cta_first[blockIdx.x];
@@ -256,6 +256,12 @@ struct mpadam_state {
   uint32_t* fp8_amax = nullptr;
   char* d_gstage = nullptr;  // mpadam_step_host gradient staging (global-index layout)
   std::vector<const void*> stage_ptrs;
+  // mpadam_step_host pipeline: chunks of whole tiles, copied and stepped in turn
+  cudaStream_t s_h2d = nullptr, s_d2h = nullptr;
+  std::vector<cudaEvent_t> ev;                // per chunk: h2d done, kernel done; plus start / end
+  std::vector<int64_t> chunk_tile;            // chunk c covers tiles [chunk_tile[c], chunk_tile[c+1])
+  std::vector<int64_t> chunk_elem;            // and global elements [chunk_elem[2c], chunk_elem[2c+1])
+  int32_t* d_chunk_first = nullptr;           // [chunks][grid] CTA start tensors
 };
 
 namespace {
@@ -267,6 +273,10 @@ void release(mpadam_state* s) {
   if (s->d_cta_first) cudaFree(s->d_cta_first);
   if (s->d_err) cudaFree(s->d_err);
   if (s->d_gstage) cudaFree(s->d_gstage);
+  if (s->d_chunk_first) cudaFree(s->d_chunk_first);
+  for (cudaEvent_t e : s->ev) cudaEventDestroy(e);
+  if (s->s_h2d) cudaStreamDestroy(s->s_h2d);
+  if (s->s_d2h) cudaStreamDestroy(s->s_d2h);
   if (s->h_grads) cudaFreeHost(const_cast<void**>(s->h_grads));
   if (s->upload_done) cudaEventDestroy(s->upload_done);
   delete s;
@@ -274,12 +284,14 @@ void release(mpadam_state* s) {
 
 int64_t tiles_of(int64_t numel) { return (numel + mpadam::kTile - 1) / mpadam::kTile; }
 
-// Tensor holding each CTA's first tile (n when the CTA has no tiles).
-void cta_first_table(const int64_t* numel, int32_t n, int64_t total_tiles, int32_t grid, int32_t* first) {
+// Tensor holding each CTA's first tile of the range [tile_base, tile_base +
+// total_tiles) (n when the CTA has no tiles).
+void cta_first_table(const int64_t* numel, int32_t n, int64_t total_tiles, int32_t grid, int32_t* first,
+                     int64_t tile_base = 0) {
   int32_t k = 0;
   int64_t tile_off = 0;
   for (int32_t b = 0; b < grid; ++b) {
-    const int64_t tb = (int64_t)b * total_tiles / grid;
+    const int64_t tb = tile_base + (int64_t)b * total_tiles / grid;
     while (k < n && tile_off + tiles_of(numel[k]) <= tb) {
       tile_off += tiles_of(numel[k]);
       ++k;
@@ -366,6 +378,90 @@ int32_t check_device(const mpadam_state* s) {
   if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
   if (dev != s->device)
     return fail(MPADAM_EINVAL, "current device %d differs from the state's device %d", dev, s->device);
+  return MPADAM_OK;
+}
+
+}  // namespace
+
+
+namespace {
+
+// Re-upload the gradient pointer table when it differs from the last one.
+int32_t upload_grad_table(mpadam_state* s, const void* const* grads, cudaStream_t stream) {
+  cudaError_t e;
+  if (s->grads_uploaded && std::memcmp(s->last_grads.data(), grads, sizeof(void*) * s->n) == 0) return MPADAM_OK;
+  if (s->upload_pending) {  // the pinned table may still be read by the last copy
+    e = cudaEventSynchronize(s->upload_done);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaEventSynchronize");
+  }
+  std::memcpy(s->h_grads, grads, sizeof(void*) * s->n);
+  e = cudaMemcpyAsync(s->d_grads, s->h_grads, sizeof(void*) * s->n, cudaMemcpyHostToDevice, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "upload of the gradient table");
+  e = cudaEventRecord(s->upload_done, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
+  s->upload_pending = true;
+  std::memcpy(s->last_grads.data(), grads, sizeof(void*) * s->n);
+  s->grads_uploaded = true;
+  return MPADAM_OK;
+}
+
+// One launch of the step kernel over tiles [tile_base, tile_base + count).
+int32_t launch_step(mpadam_state* s, int64_t step, cudaStream_t stream, int64_t tile_base, int64_t count,
+                    const int32_t* cta_first, int32_t grid) {
+  StepArgs a = base_args(s);
+  a.cta_first = cta_first;
+  a.tile_base = tile_base;
+  a.total_tiles = count;
+  fill_step(a, s->cfg, step);
+  void* params[] = {&a};
+  cudaError_t e = cudaLaunchKernel(s->kernel, dim3(grid), dim3(mpadam::kThreads), params, (size_t)s->geo.dyn_smem,
+                                   stream);
+  if (e != cudaSuccess) return cuda_fail(e, "launch of the step kernel");
+  return MPADAM_OK;
+}
+
+// Global element index of a tile's first element, and one past its last.
+void tile_elements(const mpadam_state* s, int64_t t, int64_t* first, int64_t* end) {
+  const auto it = std::upper_bound(s->tile_off.begin(), s->tile_off.end(), t);
+  int32_t k = (int32_t)(it - s->tile_off.begin()) - 1;
+  while (tiles_of(s->numel[k]) == 0 || t >= s->tile_off[k] + tiles_of(s->numel[k])) ++k;
+  const int64_t j = t - s->tile_off[k];
+  *first = s->goff[k] + j * mpadam::kTile;
+  *end = s->goff[k] + std::min<int64_t>((j + 1) * mpadam::kTile, s->numel[k]);
+}
+
+// The host-buffer pipeline: chunks of whole tiles, their CTA tables, two
+// copy streams and the events that order them (created on first use).
+int32_t prepare_pipeline(mpadam_state* s) {
+  if (!s->chunk_tile.empty()) return MPADAM_OK;
+  const int32_t chunks = (int32_t)std::max<int64_t>(1, std::min<int64_t>(8, s->tiles / 256));  // 8: best measured
+  std::vector<int64_t> ct(chunks + 1), ce(2 * (size_t)chunks);
+  for (int32_t c = 0; c <= chunks; ++c) ct[c] = (int64_t)c * s->tiles / chunks;
+  for (int32_t c = 0; c < chunks; ++c) {
+    int64_t f0, e0, f1, e1;
+    tile_elements(s, ct[c], &f0, &e0);
+    tile_elements(s, ct[c + 1] - 1, &f1, &e1);
+    ce[2 * c] = f0;
+    ce[2 * c + 1] = e1;
+  }
+  std::vector<int32_t> first((size_t)chunks * s->grid);
+  for (int32_t c = 0; c < chunks; ++c)
+    cta_first_table(s->numel.data(), s->n, ct[c + 1] - ct[c], s->grid, first.data() + (size_t)c * s->grid, ct[c]);
+  if (cudaMalloc(&s->d_chunk_first, sizeof(int32_t) * first.size()) != cudaSuccess)
+    return fail(MPADAM_EALLOC, "cudaMalloc of the chunk tables failed");
+  cudaError_t e = cudaMemcpy(s->d_chunk_first, first.data(), sizeof(int32_t) * first.size(), cudaMemcpyHostToDevice);
+  if (e != cudaSuccess) return cuda_fail(e, "upload of the chunk tables");
+  e = cudaStreamCreateWithFlags(&s->s_h2d, cudaStreamNonBlocking);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaStreamCreate");
+  e = cudaStreamCreateWithFlags(&s->s_d2h, cudaStreamNonBlocking);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaStreamCreate");
+  s->ev.resize(2 * (size_t)chunks + 2);
+  for (auto& ev : s->ev) {
+    e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaEventCreate");
+  }
+  s->chunk_tile = ct;
+  s->chunk_elem = ce;
   return MPADAM_OK;
 }
 
@@ -531,29 +627,9 @@ int32_t mpadam_step(mpadam_state* s, const void* const* grads, int64_t step, cud
   }
   int32_t rc = check_device(s);
   if (rc) return rc;
-
-  cudaError_t e;
-  if (!s->grads_uploaded || std::memcmp(s->last_grads.data(), grads, sizeof(void*) * s->n) != 0) {
-    if (s->upload_pending) {  // the pinned table may still be read by the last copy
-      e = cudaEventSynchronize(s->upload_done);
-      if (e != cudaSuccess) return cuda_fail(e, "cudaEventSynchronize");
-    }
-    std::memcpy(s->h_grads, grads, sizeof(void*) * s->n);
-    e = cudaMemcpyAsync(s->d_grads, s->h_grads, sizeof(void*) * s->n, cudaMemcpyHostToDevice, stream);
-    if (e != cudaSuccess) return cuda_fail(e, "upload of the gradient table");
-    e = cudaEventRecord(s->upload_done, stream);
-    if (e != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
-    s->upload_pending = true;
-    std::memcpy(s->last_grads.data(), grads, sizeof(void*) * s->n);
-    s->grads_uploaded = true;
-  }
-
-  StepArgs a = base_args(s);
-  fill_step(a, s->cfg, step);
-  void* params[] = {&a};
-  e = cudaLaunchKernel(s->kernel, dim3(s->grid), dim3(mpadam::kThreads), params, (size_t)s->geo.dyn_smem, stream);
-  if (e != cudaSuccess) return cuda_fail(e, "launch of the step kernel");
-  return MPADAM_OK;
+  rc = upload_grad_table(s, grads, stream);
+  if (rc) return rc;
+  return launch_step(s, step, stream, 0, s->tiles, s->d_cta_first, s->grid);
 }
 
 int32_t mpadam_fp8_init(mpadam_state* s, const int32_t* init_exp, int64_t first_step, cudaStream_t stream) {
@@ -649,6 +725,43 @@ int32_t mpadam_step_host(mpadam_state* s, const void* const* host_grads, void* c
   const size_t lo_e = (size_t)s->goff[first], hi_e = (size_t)(s->goff[last] + s->numel[last]);
 
   const char* hb = nullptr;
+  const char* dw0 = nullptr;
+  const char* hw0 = nullptr;
+  if (flat_base(host_grads, gsz, &hb) && flat_base(s->w.data(), wsz, &dw0) && flat_base(host_w_out, wsz, &hw0)) {
+    // Pipelined: chunk c's gradients upload on s_h2d, its step runs on
+    // `stream` after them, its weights download on s_d2h after the step.
+    rc = prepare_pipeline(s);
+    if (rc) return rc;
+    rc = upload_grad_table(s, s->stage_ptrs.data(), stream);
+    if (rc) return rc;
+    const int32_t chunks = (int32_t)s->chunk_tile.size() - 1;
+    cudaEvent_t ev_start = s->ev[2 * chunks], ev_end = s->ev[2 * chunks + 1];
+    // the copies must not overtake earlier work on `stream` (a previous step
+    // still reading the staging buffer or writing the weights)
+    if ((e = cudaEventRecord(ev_start, stream)) != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
+    if ((e = cudaStreamWaitEvent(s->s_h2d, ev_start, 0)) != cudaSuccess) return cuda_fail(e, "cudaStreamWaitEvent");
+    if ((e = cudaStreamWaitEvent(s->s_d2h, ev_start, 0)) != cudaSuccess) return cuda_fail(e, "cudaStreamWaitEvent");
+    for (int32_t c = 0; c < chunks; ++c) {
+      const size_t a0 = (size_t)s->chunk_elem[2 * c], a1 = (size_t)s->chunk_elem[2 * c + 1];
+      e = cudaMemcpyAsync(s->d_gstage + a0 * gsz, hb + a0 * gsz, (a1 - a0) * gsz, cudaMemcpyHostToDevice, s->s_h2d);
+      if (e != cudaSuccess) return cuda_fail(e, "gradient upload");
+      if ((e = cudaEventRecord(s->ev[2 * c], s->s_h2d)) != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
+      if ((e = cudaStreamWaitEvent(stream, s->ev[2 * c], 0)) != cudaSuccess) return cuda_fail(e, "cudaStreamWaitEvent");
+      rc = launch_step(s, step, stream, s->chunk_tile[c], s->chunk_tile[c + 1] - s->chunk_tile[c],
+                       s->d_chunk_first + (size_t)c * s->grid, s->grid);
+      if (rc) return rc;
+      if ((e = cudaEventRecord(s->ev[2 * c + 1], stream)) != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
+      if ((e = cudaStreamWaitEvent(s->s_d2h, s->ev[2 * c + 1], 0)) != cudaSuccess)
+        return cuda_fail(e, "cudaStreamWaitEvent");
+      e = cudaMemcpyAsync(const_cast<char*>(hw0) + a0 * wsz, dw0 + a0 * wsz, (a1 - a0) * wsz, cudaMemcpyDeviceToHost,
+                          s->s_d2h);
+      if (e != cudaSuccess) return cuda_fail(e, "weight download");
+    }
+    // `stream` completes only after every download
+    if ((e = cudaEventRecord(ev_end, s->s_d2h)) != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
+    if ((e = cudaStreamWaitEvent(stream, ev_end, 0)) != cudaSuccess) return cuda_fail(e, "cudaStreamWaitEvent");
+    return MPADAM_OK;
+  }
   if (flat_base(host_grads, gsz, &hb)) {
     e = cudaMemcpyAsync(s->d_gstage + lo_e * gsz, hb + lo_e * gsz, (hi_e - lo_e) * gsz,
                         cudaMemcpyHostToDevice, stream);

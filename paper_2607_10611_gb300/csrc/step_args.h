@@ -68,6 +68,7 @@ struct StepArgs {
   const TensorDesc* desc;    // [n_tensors]
   const void* const* grads;  // [n_tensors] device pointers
   const int32_t* cta_first;  // [gridDim.x] tensor holding each CTA's first tile
+  int64_t tile_base;         // this launch covers tiles [tile_base, tile_base + total_tiles)
   int64_t total_tiles;
   int32_t n_tensors;
   int32_t stages;            // shared-memory pipeline depth (2..kMaxStages)

@@ -735,8 +735,8 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
   __syncthreads();
 
   const int64_t T = a.total_tiles;
-  const int64_t tb = static_cast<int64_t>(blockIdx.x) * T / gridDim.x;
-  const int64_t te = (static_cast<int64_t>(blockIdx.x) + 1) * T / gridDim.x;
+  const int64_t tb = a.tile_base + static_cast<int64_t>(blockIdx.x) * T / gridDim.x;
+  const int64_t te = a.tile_base + (static_cast<int64_t>(blockIdx.x) + 1) * T / gridDim.x;
   if (tb >= te) return;
   const uint32_t smem0 = smem_addr(smem);
 
