@@ -248,6 +248,19 @@ def run_gpu(wl, steps: int, warmup: int, rank: int, e2e_steps: int):
     return res
 
 
+def max_over_ranks(ms: float, device: str) -> float:
+    """The slowest rank's timed-region length (every rank gets it)."""
+    import torch
+    t = torch.tensor([ms], dtype=torch.float64, device=device)
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(params_per_rank: int, ranks: int, ms_per_step: float) -> float:
+    """Whole-job Gparams/s: every rank steps its own replica (weak scaling)."""
+    return ranks * params_per_rank / (ms_per_step * 1e-3) / 1e9
+
+
 def summarize(wl, res, n_gpus, peak, peak_kind):
     n = wl.n_params
     ms = res["total_ms"] / len(res["launch_ms"])
@@ -257,7 +270,7 @@ def summarize(wl, res, n_gpus, peak, peak_kind):
     achieved = bpp * n / (avg_launch * 1e-3) / 1e9
     out = {
         "workload": wl.name, "params": n, "tensors": len(wl.specs),
-        "ms_per_step": ms, "gparams_per_s": n_gpus * n / (ms * 1e-3) / 1e9,
+        "ms_per_step": ms, "gparams_per_s": whole_job_rate(n, n_gpus, ms),
         "hbm_gbs": bpp * n / (ms * 1e-3) / 1e9,
         "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
                      "frac": round(achieved / peak, 4), "traffic": recorded_traffic(wl.name),
@@ -333,12 +346,8 @@ def main():
     time.sleep(0.3 if sampler else 0)
 
     res = run_gpu(wl, args.steps, warmup, rank, args.e2e_steps if rank == 0 else 0)
-    total_ms = res["total_ms"]
     if world > 1:
-        tt = torch.tensor([total_ms], device="cuda")
-        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
-        total_ms = float(tt.item())
-        res["total_ms"] = total_ms
+        res["total_ms"] = max_over_ranks(res["total_ms"], "cuda")
     clocks = sampler.summary(*res["wall"]) if sampler else None
     main_sum = summarize(wl, res, world, peak, peak_kind)
 
