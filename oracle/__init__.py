@@ -20,9 +20,10 @@ import numpy as np
 
 from . import build as _build
 
-F32, BF16, E4M3 = 0, 1, 2
-DTYPES = {"f32": F32, "bf16": BF16, "e4m3": E4M3}
+F32, BF16, E4M3, E4M3_B32 = 0, 1, 2, 3
+DTYPES = {"f32": F32, "bf16": BF16, "e4m3": E4M3, "e4m3_b32": E4M3_B32}
 ALIGN = 8
+BLOCK = 32
 
 _LIB = None
 
@@ -89,6 +90,12 @@ def lib() -> ctypes.CDLL:
         L.orc_philox_n.argtypes = [i64, P, P, P]
         L.orc_update_elements_n.argtypes = [P, i64, i64, P, P, P, P, P, P, P, P, P]
         L.orc_update_elements_n.restype = i32
+        L.orc_fp16_pow2.argtypes = [i32]; L.orc_fp16_pow2.restype = ctypes.c_uint16
+        L.orc_fp16_decode.argtypes = [ctypes.c_uint16]; L.orc_fp16_decode.restype = ctypes.c_float
+        L.orc_block_exponent.argtypes = [ctypes.c_float, i32]; L.orc_block_exponent.restype = i32
+        L.orc_step_block_e4m3.argtypes = [i64, i64, i32, i32, P, P, P, P, P, P, P, i64]
+        L.orc_step_block_e4m3.restype = i32
+        L.orc_dequant_bf16.argtypes = [i64, P, i32, P, P]
         _LIB = L
     return _LIB
 
@@ -201,6 +208,40 @@ def step_elements(hp: HParams, t: int, wdt: int, gdt: int, mdt: int, w, g, m, v,
     return float(amax.value)
 
 
+def fp16_pow2(k: int) -> int:
+    """FP16 bits of 2^k, k clamped to [-24, 15]."""
+    return int(lib().orc_fp16_pow2(int(k)))
+
+
+def fp16_decode(h) -> np.ndarray:
+    return np.array([lib().orc_fp16_decode(int(x)) for x in np.atleast_1d(h)], np.float32)
+
+
+def block_exponent(amax: float, k_old: int) -> int:
+    return int(lib().orc_block_exponent(ctypes.c_float(amax), int(k_old)))
+
+
+def step_block_e4m3(hp: HParams, t: int, gdt: int, mdt: int, q, bscale, g, m, v, ve, gidx0: int = 0) -> None:
+    """One step of a whole tensor with per-32-block FP16 power-of-two scales;
+    q (uint8 codes), bscale (uint16 FP16 bits) and the moments update in place."""
+    for a in (q, bscale, g, m, v, ve):
+        assert a.flags.c_contiguous
+    assert bscale.size == -(-q.size // BLOCK)
+    rc = lib().orc_step_block_e4m3(q.size, gidx0, gdt, mdt, _p(q), _p(bscale), _p(g), _p(m), _p(v), _p(ve),
+                                   ctypes.byref(hp), t)
+    if rc != 0:
+        raise ValueError("invalid arguments")
+
+
+def dequant_bf16(q, e: int = 0, bscale=None) -> np.ndarray:
+    """BF16 compute copy of stored E4M3 weights (per-tensor 2^e, or per-block scales)."""
+    q = _c(q, np.uint8)
+    out = np.zeros(q.size, np.uint16)
+    bs = None if bscale is None else _c(bscale, np.uint16)
+    lib().orc_dequant_bf16(q.size, _p(q), int(e), None if bs is None else _p(bs), _p(out))
+    return out
+
+
 def global_offsets(numels) -> List[int]:
     """First global element index of each tensor: the previous tensor's end
     rounded up to a multiple of 8."""
@@ -217,18 +258,26 @@ def fp8_init(tensors, exps: Sequence[int]) -> List[list]:
     return [[int(e), e4m3_amax(t["w"], int(e))] for t, e in zip(tensors, exps)]
 
 
-def step(tensors, *, wdt: int, gdt: int, mdt: int, hp: HParams, t: int,
+def step(tensors, *, wdt, gdt: int, mdt: int, hp: HParams, t: int,
          fp8_state: Optional[List[list]] = None) -> None:
     """One optimizer step over a tensor list.  tensors: list of dicts of 1-D
-    numpy arrays w, g, m, v, ve (updated in place).  For E4M3 storage,
+    numpy arrays w, g, m, v, ve (updated in place).  wdt is the weight format
+    of every tensor, or a list with one format per tensor.  For E4M3 storage,
     fp8_state[k] = [exponent the stored weights use, largest |w| before this
     step]; it is advanced in place: the weights are re-encoded with the
-    exponent chosen from that largest |w|, and the new largest |w| is recorded."""
+    exponent chosen from that largest |w|, and the new largest |w| is recorded.
+    For E4M3_B32 storage the dict also holds "bscale" (FP16 block scales,
+    updated in place)."""
     offs = global_offsets([d["w"].size for d in tensors])
+    formats = list(wdt) if isinstance(wdt, (list, tuple)) else [wdt] * len(tensors)
     for k, d in enumerate(tensors):
+        wdt = formats[k]
         if d["w"].size == 0:
             continue
-        if wdt == E4M3:
+        if wdt == E4M3_B32:
+            step_block_e4m3(hp, t, gdt, mdt, d["w"], d["bscale"], d["g"], d["m"], d["v"], d["ve"],
+                            gidx0=offs[k])
+        elif wdt == E4M3:
             e_cur, a_cur = fp8_state[k]
             e_next = fp8_next_exponent(a_cur, e_cur)
             a_next = step_elements(hp, t, wdt, gdt, mdt, d["w"], d["g"], d["m"], d["v"], d["ve"],

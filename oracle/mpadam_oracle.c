@@ -360,6 +360,93 @@ int32_t orc_step_elements(int64_t n, const int64_t* gidx, int64_t gidx0,
 }
 
 /* ------------------------------------------------------------------------ */
+/* Block-scaled E4M3 (reading of Sec. 5.2 and the FP8-master figure: FP8     */
+/* weights "quantized in blocks with FP16 scales"; block size and scale rule */
+/* are not given).  Blocks are 32 consecutive elements of a tensor; a scale  */
+/* is a power of two (a subset of FP16, so scaling is exact), chosen from    */
+/* the block's own updated weights at each step.                             */
+/* ------------------------------------------------------------------------ */
+uint16_t orc_fp16_pow2(int32_t k) {
+  if (k < -24) k = -24;
+  if (k > 15) k = 15;
+  if (k >= -14) return (uint16_t)((k + 15) << 10);      /* normal: exponent field k + 15 */
+  return (uint16_t)(1u << (k + 24));                     /* subnormal: 2^-24 units */
+}
+
+float orc_fp16_decode(uint16_t h) {
+  uint32_t e = (h >> 10) & 0x1Fu, f = h & 0x3FFu;
+  double val;
+  if (e == 0) val = ldexp((double)f, -24);
+  else if (e == 31) val = f ? NAN : INFINITY;
+  else val = ldexp((double)(1024u + f), (int)e - 25);
+  return (float)((h & 0x8000u) ? -val : val);
+}
+
+int32_t orc_block_exponent(float amax, int32_t k_old) {
+  if (!(amax > 0.0f) || isinf(amax)) return k_old;
+  int x;
+  float f = frexpf(amax, &x);                 /* amax = f 2^x, f in [0.5, 1) */
+  int32_t k = (f <= 0.875f) ? x - 9 : x - 8;  /* smallest k with amax <= 0.875 2^(9+k) */
+  if (k < -24) k = -24;
+  if (k > 15) k = 15;
+  return k;
+}
+
+static int32_t fp16_pow2_exponent(uint16_t h) {
+  uint32_t e = (h >> 10) & 0x1Fu;
+  if (e != 0) return (int32_t)e - 15;
+  int32_t k = -24;
+  for (uint32_t f = h & 0x3FFu; f > 1u; f >>= 1) ++k;
+  return k;
+}
+
+int32_t orc_step_block_e4m3(int64_t n, int64_t gidx0, int32_t gdt, int32_t mdt,
+                            uint8_t* q, uint16_t* bscale, const void* g, void* m, void* v, void* ve,
+                            const orc_hparams* hp, int64_t t) {
+  if (gdt != ORC_F32 && gdt != ORC_BF16) return -1;
+  if (mdt != ORC_F32 && mdt != ORC_BF16) return -1;
+  orc_scalars s;
+  if (orc_scalars_for_step(hp, t, &s) != 0) return -1;
+  for (int64_t b0 = 0; b0 < n; b0 += ORC_BLOCK) {
+    const int64_t bn = (n - b0 < ORC_BLOCK) ? n - b0 : ORC_BLOCK;
+    const int64_t blk = b0 / ORC_BLOCK;
+    const float dec = orc_fp16_decode(bscale[blk]);
+    float wn[ORC_BLOCK];
+    float amax = 0.0f;
+    for (int64_t j = 0; j < bn; ++j) {
+      const int64_t k = b0 + j;
+      float wk = orc_e4m3_decode(q[k]) * dec;
+      float gk = load_elem(g, k, gdt), mk = load_elem(m, k, mdt), vk = load_elem(v, k, mdt);
+      float vek = load_elem(ve, k, mdt);
+      float m1, v1, ve1;
+      orc_update_element(&s, wk, gk, mk, vk, vek, &wn[j], &m1, &v1, &ve1);
+      if (isfinite(wn[j]) && fabsf(wn[j]) > amax) amax = fabsf(wn[j]);
+      store_moment(m, k, mdt, m1);
+      store_moment(v, k, mdt, v1);
+      store_moment(ve, k, mdt, ve1);
+    }
+    /* current scaling: the block's new scale fits its largest updated |w| */
+    const int32_t k_new = orc_block_exponent(amax, fp16_pow2_exponent(bscale[blk]));
+    bscale[blk] = orc_fp16_pow2(k_new);
+    const float enc = ldexpf(1.0f, -k_new);
+    for (int64_t j = 0; j < bn; ++j) {
+      const int64_t k = b0 + j;
+      const float x = wn[j] * enc;
+      q[k] = hp->stochastic ? orc_e4m3_sr(x, orc_rng_lane(hp->seed, (uint64_t)t, (uint64_t)(gidx0 + k), ORC_E4M3))
+                            : orc_e4m3_rne(x);
+    }
+  }
+  return 0;
+}
+
+void orc_dequant_bf16(int64_t n, const uint8_t* q, int32_t e, const uint16_t* bscale, uint16_t* out) {
+  for (int64_t k = 0; k < n; ++k) {
+    const float scale = bscale ? orc_fp16_decode(bscale[k / ORC_BLOCK]) : ldexpf(1.0f, e);
+    out[k] = orc_bf16_rne(orc_e4m3_decode(q[k]) * scale);
+  }
+}
+
+/* ------------------------------------------------------------------------ */
 /* Array helpers for the tests: plain loops over the scalar functions above. */
 /* ------------------------------------------------------------------------ */
 void orc_bf16_rne_n(int64_t n, const float* x, uint16_t* out) {

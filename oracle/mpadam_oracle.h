@@ -23,8 +23,10 @@
 extern "C" {
 #endif
 
-/* Element formats. */
-enum { ORC_F32 = 0, ORC_BF16 = 1, ORC_E4M3 = 2 };
+/* Element formats.  ORC_E4M3_B32: E4M3 codes with one power-of-two scale
+ * per 32 consecutive elements, stored as FP16 bits. */
+enum { ORC_F32 = 0, ORC_BF16 = 1, ORC_E4M3 = 2, ORC_E4M3_B32 = 3 };
+enum { ORC_BLOCK = 32 };
 
 /* Hyper-parameters (Algorithm 1 inputs; Algorithm 2 optional clips). */
 typedef struct {
@@ -94,6 +96,27 @@ int32_t orc_step_elements(int64_t n, const int64_t* gidx, int64_t gidx0,
 
 /* Largest finite |decoded E4M3 weight| of a tensor stored with exponent e. */
 float orc_e4m3_amax(int64_t n, const uint8_t* q, int32_t e);
+
+/* FP16 bit pattern of 2^k, k in [-24, 15] (exact: subnormal below 2^-14). */
+uint16_t orc_fp16_pow2(int32_t k);
+/* Value of an FP16 bit pattern (exact). */
+float orc_fp16_decode(uint16_t h);
+/* Block scale exponent: smallest k with amax <= 448 2^k, clamped to
+ * [-24, 15]; k_old when amax is 0. */
+int32_t orc_block_exponent(float amax, int32_t k_old);
+
+/* One optimizer step over a whole tensor of E4M3 weights with FP16
+ * power-of-two scales per 32-element block (current scaling: each block's
+ * new scale comes from the largest finite |updated weight| of that block).
+ * q: n codes, bscale: ceil(n/32) FP16 scales (both updated in place);
+ * element j has global index gidx0 + j.  Returns 0 or -1. */
+int32_t orc_step_block_e4m3(int64_t n, int64_t gidx0, int32_t gdt, int32_t mdt,
+                            uint8_t* q, uint16_t* bscale, const void* g, void* m, void* v, void* ve,
+                            const orc_hparams* hp, int64_t t);
+
+/* BF16 compute copy of stored E4M3 weights: bf16(decode(q) * scale), exact.
+ * Per-tensor scale 2^e (bscale NULL) or per-32-block FP16 scales. */
+void orc_dequant_bf16(int64_t n, const uint8_t* q, int32_t e, const uint16_t* bscale, uint16_t* out);
 
 /* Array forms of the scalar functions (plain loops), for the tests. */
 void orc_bf16_rne_n(int64_t n, const float* x, uint16_t* out);
