@@ -37,12 +37,26 @@ sys.path.insert(0, str(ROOT))
 
 METRIC = "fused M+Adam step Gparams/s and HBM GB/s as % of GB300 peak (1 GPU)"
 UNIT = "Gparams/s"
-BYTES = {"f32": 4, "bf16": 2, "e4m3": 1}
+BYTES = {"f32": 4, "bf16": 2, "e4m3": 1, "e4m3_b32": 1}
 
 
-def algorithmic_bytes_per_param(wl) -> int:
-    """Reads + writes of one element: w (r+w), g (r), mu, nu, nu_e (r+w)."""
-    return 2 * BYTES[wl.weight_dtype] + BYTES[wl.grad_dtype] + 6 * BYTES[wl.moment_dtype]
+def algorithmic_bytes(wl) -> float:
+    """Reads + writes of one step over the list: per element w (r+w), g (r),
+    mu, nu, nu_e (r+w); per 32-element block of block-scaled E4M3 its FP16
+    scale (r+w); per element of a BF16 compute copy 2 bytes (w)."""
+    total = 0
+    for spec, fmt in zip(wl.specs, wl.formats):
+        n = spec.numel
+        total += n * (2 * BYTES[fmt] + BYTES[wl.grad_dtype] + 6 * BYTES[wl.moment_dtype])
+        if fmt == "e4m3_b32":
+            total += 4 * ((n + 31) // 32)
+        if wl.compute_copy and fmt != "bf16":
+            total += 2 * n
+    return float(total)
+
+
+def algorithmic_bytes_per_param(wl) -> float:
+    return algorithmic_bytes(wl) / wl.n_params
 
 
 def measured_peaks():
@@ -148,7 +162,13 @@ def host_lists(mt):
     import workloads as W
     tensors = [dict(w=W.to_numpy_bits(mt.w[k]), g=W.to_numpy_bits(mt.g[k]), m=W.to_numpy_bits(mt.m[k]),
                     v=W.to_numpy_bits(mt.v[k]), ve=W.to_numpy_bits(mt.ve[k])) for k in range(len(mt.w))]
-    fp8 = oracle.fp8_init(tensors, mt.fp8_exp) if mt.fp8_exp is not None else None
+    for k, b in enumerate(mt.bscale or []):
+        if b is not None:
+            tensors[k]["bscale"] = W.to_numpy_bits(b)
+    fp8 = None
+    if mt.fp8_exp is not None:
+        fp8 = [oracle.fp8_init([tensors[k]], [mt.fp8_exp[k]])[0] if f == "e4m3" else None
+               for k, f in enumerate(mt.formats)]
     return tensors, fp8
 
 
@@ -163,10 +183,16 @@ def time_oracle(wl, target_s: float, t_step: int = 1):
         mt = W.materialize(swl, "cpu")
         tensors, fp8 = host_lists(mt)
         hp = oracle.hparams(stochastic=1 if wl.rounding == "stochastic" else 0, seed=wl.seed)
-        kw = dict(wdt=oracle.DTYPES[wl.weight_dtype], gdt=oracle.DTYPES[wl.grad_dtype],
+        kw = dict(wdt=[oracle.DTYPES[f] for f in mt.formats], gdt=oracle.DTYPES[wl.grad_dtype],
                   mdt=oracle.DTYPES[wl.moment_dtype], hp=hp, t=t_step, fp8_state=fp8)
         t0 = time.perf_counter()
         oracle.step(tensors, **kw)
+        for k, x in enumerate(mt.cc or []):  # the compute copy the step also writes
+            if x is not None:
+                if "bscale" in tensors[k]:
+                    oracle.dequant_bf16(tensors[k]["w"], bscale=tensors[k]["bscale"])
+                else:
+                    oracle.dequant_bf16(tensors[k]["w"], e=fp8[k][0])
         dt = time.perf_counter() - t0
         rate = got / dt
         if dt >= 0.5 * target_s or got < n:
@@ -186,9 +212,12 @@ def run_gpu(wl, steps: int, warmup: int, rank: int, e2e_steps: int):
     build()
     dev = torch.device("cuda", torch.cuda.current_device())
     mt = W.materialize(wl, dev, layout="flat")
-    opt = MPAdam(mt.w, mt.m, mt.v, mt.ve, weight_dtype=wl.weight_dtype, grad_dtype=wl.grad_dtype,
-                 moment_dtype=wl.moment_dtype, rounding=wl.rounding, seed=wl.seed + rank,
-                 fp8_exp=mt.fp8_exp)
+    extended = wl.weight_dtype not in ("bf16", "e4m3") or wl.compute_copy
+    opt = MPAdam(mt.w, mt.m, mt.v, mt.ve, weight_dtype=mt.formats if extended else wl.weight_dtype,
+                 grad_dtype=wl.grad_dtype, moment_dtype=wl.moment_dtype, rounding=wl.rounding,
+                 seed=wl.seed + rank, fp8_exp=mt.fp8_exp, block_scales=mt.bscale if extended else None,
+                 compute=mt.cc if extended else None)
+    launches_per_step = len(set(mt.formats))
     stream = torch.cuda.current_stream(dev)
     gptrs = [g.data_ptr() for g in mt.g]
     t = 1
@@ -217,10 +246,10 @@ def run_gpu(wl, steps: int, warmup: int, rank: int, e2e_steps: int):
     total_ms = region0.elapsed_time(region1)
     launch_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
     res = {"total_ms": total_ms, "launch_ms": launch_ms, "wall": (wall0, wall1),
-           "grid": opt.launch_info()}
+           "grid": opt.launch_info(), "launches_per_step": launches_per_step}
 
-    # end to end through the host-buffer entry point
-    if e2e_steps > 0:
+    # end to end through the host-buffer entry point (one weight format: flat host buffers)
+    if e2e_steps > 0 and "w" in mt.flat:
         hg = torch.empty(mt.flat["g"].shape, dtype=mt.flat["g"].dtype, pin_memory=True)
         hg.copy_(mt.flat["g"])
         hw = torch.empty(mt.flat["w"].shape, dtype=mt.flat["w"].dtype, pin_memory=True)
@@ -267,14 +296,15 @@ def summarize(wl, res, n_gpus, peak, peak_kind):
     bpp = algorithmic_bytes_per_param(wl)
     launch = sorted(res["launch_ms"])
     avg_launch = sum(launch) / len(launch)
-    achieved = bpp * n / (avg_launch * 1e-3) / 1e9
+    achieved = algorithmic_bytes(wl) / (avg_launch * 1e-3) / 1e9
     out = {
         "workload": wl.name, "params": n, "tensors": len(wl.specs),
         "ms_per_step": ms, "gparams_per_s": whole_job_rate(n, n_gpus, ms),
-        "hbm_gbs": bpp * n / (ms * 1e-3) / 1e9,
+        "hbm_gbs": algorithmic_bytes(wl) / (ms * 1e-3) / 1e9,
         "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
                      "frac": round(achieved / peak, 4), "traffic": recorded_traffic(wl.name),
-                     "peak_source": peak_kind, "bytes_per_param": bpp,
+                     "peak_source": peak_kind, "bytes_per_param": round(bpp, 4),
+                     "launches_per_step": res["launches_per_step"],
                      "kernel": "mpadam::step_kernel", "launch_ms_avg": round(avg_launch, 4),
                      "launch_ms_min": round(launch[0], 4), "launch_ms_max": round(launch[-1], 4),
                      "launch_ms_first_last": [round(res["launch_ms"][0], 4), round(res["launch_ms"][-1], 4)]},
@@ -292,7 +322,8 @@ def main():
     ap.add_argument("--steps", type=int, default=50)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--config", default="llama_7b")
-    ap.add_argument("--secondary", default="llama_1p5b,gpt2_124m,ragged_20k", help="'' to skip")
+    ap.add_argument("--secondary", default="llama_1p5b,llama_1p5b_mixed,gpt2_124m,ragged_20k",
+                    help="'' to skip")
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--e2e-steps", type=int, default=5)
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
@@ -388,7 +419,7 @@ def main():
         "roofline": main_sum["roofline"],
         "cpu_baseline": cpu,
         "e2e": main_sum.get("e2e"),
-        "gpu_launches": args.steps,
+        "gpu_launches": args.steps * res["launches_per_step"],
         "clocks": clocks,
         "secondary": secondary,
     }

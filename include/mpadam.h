@@ -94,7 +94,9 @@ typedef enum {
   MPADAM_EUNSUPPORTED = 4  /* valid request this build does not implement */
 } mpadam_status;
 
-typedef enum { MPADAM_F32 = 0, MPADAM_BF16 = 1, MPADAM_E4M3 = 2 } mpadam_dtype;
+/* MPADAM_E4M3_B32: E4M3 codes with one FP16 power-of-two scale per 32
+ * consecutive elements (block scaling; weights only, mpadam_create_ex). */
+typedef enum { MPADAM_F32 = 0, MPADAM_BF16 = 1, MPADAM_E4M3 = 2, MPADAM_E4M3_B32 = 3 } mpadam_dtype;
 typedef enum { MPADAM_ROUND_NEAREST = 0, MPADAM_ROUND_STOCHASTIC = 1 } mpadam_rounding;
 
 /* One parameter tensor (Algorithm 1's state per parameter: w, mu, nu, nu_e),
@@ -139,6 +141,42 @@ typedef struct {
 
 typedef struct mpadam_state mpadam_state;
 
+/* One parameter tensor of a list that may mix weight formats (the paper's
+ * FP8 regime, Sec. 5.2 and the FP8-master figure: FP8 linear layers with
+ * FP16 block scales, BF16 embeddings, norms and head).  w, m, v, ve, numel
+ * as in mpadam_tensor (m, v, ve of the config's moment_dtype).
+ *   weight_dtype: MPADAM_BF16, MPADAM_E4M3 (per-tensor scale, delayed, held
+ *     in the fp8 rings as described above) or MPADAM_E4M3_B32;
+ *   block_scale: E4M3_B32 only (else NULL): device array of ceil(numel/32)
+ *     FP16 bit patterns, the scale of elements [32b, 32b + 32) at index b,
+ *     2-byte aligned (16-byte aligned for the staged fast path).  Stored
+ *     weights decode as code * scale.  A step rewrites every block's scale
+ *     with 2^k, k the smallest integer with A <= 448 * 2^k (A = the block's
+ *     largest finite |w'| of this step; current scaling), clamped to
+ *     [-24, 15] (every such power is an FP16 number); a block whose A is 0
+ *     keeps the exponent of its old scale.  The new codes encode w' * 2^-k
+ *     (nearest-even or stochastic, saturating at +-448, as for E4M3).
+ *     Scales should be powers of two; another FP16 value decodes as itself
+ *     and counts as the power of two at or below it;
+ *   compute: optional (NULL = none; E4M3 formats only): device array of
+ *     numel BF16 values, 2-byte aligned (16-byte for the vector path),
+ *     overwritten every step with the dequantised updated weights
+ *     bf16(code * scale) -- exact, since every E4M3 value times a scale is a
+ *     BF16 number -- from the same kernel pass that writes the codes
+ *     (Sec. 5.2's low-precision master weights feed a BF16 forward pass).
+ *   reserved: must be 0. */
+typedef struct {
+  void* w;
+  void* m;
+  void* v;
+  void* ve;
+  int64_t numel;
+  int32_t weight_dtype;
+  int32_t reserved;
+  uint16_t* block_scale;
+  uint16_t* compute;
+} mpadam_tensor_ex;
+
 /* Build the fused step for a tensor list (Algorithm 1 "State").  Copies
  * `tensors` (the caller may free the array), validates, lays out the global
  * element index, allocates and uploads device metadata (synchronously, on the
@@ -148,11 +186,25 @@ typedef struct mpadam_state mpadam_state;
 int32_t mpadam_create(const mpadam_tensor* tensors, int32_t n, const mpadam_config* cfg,
                       int32_t* fp8_exp, uint32_t* fp8_amax, mpadam_state** out);
 
+/* The same for a list whose tensors each name their weight format (and
+ * carry block scales and compute copies, see mpadam_tensor_ex); cfg's
+ * weight_dtype is not used.  The tensors are stepped by one kernel launch
+ * per format present, in the order BF16, E4M3, E4M3_B32, all on the stream
+ * given to mpadam_step; global element indices (stochastic rounding) are
+ * those of the whole list, and the fp8 rings (required when any tensor is
+ * E4M3, else may be NULL) are indexed by list position k over all n
+ * tensors; entries of other tensors are left alone by the step.
+ * Errors: EINVAL (arguments), EALLOC, ECUDA.  On error *out is NULL. */
+int32_t mpadam_create_ex(const mpadam_tensor_ex* tensors, int32_t n, const mpadam_config* cfg,
+                         int32_t* fp8_exp, uint32_t* fp8_amax, mpadam_state** out);
+
 /* E4M3 only: seed the scale state before `first_step` (t0 >= 1).  Writes
  * init_exp (host array of n exponents in [-100, 100], the exponents the
  * stored weights are currently encoded with) into both fp8_exp slots, clears
  * all fp8_amax slots and writes A_t0 = largest |decoded stored weight| of
- * each tensor into slot t0 mod 3, on `stream`.  Errors: EINVAL, ECUDA. */
+ * each tensor into slot t0 mod 3, on `stream`.  In a mixed list only the
+ * per-tensor-scaled E4M3 tensors' entries are checked and used (the others
+ * are written as 0).  Errors: EINVAL, ECUDA. */
 int32_t mpadam_fp8_init(mpadam_state* s, const int32_t* init_exp, int64_t first_step,
                         struct CUstream_st* stream);
 
@@ -168,10 +220,12 @@ int32_t mpadam_step(mpadam_state* s, const void* const* grads, int64_t step,
 /* The same step with gradients and weights in host memory: copies
  * host_grads[k] (numel[k] gradients each) to library-owned device staging,
  * runs the step, and copies every updated weight tensor back to
- * host_w_out[k] (numel[k] weights of weight_dtype each).  The host buffers
- * should be pinned.  When host_grads, host_w_out and the device weights each
- * follow the global-index layout of one flat allocation (pointer k = base +
- * off[k] * element size), the step is pipelined in up to 8 chunks of whole
+ * host_w_out[k] (numel[k] weights of its weight format each; block scales
+ * and compute copies stay in device memory).  The host buffers should be
+ * pinned.  When the list has one weight format and host_grads, host_w_out
+ * and the device weights each follow the global-index layout of one flat
+ * allocation (pointer k = base + off[k] * element size), the step is
+ * pipelined in up to 8 chunks of whole
  * tiles: chunk c's gradients upload on an internal stream while chunk c-1 is
  * stepped on `stream` and chunk c-2's weights download on a second internal
  * stream (copies cover each chunk's whole global-index range, padding
@@ -195,9 +249,10 @@ const char* mpadam_last_error(void);
 int32_t mpadam_global_offset(const mpadam_state* s, int32_t k, int64_t* offset);
 int32_t mpadam_global_length(const mpadam_state* s, int64_t* length);
 
-/* Launch shape: ctas = number of CTAs of the step kernel (0 restores the
- * default, one full wave at the kernel's occupancy).  Results do not depend
- * on it.  mpadam_launch_info reports the current grid and threads per CTA. */
+/* Launch shape: ctas = number of CTAs of each step-kernel launch (0
+ * restores the default, one full wave at the kernel's occupancy).  Results
+ * do not depend on it.  Synchronises the device.  mpadam_launch_info
+ * reports the current grid (of the first launch) and threads per CTA. */
 int32_t mpadam_set_grid(mpadam_state* s, int32_t ctas);
 int32_t mpadam_launch_info(const mpadam_state* s, int32_t* ctas, int32_t* threads);
 
@@ -210,7 +265,7 @@ int32_t mpadam_device_status(mpadam_state* s, int32_t* code);
 /* Diagnostics: the random bits the step draws.  Writes into out (device,
  * uint32[n]) the lane of global element indices first, ..., first + n - 1 at
  * step `step` for weight storage `weight_dtype` (16-bit lanes for BF16,
- * 32-bit for E4M3), on `stream`.  Errors: EINVAL, ECUDA. */
+ * 32-bit for both E4M3 formats), on `stream`.  Errors: EINVAL, ECUDA. */
 int32_t mpadam_rng_lanes(uint64_t seed, int64_t step, int32_t weight_dtype, int64_t first,
                          int64_t n, uint32_t* out, struct CUstream_st* stream);
 

@@ -14,13 +14,13 @@ from typing import Optional, Sequence
 from . import builder as _build
 
 MPADAM_OK, MPADAM_EINVAL, MPADAM_EALLOC, MPADAM_ECUDA, MPADAM_EUNSUPPORTED = 0, 1, 2, 3, 4
-MPADAM_F32, MPADAM_BF16, MPADAM_E4M3 = 0, 1, 2
+MPADAM_F32, MPADAM_BF16, MPADAM_E4M3, MPADAM_E4M3_B32 = 0, 1, 2, 3
 MPADAM_ROUND_NEAREST, MPADAM_ROUND_STOCHASTIC = 0, 1
-DTYPE = {"f32": MPADAM_F32, "bf16": MPADAM_BF16, "e4m3": MPADAM_E4M3}
+DTYPE = {"f32": MPADAM_F32, "bf16": MPADAM_BF16, "e4m3": MPADAM_E4M3, "e4m3_b32": MPADAM_E4M3_B32}
 ROUNDING = {"nearest": MPADAM_ROUND_NEAREST, "stochastic": MPADAM_ROUND_STOCHASTIC}
 
-EXPORTED = ["mpadam_create", "mpadam_fp8_init", "mpadam_step", "mpadam_step_host", "mpadam_destroy",
-            "mpadam_last_error", "mpadam_global_offset", "mpadam_global_length", "mpadam_set_grid",
+EXPORTED = ["mpadam_create", "mpadam_create_ex", "mpadam_fp8_init", "mpadam_step", "mpadam_step_host",
+            "mpadam_destroy", "mpadam_last_error", "mpadam_global_offset", "mpadam_global_length", "mpadam_set_grid",
             "mpadam_launch_info", "mpadam_rng_lanes", "mpadam_step_noalloc", "mpadam_device_status"]
 
 
@@ -33,6 +33,12 @@ class MPAdamError(RuntimeError):
 class mpadam_tensor(ctypes.Structure):
     _fields_ = [("w", ctypes.c_void_p), ("m", ctypes.c_void_p), ("v", ctypes.c_void_p),
                 ("ve", ctypes.c_void_p), ("numel", ctypes.c_int64)]
+
+
+class mpadam_tensor_ex(ctypes.Structure):
+    _fields_ = [("w", ctypes.c_void_p), ("m", ctypes.c_void_p), ("v", ctypes.c_void_p),
+                ("ve", ctypes.c_void_p), ("numel", ctypes.c_int64), ("weight_dtype", ctypes.c_int32),
+                ("reserved", ctypes.c_int32), ("block_scale", ctypes.c_void_p), ("compute", ctypes.c_void_p)]
 
 
 class mpadam_config(ctypes.Structure):
@@ -83,6 +89,7 @@ def lib() -> ctypes.CDLL:
         P, i32, i64, u64 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_uint64
         sig = {
             "mpadam_create": [P, i32, P, P, P, P],
+            "mpadam_create_ex": [P, i32, P, P, P, P],
             "mpadam_fp8_init": [P, P, i64, P],
             "mpadam_step": [P, P, i64, P],
             "mpadam_step_host": [P, P, P, i64, P],
@@ -129,6 +136,19 @@ def mpadam_create(tensors: Sequence[tuple], cfg: mpadam_config, fp8_exp: int = 0
     out = ctypes.c_void_p()
     _check(lib().mpadam_create(arr, len(tensors), ctypes.byref(cfg), fp8_exp or None, fp8_amax or None,
                                ctypes.byref(out)))
+    return out.value
+
+
+def mpadam_create_ex(tensors: Sequence[tuple], cfg: mpadam_config, fp8_exp: int = 0, fp8_amax: int = 0) -> int:
+    """tensors: (w, m, v, ve, numel, weight_dtype, block_scale, compute) per tensor,
+    pointers as ints (0 = NULL), weight_dtype an MPADAM_* value or its name."""
+    arr = (mpadam_tensor_ex * max(1, len(tensors)))()
+    for i, (w, m, v, ve, n, wd, bs, cc) in enumerate(tensors):
+        arr[i] = mpadam_tensor_ex(w, m, v, ve, n, DTYPE[wd] if isinstance(wd, str) else wd, 0, bs or None,
+                                  cc or None)
+    out = ctypes.c_void_p()
+    _check(lib().mpadam_create_ex(arr, len(tensors), ctypes.byref(cfg), fp8_exp or None, fp8_amax or None,
+                                  ctypes.byref(out)))
     return out.value
 
 

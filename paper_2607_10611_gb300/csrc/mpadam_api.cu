@@ -20,6 +20,7 @@
 
 using mpadam::StepArgs;
 using mpadam::StepScalars;
+using mpadam::TensorAux;
 using mpadam::TensorDesc;
 
 namespace {
@@ -92,20 +93,25 @@ void round_keys(uint64_t seed, uint32_t* rk0, uint32_t* rk1) {
 }
 
 // Shared-memory ring of the step kernel: one stage holds one tile of every
-// array (w | g | mu | nu | nu_e); as many stages as fit, 2 to kMaxStages.
+// array (w | g | mu | nu | nu_e | block scales); as many stages as fit, 2 to
+// kMaxStages.
 struct Geometry {
-  int32_t stages = 0, stage_bytes = 0, off_g = 0, off_m = 0, off_v = 0, off_ve = 0, dyn_smem = 0;
+  int32_t stages = 0, stage_bytes = 0, off_g = 0, off_m = 0, off_v = 0, off_ve = 0, off_s = 0, dyn_smem = 0;
 };
 
-int32_t make_geometry(const mpadam_config& c, int dev, Geometry* g);
+int32_t make_geometry(const mpadam_config& c, int32_t wd, int dev, Geometry* g);
 
 bool kernel_options(const mpadam_config& c) {
   return std::isfinite(c.g_max) || std::isfinite(c.w_max) || c.wd_add != 0.0f;
 }
 
-int32_t check_config(const mpadam_config* c) {
+// per_tensor_weights: the weight formats come with the tensors
+// (mpadam_create_ex) and cfg->weight_dtype is not used.
+int32_t check_config(const mpadam_config* c, bool per_tensor_weights = false) {
   if (!c) return fail(MPADAM_EINVAL, "config is NULL");
-  if (c->weight_dtype != MPADAM_BF16 && c->weight_dtype != MPADAM_E4M3)
+  if (!per_tensor_weights && c->weight_dtype == MPADAM_E4M3_B32)
+    return fail(MPADAM_EINVAL, "block-scaled E4M3 weights need their scale arrays: use mpadam_create_ex");
+  if (!per_tensor_weights && c->weight_dtype != MPADAM_BF16 && c->weight_dtype != MPADAM_E4M3)
     return fail(MPADAM_EINVAL, "weight_dtype must be MPADAM_BF16 or MPADAM_E4M3 (got %d)", c->weight_dtype);
   if (c->grad_dtype != MPADAM_F32 && c->grad_dtype != MPADAM_BF16)
     return fail(MPADAM_EINVAL, "grad_dtype must be MPADAM_F32 or MPADAM_BF16 (got %d)", c->grad_dtype);
@@ -133,19 +139,21 @@ int32_t check_config(const mpadam_config* c) {
   return MPADAM_OK;
 }
 
-int32_t make_geometry(const mpadam_config& c, int dev, Geometry* g) {
-  const int32_t rw = mpadam::kTile * (int32_t)elem_size(c.weight_dtype);
+int32_t make_geometry(const mpadam_config& c, int32_t wd, int dev, Geometry* g) {
+  const int32_t rw = mpadam::kTile * (int32_t)elem_size(wd);
   const int32_t rg = mpadam::kTile * (int32_t)elem_size(c.grad_dtype);
   const int32_t rm = mpadam::kTile * (int32_t)elem_size(c.moment_dtype);
+  const int32_t rs = wd == MPADAM_E4M3_B32 ? mpadam::kTileBlocks * 2 : 0;  // 240 bytes, a 16-byte multiple
   g->off_g = rw;
   g->off_m = rw + rg;
   g->off_v = g->off_m + rm;
   g->off_ve = g->off_v + rm;
-  g->stage_bytes = g->off_ve + rm;
+  g->off_s = g->off_ve + rm;
+  g->stage_bytes = g->off_s + rs;
   int optin = 0;
   cudaError_t e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
   if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceGetAttribute(MaxSharedMemoryPerBlockOptin)");
-  const int32_t budget = optin - 2048;  // static barriers and slack
+  const int32_t budget = optin - 1024;  // static barriers (128 bytes) and slack
   g->stages = std::min<int32_t>(mpadam::kMaxStages, budget / g->stage_bytes);
   if (g->stages < 2) return fail(MPADAM_EUNSUPPORTED, "device shared memory too small for the step pipeline");
   g->dyn_smem = g->stages * g->stage_bytes;
@@ -158,7 +166,8 @@ int32_t make_geometry(const mpadam_config& c, int dev, Geometry* g) {
 
 // Largest |decoded stored E4M3 weight| of each tensor -> fp8_amax[slot], over
 // the same per-CTA tile ranges as the step kernel (kConsumers threads; thread
-// c reads the 8 codes [8c, 8c + 8) of each tile).
+// c reads the 8 codes [8c, 8c + 8) of each tile).  Launched over the
+// per-tensor-scaled E4M3 tensors only; rings are indexed by list position.
 __global__ void __launch_bounds__(mpadam::kConsumers) fp8_amax_kernel(const __grid_constant__ StepArgs a,
                                                                       int32_t exp_slot, int32_t amax_slot) {
   const int64_t T = a.total_tiles;
@@ -174,9 +183,9 @@ __global__ void __launch_bounds__(mpadam::kConsumers) fp8_amax_kernel(const __gr
     if (t >= d.tile_off + tiles) {
       const uint32_t wmag = __reduce_max_sync(0xFFFFFFFFu, mag);
       if ((threadIdx.x & 31) == 0 && wmag != 0u) {
-        const int32_t e = a.fp8_exp[(int64_t)exp_slot * n + k];
+        const int32_t e = a.fp8_exp[(int64_t)exp_slot * n + d.ring];
         const float v = __fmul_rn(mpadam::e4m3_value(wmag), mpadam::pow2f(e));
-        atomicMax(&a.fp8_amax[(int64_t)amax_slot * n + k], __float_as_uint(v));
+        atomicMax(&a.fp8_amax[(int64_t)amax_slot * n + d.ring], __float_as_uint(v));
       }
       mag = 0;
       do {
@@ -196,9 +205,9 @@ __global__ void __launch_bounds__(mpadam::kConsumers) fp8_amax_kernel(const __gr
   }
   const uint32_t wmag = __reduce_max_sync(0xFFFFFFFFu, mag);
   if ((threadIdx.x & 31) == 0 && wmag != 0u) {
-    const int32_t e = a.fp8_exp[(int64_t)exp_slot * n + k];
+    const int32_t e = a.fp8_exp[(int64_t)exp_slot * n + d.ring];
     const float v = __fmul_rn(mpadam::e4m3_value(wmag), mpadam::pow2f(e));
-    atomicMax(&a.fp8_amax[(int64_t)amax_slot * n + k], __float_as_uint(v));
+    atomicMax(&a.fp8_amax[(int64_t)amax_slot * n + d.ring], __float_as_uint(v));
   }
 }
 
@@ -228,26 +237,42 @@ __global__ void rng_lanes_kernel(const __grid_constant__ RngArgs a) {
 
 // ---------------------------------------------------------------------------
 // State
+//
+// A tensor list is stepped by one kernel launch per weight format present
+// (a "group"): the descriptor, aux and gradient tables are stored in group
+// order (group 0's tensors first, each group in list order), every group
+// numbers its own tiles from 0 and has its own per-CTA start table.  Global
+// element indices and the E4M3 scale rings follow list positions.
 // ---------------------------------------------------------------------------
+struct Group {
+  int32_t wd = 0;                 // weight format of the launch
+  int32_t first = 0, count = 0;   // positions [first, first + count) of the group-ordered tables
+  int64_t tiles = 0;
+  std::vector<int64_t> numel;     // of its tensors, in order
+  bool aux = false;               // the launch reads the aux table
+  const void* kernel = nullptr;
+  Geometry geo;
+  int32_t default_grid = 0, grid = 0;
+  int32_t* d_cta_first = nullptr;
+  int32_t cta_cap = 0;
+};
+
 struct mpadam_state {
   int32_t n = 0;
   mpadam_config cfg{};
-  std::vector<int64_t> numel, goff, tile_off;
+  std::vector<int32_t> wdt;                    // weight format of each tensor (list order)
+  std::vector<int64_t> numel, goff, tile_off;  // list order; tile_off in its group's numbering
   std::vector<void*> w;
+  std::vector<int32_t> order;                  // group-ordered position -> list position
+  std::vector<Group> groups;
   int64_t length = 0;  // padded global index space
-  int64_t tiles = 0;   // total tiles
   int device = 0;
   int sm_count = 0;
-  const void* kernel = nullptr;
-  Geometry geo;
-  int32_t default_grid = 0;
-  int32_t grid = 0;
   TensorDesc* d_desc = nullptr;
+  TensorAux* d_aux = nullptr;
   const void** d_grads = nullptr;
-  int32_t* d_cta_first = nullptr;
-  int32_t cta_cap = 0;
   int32_t* d_err = nullptr;        // device error bits of the step kernel
-  const void** h_grads = nullptr;  // pinned staging of the grad pointer table
+  const void** h_grads = nullptr;  // pinned staging of the grad pointer table (group order)
   std::vector<const void*> last_grads;
   bool grads_uploaded = false;
   cudaEvent_t upload_done = nullptr;
@@ -256,7 +281,7 @@ struct mpadam_state {
   uint32_t* fp8_amax = nullptr;
   char* d_gstage = nullptr;  // mpadam_step_host gradient staging (global-index layout)
   std::vector<const void*> stage_ptrs;
-  // mpadam_step_host pipeline: chunks of whole tiles, copied and stepped in turn
+  // mpadam_step_host pipeline (single-group states): chunks of whole tiles, copied and stepped in turn
   cudaStream_t s_h2d = nullptr, s_d2h = nullptr;
   std::vector<cudaEvent_t> ev;                // per chunk: h2d done, kernel done; plus start / end
   std::vector<int64_t> chunk_tile;            // chunk c covers tiles [chunk_tile[c], chunk_tile[c+1])
@@ -266,17 +291,28 @@ struct mpadam_state {
 
 namespace {
 
+void release_pipeline(mpadam_state* s) {
+  if (s->d_chunk_first) cudaFree(s->d_chunk_first);
+  s->d_chunk_first = nullptr;
+  for (cudaEvent_t e : s->ev) cudaEventDestroy(e);
+  s->ev.clear();
+  if (s->s_h2d) cudaStreamDestroy(s->s_h2d);
+  if (s->s_d2h) cudaStreamDestroy(s->s_d2h);
+  s->s_h2d = s->s_d2h = nullptr;
+  s->chunk_tile.clear();
+  s->chunk_elem.clear();
+}
+
 void release(mpadam_state* s) {
   if (!s) return;
   if (s->d_desc) cudaFree(s->d_desc);
+  if (s->d_aux) cudaFree(s->d_aux);
   if (s->d_grads) cudaFree(const_cast<void**>(s->d_grads));
-  if (s->d_cta_first) cudaFree(s->d_cta_first);
+  for (auto& g : s->groups)
+    if (g.d_cta_first) cudaFree(g.d_cta_first);
   if (s->d_err) cudaFree(s->d_err);
   if (s->d_gstage) cudaFree(s->d_gstage);
-  if (s->d_chunk_first) cudaFree(s->d_chunk_first);
-  for (cudaEvent_t e : s->ev) cudaEventDestroy(e);
-  if (s->s_h2d) cudaStreamDestroy(s->s_h2d);
-  if (s->s_d2h) cudaStreamDestroy(s->s_d2h);
+  release_pipeline(s);
   if (s->h_grads) cudaFreeHost(const_cast<void**>(s->h_grads));
   if (s->upload_done) cudaEventDestroy(s->upload_done);
   delete s;
@@ -300,20 +336,20 @@ void cta_first_table(const int64_t* numel, int32_t n, int64_t total_tiles, int32
   }
 }
 
-int32_t upload_cta_table(mpadam_state* s, int32_t grid) {
-  if (grid > s->cta_cap) {
-    if (s->d_cta_first) cudaFree(s->d_cta_first);
-    s->d_cta_first = nullptr;
-    s->cta_cap = 0;
-    if (cudaMalloc(&s->d_cta_first, sizeof(int32_t) * grid) != cudaSuccess)
+int32_t upload_cta_table(Group& g, int32_t grid) {
+  if (grid > g.cta_cap) {
+    if (g.d_cta_first) cudaFree(g.d_cta_first);
+    g.d_cta_first = nullptr;
+    g.cta_cap = 0;
+    if (cudaMalloc(&g.d_cta_first, sizeof(int32_t) * grid) != cudaSuccess)
       return fail(MPADAM_EALLOC, "cudaMalloc of %d CTA entries failed", grid);
-    s->cta_cap = grid;
+    g.cta_cap = grid;
   }
   std::vector<int32_t> first(grid);
-  cta_first_table(s->numel.data(), s->n, s->tiles, grid, first.data());
-  cudaError_t e = cudaMemcpy(s->d_cta_first, first.data(), sizeof(int32_t) * grid, cudaMemcpyHostToDevice);
+  cta_first_table(g.numel.data(), g.count, g.tiles, grid, first.data());
+  cudaError_t e = cudaMemcpy(g.d_cta_first, first.data(), sizeof(int32_t) * grid, cudaMemcpyHostToDevice);
   if (e != cudaSuccess) return cuda_fail(e, "upload of the CTA table");
-  s->grid = grid;
+  g.grid = grid;
   return MPADAM_OK;
 }
 
@@ -328,6 +364,7 @@ void fill_common(StepArgs& a, const mpadam_config& cfg, const Geometry& geo, int
   a.off_m = geo.off_m;
   a.off_v = geo.off_v;
   a.off_ve = geo.off_ve;
+  a.off_s = geo.off_s;
   round_keys(cfg.seed, a.rk0, a.rk1);
   a.fp8_exp = fp8_exp;
   a.fp8_amax = fp8_amax;
@@ -344,20 +381,23 @@ void fill_step(StepArgs& a, const mpadam_config& cfg, int64_t step) {
   a.a_zero_slot = (int32_t)((step + 2) % 3);
 }
 
-StepArgs base_args(const mpadam_state* s) {
+StepArgs base_args(const mpadam_state* s, const Group& g) {
   StepArgs a;
-  fill_common(a, s->cfg, s->geo, s->tiles, s->n, s->fp8_exp, s->fp8_amax);
-  a.desc = s->d_desc;
-  a.grads = s->d_grads;
-  a.cta_first = s->d_cta_first;
+  fill_common(a, s->cfg, g.geo, g.tiles, s->n, s->fp8_exp, s->fp8_amax);
+  a.desc = s->d_desc + g.first;
+  a.aux = g.aux ? s->d_aux + g.first : nullptr;
+  a.grads = s->d_grads + g.first;
+  a.cta_first = g.d_cta_first;
   a.err = s->d_err;
   return a;
 }
 
-const void* select_kernel(const mpadam_config& c) {
+const void* select_kernel(const mpadam_config& c, int32_t wd) {
   const int opt = kernel_options(c) ? 1 : 0;
-  return c.weight_dtype == MPADAM_BF16 ? mpadam::step_kernel_bf16(c.grad_dtype, c.moment_dtype, c.rounding, opt)
-                                       : mpadam::step_kernel_e4m3(c.grad_dtype, c.moment_dtype, c.rounding, opt);
+  if (wd == MPADAM_BF16) return mpadam::step_kernel_bf16(c.grad_dtype, c.moment_dtype, c.rounding, opt);
+  if (wd == MPADAM_E4M3) return mpadam::step_kernel_e4m3(c.grad_dtype, c.moment_dtype, c.rounding, opt);
+  if (wd == MPADAM_E4M3_B32) return mpadam::step_kernel_e4m3b(c.grad_dtype, c.moment_dtype, c.rounding, opt);
+  return nullptr;
 }
 
 // Opt the kernel into the ring's shared memory and size one full wave.
@@ -381,12 +421,149 @@ int32_t check_device(const mpadam_state* s) {
   return MPADAM_OK;
 }
 
-}  // namespace
+// One tensor of either creation call, with its format resolved.
+struct TensorIn {
+  void *w, *m, *v, *ve;
+  int64_t numel;
+  int32_t wd;
+  uint16_t* scale;
+  uint16_t* compute;
+};
 
+// Validate a tensor list, lay out its global index and format groups, and
+// allocate and upload the device tables.  `fallback_wd` is the format of the
+// single (empty) group of an empty list.
+int32_t create_state(const std::vector<TensorIn>& t, const mpadam_config* cfg, int32_t fallback_wd,
+                     int32_t* fp8_exp, uint32_t* fp8_amax, mpadam_state** out) {
+  const int32_t n = (int32_t)t.size();
+  const size_t msz = elem_size(cfg->moment_dtype);
+  bool any_e4m3 = false;
+  int64_t off = 0;
+  for (int32_t k = 0; k < n; ++k) {
+    const TensorIn& x = t[k];
+    if (x.wd != MPADAM_BF16 && x.wd != MPADAM_E4M3 && x.wd != MPADAM_E4M3_B32)
+      return fail(MPADAM_EINVAL, "tensor %d: weight_dtype must be BF16, E4M3 or E4M3_B32 (got %d)", k, x.wd);
+    if (x.numel < 0) return fail(MPADAM_EINVAL, "tensor %d: numel < 0", k);
+    any_e4m3 = any_e4m3 || x.wd == MPADAM_E4M3;
+    if (x.numel > 0) {
+      if (!x.w || !x.m || !x.v || !x.ve) return fail(MPADAM_EINVAL, "tensor %d: NULL pointer", k);
+      if (!is_aligned(x.w, elem_size(x.wd)) || !is_aligned(x.m, msz) || !is_aligned(x.v, msz) ||
+          !is_aligned(x.ve, msz))
+        return fail(MPADAM_EINVAL, "tensor %d: pointer not aligned to its element size", k);
+      if (x.wd == MPADAM_E4M3_B32 && (!x.scale || !is_aligned(x.scale, 2)))
+        return fail(MPADAM_EINVAL, "tensor %d: block-scaled weights need a 2-byte aligned block_scale array", k);
+      if (x.compute && !is_aligned(x.compute, 2))
+        return fail(MPADAM_EINVAL, "tensor %d: compute copy not 2-byte aligned", k);
+    }
+    if (x.wd != MPADAM_E4M3_B32 && x.scale)
+      return fail(MPADAM_EINVAL, "tensor %d: block_scale is only for E4M3_B32 weights", k);
+    if (x.wd == MPADAM_BF16 && x.compute)
+      return fail(MPADAM_EINVAL, "tensor %d: BF16 weights are their own compute copy (compute must be NULL)", k);
+    if (x.numel > (int64_t(1) << 56) || off > (int64_t(1) << 58))
+      return fail(MPADAM_EINVAL, "tensor %d: element index space too large", k);
+    off = (off + x.numel + 7) / 8 * 8;
+  }
+  if (any_e4m3) {
+    if (!fp8_exp || !fp8_amax) return fail(MPADAM_EINVAL, "E4M3 weights need the fp8_exp and fp8_amax rings");
+    if (!is_aligned(fp8_exp, 4) || !is_aligned(fp8_amax, 4))
+      return fail(MPADAM_EINVAL, "fp8_exp / fp8_amax must be 4-byte aligned");
+  }
 
-namespace {
+  mpadam_state* s = new (std::nothrow) mpadam_state();
+  if (!s) return fail(MPADAM_EALLOC, "host allocation failed");
+  try {
+    s->n = n;
+    s->cfg = *cfg;
+    s->wdt.resize(n);
+    s->numel.resize(n);
+    s->goff.resize(n);
+    s->tile_off.resize(n);
+    s->w.resize(n);
+    s->last_grads.assign(n, nullptr);
+    int64_t o = 0;
+    for (int32_t k = 0; k < n; ++k) {
+      s->wdt[k] = t[k].wd;
+      s->numel[k] = t[k].numel;
+      s->goff[k] = o;
+      s->w[k] = t[k].w;
+      o = (o + t[k].numel + 7) / 8 * 8;
+    }
+    s->length = o;
+    s->fp8_exp = fp8_exp;
+    s->fp8_amax = fp8_amax;
 
-// Re-upload the gradient pointer table when it differs from the last one.
+    // format groups, in the fixed order BF16, E4M3, E4M3_B32
+    std::vector<TensorDesc> desc;
+    std::vector<TensorAux> aux;
+    bool any_aux = false;
+    for (int32_t wd : {MPADAM_BF16, MPADAM_E4M3, MPADAM_E4M3_B32}) {
+      Group g;
+      g.wd = wd;
+      g.first = (int32_t)s->order.size();
+      for (int32_t k = 0; k < n; ++k) {
+        if (t[k].wd != wd) continue;
+        s->tile_off[k] = g.tiles;
+        desc.push_back(TensorDesc{t[k].w, t[k].m, t[k].v, t[k].ve, t[k].numel, s->goff[k], g.tiles, k, 0});
+        aux.push_back(TensorAux{t[k].scale, t[k].compute});
+        g.aux = g.aux || t[k].scale != nullptr || t[k].compute != nullptr;
+        g.numel.push_back(t[k].numel);
+        g.tiles += tiles_of(t[k].numel);
+        s->order.push_back(k);
+      }
+      g.count = (int32_t)s->order.size() - g.first;
+      any_aux = any_aux || g.aux;
+      if (g.count > 0 || (n == 0 && wd == fallback_wd)) s->groups.push_back(std::move(g));
+    }
+
+    cudaError_t e = cudaGetDevice(&s->device);
+    if (e != cudaSuccess) { release(s); return cuda_fail(e, "cudaGetDevice"); }
+    e = cudaDeviceGetAttribute(&s->sm_count, cudaDevAttrMultiProcessorCount, s->device);
+    if (e != cudaSuccess) { release(s); return cuda_fail(e, "cudaDeviceGetAttribute"); }
+    int32_t rc;
+    for (auto& g : s->groups) {
+      g.kernel = select_kernel(*cfg, g.wd);
+      if (!g.kernel) { release(s); return fail(MPADAM_EUNSUPPORTED, "no kernel for these formats"); }
+      rc = make_geometry(*cfg, g.wd, s->device, &g.geo);
+      if (rc) { release(s); return rc; }
+      rc = prepare_kernel(g.kernel, g.geo, s->sm_count, &g.default_grid);
+      if (rc) { release(s); return rc; }
+    }
+
+    const size_t nn = n > 0 ? (size_t)n : 1;
+    if (cudaMalloc(&s->d_desc, sizeof(TensorDesc) * nn) != cudaSuccess ||
+        cudaMalloc(reinterpret_cast<void**>(&s->d_grads), sizeof(void*) * nn) != cudaSuccess ||
+        (any_aux && cudaMalloc(&s->d_aux, sizeof(TensorAux) * nn) != cudaSuccess) ||
+        cudaMalloc(&s->d_err, sizeof(int32_t)) != cudaSuccess ||
+        cudaMallocHost(reinterpret_cast<void**>(&s->h_grads), sizeof(void*) * nn) != cudaSuccess) {
+      release(s);
+      return fail(MPADAM_EALLOC, "allocation of the tensor tables failed");
+    }
+    e = cudaMemset(s->d_err, 0, sizeof(int32_t));
+    if (e != cudaSuccess) { release(s); return cuda_fail(e, "clearing the error word"); }
+    e = cudaEventCreateWithFlags(&s->upload_done, cudaEventDisableTiming);
+    if (e != cudaSuccess) { release(s); return cuda_fail(e, "cudaEventCreate"); }
+    if (n > 0) {
+      e = cudaMemcpy(s->d_desc, desc.data(), sizeof(TensorDesc) * n, cudaMemcpyHostToDevice);
+      if (e != cudaSuccess) { release(s); return cuda_fail(e, "upload of the tensor table"); }
+      if (any_aux) {
+        e = cudaMemcpy(s->d_aux, aux.data(), sizeof(TensorAux) * n, cudaMemcpyHostToDevice);
+        if (e != cudaSuccess) { release(s); return cuda_fail(e, "upload of the aux table"); }
+      }
+    }
+    for (auto& g : s->groups) {
+      rc = upload_cta_table(g, g.default_grid);
+      if (rc) { release(s); return rc; }
+    }
+  } catch (const std::bad_alloc&) {
+    release(s);
+    return fail(MPADAM_EALLOC, "host allocation failed");
+  }
+  *out = s;
+  return MPADAM_OK;
+}
+
+// Re-upload the gradient pointer table (in group order) when it differs from
+// the last one.
 int32_t upload_grad_table(mpadam_state* s, const void* const* grads, cudaStream_t stream) {
   cudaError_t e;
   if (s->grads_uploaded && std::memcmp(s->last_grads.data(), grads, sizeof(void*) * s->n) == 0) return MPADAM_OK;
@@ -394,7 +571,7 @@ int32_t upload_grad_table(mpadam_state* s, const void* const* grads, cudaStream_
     e = cudaEventSynchronize(s->upload_done);
     if (e != cudaSuccess) return cuda_fail(e, "cudaEventSynchronize");
   }
-  std::memcpy(s->h_grads, grads, sizeof(void*) * s->n);
+  for (int32_t p = 0; p < s->n; ++p) s->h_grads[p] = grads[s->order[p]];
   e = cudaMemcpyAsync(s->d_grads, s->h_grads, sizeof(void*) * s->n, cudaMemcpyHostToDevice, stream);
   if (e != cudaSuccess) return cuda_fail(e, "upload of the gradient table");
   e = cudaEventRecord(s->upload_done, stream);
@@ -405,22 +582,23 @@ int32_t upload_grad_table(mpadam_state* s, const void* const* grads, cudaStream_
   return MPADAM_OK;
 }
 
-// One launch of the step kernel over tiles [tile_base, tile_base + count).
-int32_t launch_step(mpadam_state* s, int64_t step, cudaStream_t stream, int64_t tile_base, int64_t count,
-                    const int32_t* cta_first, int32_t grid) {
-  StepArgs a = base_args(s);
+// One launch of a group's step kernel over its tiles [tile_base, tile_base + count).
+int32_t launch_step(mpadam_state* s, const Group& g, int64_t step, cudaStream_t stream, int64_t tile_base,
+                    int64_t count, const int32_t* cta_first, int32_t grid) {
+  StepArgs a = base_args(s, g);
   a.cta_first = cta_first;
   a.tile_base = tile_base;
   a.total_tiles = count;
   fill_step(a, s->cfg, step);
   void* params[] = {&a};
-  cudaError_t e = cudaLaunchKernel(s->kernel, dim3(grid), dim3(mpadam::kThreads), params, (size_t)s->geo.dyn_smem,
+  cudaError_t e = cudaLaunchKernel(g.kernel, dim3(grid), dim3(mpadam::kThreads), params, (size_t)g.geo.dyn_smem,
                                    stream);
   if (e != cudaSuccess) return cuda_fail(e, "launch of the step kernel");
   return MPADAM_OK;
 }
 
-// Global element index of a tile's first element, and one past its last.
+// Global element index of a tile's first element, and one past its last
+// (single-group states: tile numbering follows the list).
 void tile_elements(const mpadam_state* s, int64_t t, int64_t* first, int64_t* end) {
   const auto it = std::upper_bound(s->tile_off.begin(), s->tile_off.end(), t);
   int32_t k = (int32_t)(it - s->tile_off.begin()) - 1;
@@ -434,9 +612,11 @@ void tile_elements(const mpadam_state* s, int64_t t, int64_t* first, int64_t* en
 // copy streams and the events that order them (created on first use).
 int32_t prepare_pipeline(mpadam_state* s) {
   if (!s->chunk_tile.empty()) return MPADAM_OK;
-  const int32_t chunks = (int32_t)std::max<int64_t>(1, std::min<int64_t>(8, s->tiles / 256));  // 8: best measured
+  release_pipeline(s);  // whatever a failed earlier attempt left
+  const Group& g = s->groups[0];
+  const int32_t chunks = (int32_t)std::max<int64_t>(1, std::min<int64_t>(8, g.tiles / 256));  // 8: best measured
   std::vector<int64_t> ct(chunks + 1), ce(2 * (size_t)chunks);
-  for (int32_t c = 0; c <= chunks; ++c) ct[c] = (int64_t)c * s->tiles / chunks;
+  for (int32_t c = 0; c <= chunks; ++c) ct[c] = (int64_t)c * g.tiles / chunks;
   for (int32_t c = 0; c < chunks; ++c) {
     int64_t f0, e0, f1, e1;
     tile_elements(s, ct[c], &f0, &e0);
@@ -444,9 +624,9 @@ int32_t prepare_pipeline(mpadam_state* s) {
     ce[2 * c] = f0;
     ce[2 * c + 1] = e1;
   }
-  std::vector<int32_t> first((size_t)chunks * s->grid);
+  std::vector<int32_t> first((size_t)chunks * g.grid);
   for (int32_t c = 0; c < chunks; ++c)
-    cta_first_table(s->numel.data(), s->n, ct[c + 1] - ct[c], s->grid, first.data() + (size_t)c * s->grid, ct[c]);
+    cta_first_table(s->numel.data(), s->n, ct[c + 1] - ct[c], g.grid, first.data() + (size_t)c * g.grid, ct[c]);
   if (cudaMalloc(&s->d_chunk_first, sizeof(int32_t) * first.size()) != cudaSuccess)
     return fail(MPADAM_EALLOC, "cudaMalloc of the chunk tables failed");
   cudaError_t e = cudaMemcpy(s->d_chunk_first, first.data(), sizeof(int32_t) * first.size(), cudaMemcpyHostToDevice);
@@ -482,87 +662,38 @@ int32_t mpadam_create(const mpadam_tensor* tensors, int32_t n, const mpadam_conf
   if (n > 0 && !tensors) return fail(MPADAM_EINVAL, "tensors is NULL");
   int32_t rc = check_config(cfg);
   if (rc) return rc;
-  const size_t wsz = elem_size(cfg->weight_dtype), msz = elem_size(cfg->moment_dtype);
-  if (cfg->weight_dtype == MPADAM_E4M3) {
-    if (!fp8_exp || !fp8_amax) return fail(MPADAM_EINVAL, "E4M3 weights need the fp8_exp and fp8_amax rings");
-    if (!is_aligned(fp8_exp, 4) || !is_aligned(fp8_amax, 4))
-      return fail(MPADAM_EINVAL, "fp8_exp / fp8_amax must be 4-byte aligned");
-  }
-  int64_t off = 0;
-  for (int32_t k = 0; k < n; ++k) {
-    const mpadam_tensor& t = tensors[k];
-    if (t.numel < 0) return fail(MPADAM_EINVAL, "tensor %d: numel < 0", k);
-    if (t.numel > 0) {
-      if (!t.w || !t.m || !t.v || !t.ve) return fail(MPADAM_EINVAL, "tensor %d: NULL pointer", k);
-      if (!is_aligned(t.w, wsz) || !is_aligned(t.m, msz) || !is_aligned(t.v, msz) || !is_aligned(t.ve, msz))
-        return fail(MPADAM_EINVAL, "tensor %d: pointer not aligned to its element size", k);
-    }
-    if (t.numel > (int64_t(1) << 56) || off > (int64_t(1) << 58))
-      return fail(MPADAM_EINVAL, "tensor %d: element index space too large", k);
-    off = (off + t.numel + 7) / 8 * 8;
-  }
-
-  mpadam_state* s = new (std::nothrow) mpadam_state();
-  if (!s) return fail(MPADAM_EALLOC, "host allocation failed");
+  if (cfg->weight_dtype == MPADAM_E4M3 && (!fp8_exp || !fp8_amax))
+    return fail(MPADAM_EINVAL, "E4M3 weights need the fp8_exp and fp8_amax rings");
   try {
-    s->n = n;
-    s->cfg = *cfg;
-    s->numel.resize(n);
-    s->goff.resize(n);
-    s->tile_off.resize(n);
-    s->w.resize(n);
-    s->last_grads.assign(n, nullptr);
-    std::vector<TensorDesc> desc(n);
-    int64_t o = 0, to = 0;
-    for (int32_t k = 0; k < n; ++k) {
-      s->numel[k] = tensors[k].numel;
-      s->goff[k] = o;
-      s->tile_off[k] = to;
-      s->w[k] = tensors[k].w;
-      desc[k] = TensorDesc{tensors[k].w, tensors[k].m, tensors[k].v, tensors[k].ve, tensors[k].numel, o, to, 0};
-      o = (o + tensors[k].numel + 7) / 8 * 8;
-      to += tiles_of(tensors[k].numel);
-    }
-    s->length = o;
-    s->tiles = to;
-    s->fp8_exp = fp8_exp;
-    s->fp8_amax = fp8_amax;
-    s->kernel = select_kernel(*cfg);
-    if (!s->kernel) { release(s); return fail(MPADAM_EUNSUPPORTED, "no kernel for these formats"); }
-
-    cudaError_t e = cudaGetDevice(&s->device);
-    if (e != cudaSuccess) { release(s); return cuda_fail(e, "cudaGetDevice"); }
-    e = cudaDeviceGetAttribute(&s->sm_count, cudaDevAttrMultiProcessorCount, s->device);
-    if (e != cudaSuccess) { release(s); return cuda_fail(e, "cudaDeviceGetAttribute"); }
-    rc = make_geometry(*cfg, s->device, &s->geo);
-    if (rc) { release(s); return rc; }
-    rc = prepare_kernel(s->kernel, s->geo, s->sm_count, &s->default_grid);
-    if (rc) { release(s); return rc; }
-
-    const size_t nn = n > 0 ? (size_t)n : 1;
-    if (cudaMalloc(&s->d_desc, sizeof(TensorDesc) * nn) != cudaSuccess ||
-        cudaMalloc(reinterpret_cast<void**>(&s->d_grads), sizeof(void*) * nn) != cudaSuccess ||
-        cudaMalloc(&s->d_err, sizeof(int32_t)) != cudaSuccess ||
-        cudaMallocHost(reinterpret_cast<void**>(&s->h_grads), sizeof(void*) * nn) != cudaSuccess) {
-      release(s);
-      return fail(MPADAM_EALLOC, "allocation of the tensor tables failed");
-    }
-    e = cudaMemset(s->d_err, 0, sizeof(int32_t));
-    if (e != cudaSuccess) { release(s); return cuda_fail(e, "clearing the error word"); }
-    e = cudaEventCreateWithFlags(&s->upload_done, cudaEventDisableTiming);
-    if (e != cudaSuccess) { release(s); return cuda_fail(e, "cudaEventCreate"); }
-    if (n > 0) {
-      e = cudaMemcpy(s->d_desc, desc.data(), sizeof(TensorDesc) * n, cudaMemcpyHostToDevice);
-      if (e != cudaSuccess) { release(s); return cuda_fail(e, "upload of the tensor table"); }
-    }
-    rc = upload_cta_table(s, s->default_grid);
-    if (rc) { release(s); return rc; }
+    std::vector<TensorIn> t(n);
+    for (int32_t k = 0; k < n; ++k)
+      t[k] = TensorIn{tensors[k].w, tensors[k].m, tensors[k].v, tensors[k].ve, tensors[k].numel, cfg->weight_dtype,
+                      nullptr, nullptr};
+    return create_state(t, cfg, cfg->weight_dtype, fp8_exp, fp8_amax, out);
   } catch (const std::bad_alloc&) {
-    release(s);
     return fail(MPADAM_EALLOC, "host allocation failed");
   }
-  *out = s;
-  return MPADAM_OK;
+}
+
+int32_t mpadam_create_ex(const mpadam_tensor_ex* tensors, int32_t n, const mpadam_config* cfg,
+                         int32_t* fp8_exp, uint32_t* fp8_amax, mpadam_state** out) {
+  if (!out) return fail(MPADAM_EINVAL, "out is NULL");
+  *out = nullptr;
+  if (n < 0) return fail(MPADAM_EINVAL, "n must be >= 0 (got %d)", n);
+  if (n > 0 && !tensors) return fail(MPADAM_EINVAL, "tensors is NULL");
+  int32_t rc = check_config(cfg, true);
+  if (rc) return rc;
+  try {
+    std::vector<TensorIn> t(n);
+    for (int32_t k = 0; k < n; ++k) {
+      const mpadam_tensor_ex& x = tensors[k];
+      if (x.reserved != 0) return fail(MPADAM_EINVAL, "tensor %d: reserved must be 0", k);
+      t[k] = TensorIn{x.w, x.m, x.v, x.ve, x.numel, x.weight_dtype, x.block_scale, x.compute};
+    }
+    return create_state(t, cfg, MPADAM_BF16, fp8_exp, fp8_amax, out);
+  } catch (const std::bad_alloc&) {
+    return fail(MPADAM_EALLOC, "host allocation failed");
+  }
 }
 
 int32_t mpadam_destroy(mpadam_state* s) {
@@ -591,12 +722,17 @@ int32_t mpadam_set_grid(mpadam_state* s, int32_t ctas) {
   if (rc) return rc;
   cudaError_t e = cudaDeviceSynchronize();  // the old table may be in use
   if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceSynchronize");
-  return upload_cta_table(s, ctas == 0 ? s->default_grid : ctas);
+  release_pipeline(s);  // the host-buffer pipeline's per-chunk tables follow the grid: rebuilt on next use
+  for (auto& g : s->groups) {
+    rc = upload_cta_table(g, ctas == 0 ? g.default_grid : ctas);
+    if (rc) return rc;
+  }
+  return MPADAM_OK;
 }
 
 int32_t mpadam_launch_info(const mpadam_state* s, int32_t* ctas, int32_t* threads) {
   if (!s || !ctas || !threads) return fail(MPADAM_EINVAL, "NULL argument");
-  *ctas = s->grid;
+  *ctas = s->groups.empty() ? 0 : s->groups[0].grid;
   *threads = mpadam::kThreads;
   return MPADAM_OK;
 }
@@ -617,7 +753,9 @@ int32_t mpadam_device_status(mpadam_state* s, int32_t* code) {
 int32_t mpadam_step(mpadam_state* s, const void* const* grads, int64_t step, cudaStream_t stream) {
   if (!s) return fail(MPADAM_EINVAL, "state is NULL");
   if (step < 1) return fail(MPADAM_EINVAL, "step must be >= 1 (got %lld)", (long long)step);
-  if (s->n == 0 || s->tiles == 0) return MPADAM_OK;
+  int64_t tiles = 0;
+  for (const auto& g : s->groups) tiles += g.tiles;
+  if (s->n == 0 || tiles == 0) return MPADAM_OK;
   if (!grads) return fail(MPADAM_EINVAL, "grads is NULL");
   const size_t gsz = elem_size(s->cfg.grad_dtype);
   for (int32_t k = 0; k < s->n; ++k) {
@@ -629,23 +767,31 @@ int32_t mpadam_step(mpadam_state* s, const void* const* grads, int64_t step, cud
   if (rc) return rc;
   rc = upload_grad_table(s, grads, stream);
   if (rc) return rc;
-  return launch_step(s, step, stream, 0, s->tiles, s->d_cta_first, s->grid);
+  for (const auto& g : s->groups) {
+    if (g.tiles == 0) continue;
+    rc = launch_step(s, g, step, stream, 0, g.tiles, g.d_cta_first, g.grid);
+    if (rc) return rc;
+  }
+  return MPADAM_OK;
 }
 
 int32_t mpadam_fp8_init(mpadam_state* s, const int32_t* init_exp, int64_t first_step, cudaStream_t stream) {
   if (!s) return fail(MPADAM_EINVAL, "state is NULL");
-  if (s->cfg.weight_dtype != MPADAM_E4M3) return fail(MPADAM_EINVAL, "fp8_init needs E4M3 weights");
+  const Group* g = nullptr;
+  for (const auto& x : s->groups)
+    if (x.wd == MPADAM_E4M3) g = &x;
+  if (!g) return fail(MPADAM_EINVAL, "fp8_init needs E4M3 weights");
   if (first_step < 1) return fail(MPADAM_EINVAL, "first_step must be >= 1");
   if (s->n == 0) return MPADAM_OK;
   if (!init_exp) return fail(MPADAM_EINVAL, "init_exp is NULL");
   for (int32_t k = 0; k < s->n; ++k)
-    if (init_exp[k] < -100 || init_exp[k] > 100)
+    if (s->wdt[k] == MPADAM_E4M3 && (init_exp[k] < -100 || init_exp[k] > 100))
       return fail(MPADAM_EINVAL, "init_exp[%d] = %d outside [-100, 100]", k, init_exp[k]);
   int32_t rc = check_device(s);
   if (rc) return rc;
-  std::vector<int32_t> both(2 * (size_t)s->n);
-  std::copy(init_exp, init_exp + s->n, both.begin());
-  std::copy(init_exp, init_exp + s->n, both.begin() + s->n);
+  std::vector<int32_t> both(2 * (size_t)s->n, 0);
+  for (int32_t k = 0; k < s->n; ++k)
+    if (s->wdt[k] == MPADAM_E4M3) both[k] = both[s->n + k] = init_exp[k];
   cudaError_t e = cudaMemcpyAsync(s->fp8_exp, both.data(), sizeof(int32_t) * both.size(),
                                   cudaMemcpyHostToDevice, stream);
   if (e != cudaSuccess) return cuda_fail(e, "upload of the initial exponents");
@@ -653,11 +799,11 @@ int32_t mpadam_fp8_init(mpadam_state* s, const int32_t* init_exp, int64_t first_
   if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
   e = cudaMemsetAsync(s->fp8_amax, 0, sizeof(uint32_t) * 3 * (size_t)s->n, stream);
   if (e != cudaSuccess) return cuda_fail(e, "clearing fp8_amax");
-  if (s->tiles == 0) return MPADAM_OK;
-  StepArgs a = base_args(s);
+  if (g->tiles == 0) return MPADAM_OK;
+  StepArgs a = base_args(s, *g);
   int32_t exp_slot = (int32_t)(first_step % 2), amax_slot = (int32_t)(first_step % 3);
   void* params[] = {&a, &exp_slot, &amax_slot};
-  e = cudaLaunchKernel(reinterpret_cast<const void*>(&fp8_amax_kernel), dim3(s->grid), dim3(mpadam::kConsumers),
+  e = cudaLaunchKernel(reinterpret_cast<const void*>(&fp8_amax_kernel), dim3(g->grid), dim3(mpadam::kConsumers),
                        params, 0, stream);
   if (e != cudaSuccess) return cuda_fail(e, "launch of the amax kernel");
   return MPADAM_OK;
@@ -666,8 +812,8 @@ int32_t mpadam_fp8_init(mpadam_state* s, const int32_t* init_exp, int64_t first_
 int32_t mpadam_rng_lanes(uint64_t seed, int64_t step, int32_t weight_dtype, int64_t first, int64_t n,
                          uint32_t* out, cudaStream_t stream) {
   if (step < 0) return fail(MPADAM_EINVAL, "step must be >= 0");
-  if (weight_dtype != MPADAM_BF16 && weight_dtype != MPADAM_E4M3)
-    return fail(MPADAM_EINVAL, "weight_dtype must be MPADAM_BF16 or MPADAM_E4M3");
+  if (weight_dtype != MPADAM_BF16 && weight_dtype != MPADAM_E4M3 && weight_dtype != MPADAM_E4M3_B32)
+    return fail(MPADAM_EINVAL, "weight_dtype must be MPADAM_BF16, MPADAM_E4M3 or MPADAM_E4M3_B32");
   if (first < 0 || n < 0) return fail(MPADAM_EINVAL, "first and n must be >= 0");
   if (n == 0) return MPADAM_OK;
   if (!out || !is_aligned(out, 4)) return fail(MPADAM_EINVAL, "out is NULL or misaligned");
@@ -690,14 +836,16 @@ int32_t mpadam_step_host(mpadam_state* s, const void* const* host_grads, void* c
                          int64_t step, cudaStream_t stream) {
   if (!s) return fail(MPADAM_EINVAL, "state is NULL");
   if (step < 1) return fail(MPADAM_EINVAL, "step must be >= 1");
-  if (s->n == 0 || s->tiles == 0) return MPADAM_OK;
+  int64_t tiles = 0;
+  for (const auto& g : s->groups) tiles += g.tiles;
+  if (s->n == 0 || tiles == 0) return MPADAM_OK;
   if (!host_grads || !host_w_out) return fail(MPADAM_EINVAL, "host_grads / host_w_out is NULL");
   for (int32_t k = 0; k < s->n; ++k)
     if (s->numel[k] > 0 && (!host_grads[k] || !host_w_out[k]))
       return fail(MPADAM_EINVAL, "host buffer %d is NULL", k);
   int32_t rc = check_device(s);
   if (rc) return rc;
-  const size_t gsz = elem_size(s->cfg.grad_dtype), wsz = elem_size(s->cfg.weight_dtype);
+  const size_t gsz = elem_size(s->cfg.grad_dtype);
   cudaError_t e;
   if (!s->d_gstage) {
     if (cudaMalloc(&s->d_gstage, (size_t)s->length * gsz) != cudaSuccess)
@@ -723,13 +871,18 @@ int32_t mpadam_step_host(mpadam_state* s, const void* const* host_grads, void* c
   while (last >= 0 && s->numel[last] == 0) --last;
   if (first > last) return MPADAM_OK;
   const size_t lo_e = (size_t)s->goff[first], hi_e = (size_t)(s->goff[last] + s->numel[last]);
+  // one weight format for the whole list?  (then wsz is its element size)
+  const bool single = s->groups.size() == 1;
+  const size_t wsz = elem_size(s->groups[0].wd);
 
   const char* hb = nullptr;
   const char* dw0 = nullptr;
   const char* hw0 = nullptr;
-  if (flat_base(host_grads, gsz, &hb) && flat_base(s->w.data(), wsz, &dw0) && flat_base(host_w_out, wsz, &hw0)) {
+  if (single && flat_base(host_grads, gsz, &hb) && flat_base(s->w.data(), wsz, &dw0) &&
+      flat_base(host_w_out, wsz, &hw0)) {
     // Pipelined: chunk c's gradients upload on s_h2d, its step runs on
     // `stream` after them, its weights download on s_d2h after the step.
+    const Group& g = s->groups[0];
     rc = prepare_pipeline(s);
     if (rc) return rc;
     rc = upload_grad_table(s, s->stage_ptrs.data(), stream);
@@ -747,8 +900,8 @@ int32_t mpadam_step_host(mpadam_state* s, const void* const* host_grads, void* c
       if (e != cudaSuccess) return cuda_fail(e, "gradient upload");
       if ((e = cudaEventRecord(s->ev[2 * c], s->s_h2d)) != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
       if ((e = cudaStreamWaitEvent(stream, s->ev[2 * c], 0)) != cudaSuccess) return cuda_fail(e, "cudaStreamWaitEvent");
-      rc = launch_step(s, step, stream, s->chunk_tile[c], s->chunk_tile[c + 1] - s->chunk_tile[c],
-                       s->d_chunk_first + (size_t)c * s->grid, s->grid);
+      rc = launch_step(s, g, step, stream, s->chunk_tile[c], s->chunk_tile[c + 1] - s->chunk_tile[c],
+                       s->d_chunk_first + (size_t)c * g.grid, g.grid);
       if (rc) return rc;
       if ((e = cudaEventRecord(s->ev[2 * c + 1], stream)) != cudaSuccess) return cuda_fail(e, "cudaEventRecord");
       if ((e = cudaStreamWaitEvent(s->s_d2h, s->ev[2 * c + 1], 0)) != cudaSuccess)
@@ -778,7 +931,7 @@ int32_t mpadam_step_host(mpadam_state* s, const void* const* host_grads, void* c
   if (rc) return rc;
   const char* dw = nullptr;
   const char* hw = nullptr;
-  if (flat_base(const_cast<const void* const*>(reinterpret_cast<void* const*>(s->w.data())), wsz, &dw) &&
+  if (single && flat_base(const_cast<const void* const*>(reinterpret_cast<void* const*>(s->w.data())), wsz, &dw) &&
       flat_base(const_cast<const void* const*>(host_w_out), wsz, &hw)) {
     e = cudaMemcpyAsync(const_cast<char*>(hw) + lo_e * wsz, dw + lo_e * wsz, (hi_e - lo_e) * wsz,
                         cudaMemcpyDeviceToHost, stream);
@@ -786,7 +939,8 @@ int32_t mpadam_step_host(mpadam_state* s, const void* const* host_grads, void* c
   } else {
     for (int32_t k = 0; k < s->n; ++k) {
       if (s->numel[k] == 0) continue;
-      e = cudaMemcpyAsync(host_w_out[k], s->w[k], (size_t)s->numel[k] * wsz, cudaMemcpyDeviceToHost, stream);
+      e = cudaMemcpyAsync(host_w_out[k], s->w[k], (size_t)s->numel[k] * elem_size(s->wdt[k]), cudaMemcpyDeviceToHost,
+                          stream);
       if (e != cudaSuccess) return cuda_fail(e, "weight download");
     }
   }
@@ -911,10 +1065,10 @@ extern "C" int32_t mpadam_step_noalloc(const mpadam_tensor* tensors, int32_t n, 
   int sms = 0;
   rc = noalloc_setup(dev, &scratch, &sms);
   if (rc) return rc;
-  const void* kernel = select_kernel(*cfg);
+  const void* kernel = select_kernel(*cfg, cfg->weight_dtype);
   if (!kernel) return fail(MPADAM_EUNSUPPORTED, "no kernel for these formats");
   Geometry geo;
-  rc = make_geometry(*cfg, dev, &geo);
+  rc = make_geometry(*cfg, cfg->weight_dtype, dev, &geo);
   if (rc) return rc;
   int32_t grid = 0;
   rc = prepare_kernel(kernel, geo, sms, &grid);
@@ -932,7 +1086,7 @@ extern "C" int32_t mpadam_step_noalloc(const mpadam_tensor* tensors, int32_t n, 
     const int32_t cnt = std::min(kFillChunk, n - k0);
     for (int32_t i = 0; i < cnt; ++i) {
       const mpadam_tensor& t = tensors[k0 + i];
-      fa.desc[i] = TensorDesc{t.w, t.m, t.v, t.ve, t.numel, off, toff, 0};
+      fa.desc[i] = TensorDesc{t.w, t.m, t.v, t.ve, t.numel, off, toff, k0 + i, 0};
       fa.grads[i] = grads[k0 + i];
       off = (off + t.numel + 7) / 8 * 8;
       toff += tiles_of(t.numel);

@@ -14,6 +14,13 @@
 // Element indices for stochastic rounding are independent of this
 // decomposition: element j of tensor k has global index goff[k] + j, where
 // goff[0] = 0 and goff[k+1] = goff[k] + numel[k] rounded up to a multiple of 8.
+//
+// A list that mixes weight formats is stepped by one launch per format; each
+// launch sees only its own tensors (its own descriptor, gradient and CTA
+// tables), while global indices and the E4M3 scale rings stay those of the
+// whole list.  Block-scaled E4M3 weights carry one FP16 power-of-two scale
+// per kBlock consecutive elements; a tile holds kTileBlocks whole blocks, and
+// the four consumer threads of a quad (lanes 4q .. 4q+3) own one block.
 #pragma once
 
 #include <cstdint>
@@ -27,8 +34,12 @@ constexpr int kThreads = kConsumers + 32;           // + 1 producer warp
 constexpr int kTile = kConsumers * kGroup;          // 3840 elements per tile (16-byte multiple in every format)
 constexpr int kMaxStages = 8;
 constexpr int kPhiloxRounds = 10;
+constexpr int kBlock = 32;                          // elements per block scale (block-scaled E4M3)
+constexpr int kTileBlocks = kTile / kBlock;         // 120 block scales per tile (240 bytes)
+static_assert(kTile % kBlock == 0 && kBlock == 4 * kGroup, "a block is one quad of consumer threads");
 
-enum Dtype : int { kF32 = 0, kBF16 = 1, kE4M3 = 2 };
+// kE4M3B: E4M3 codes with FP16 block scales (one per kBlock elements).
+enum Dtype : int { kF32 = 0, kBF16 = 1, kE4M3 = 2, kE4M3B = 3 };
 
 // Error bits a step kernel may set in *err (bounded waits that gave up).
 enum DeviceError : int32_t { kErrFullWait = 1, kErrEmptyWait = 2, kErrDrainWait = 4 };
@@ -42,10 +53,18 @@ struct TensorDesc {
   void* ve;
   int64_t numel;
   int64_t goff;      // global index of element 0 (multiple of 8)
-  int64_t tile_off;  // index of the tensor's first tile
-  int64_t pad;
+  int64_t tile_off;  // index of the tensor's first tile (in this launch's numbering)
+  int32_t ring;      // the tensor's position in the whole list (its E4M3 scale-ring entries)
+  int32_t pad;
 };
 static_assert(sizeof(TensorDesc) == 64, "TensorDesc must stay 64 bytes");
+
+// Per-tensor extras of the E4M3 formats; one entry per descriptor, or no
+// table at all when no tensor of the launch has any.
+struct TensorAux {
+  uint16_t* scale;    // kE4M3B: ceil(numel / kBlock) FP16 block scales, updated in place
+  uint16_t* compute;  // BF16 copy of the updated stored weights (dequantised), or nullptr
+};
 
 // Per-step binary32 scalars of the canonical update (computed on the host in
 // binary64 and rounded once).
@@ -68,13 +87,14 @@ struct StepArgs {
   const TensorDesc* desc;    // [n_tensors]
   const void* const* grads;  // [n_tensors] device pointers
   const int32_t* cta_first;  // [gridDim.x] tensor holding each CTA's first tile
+  const TensorAux* aux;      // [descriptors] or nullptr
   int64_t tile_base;         // this launch covers tiles [tile_base, tile_base + total_tiles)
   int64_t total_tiles;
-  int32_t n_tensors;
+  int32_t n_tensors;         // length of the whole list (stride of the scale rings)
   int32_t stages;            // shared-memory pipeline depth (2..kMaxStages)
-  int32_t stage_bytes;       // bytes of one stage: w | g | m | v | ve regions
+  int32_t stage_bytes;       // bytes of one stage: w | g | m | v | ve | block-scale regions
   int32_t off_g, off_m, off_v, off_ve;  // region offsets inside a stage (w at 0)
-  int32_t pad0;
+  int32_t off_s;             // block scales (kE4M3B only)
   StepScalars s;
   uint32_t rk0[kPhiloxRounds], rk1[kPhiloxRounds];  // Philox round keys: seed + r * Weyl
   uint32_t t_lo, t_hi;       // step number (Philox counter words 2, 3)
@@ -92,5 +112,6 @@ struct StepArgs {
 // step_bf16.cu / step_e4m3.cu.
 const void* step_kernel_bf16(int grad_dtype, int moment_dtype, int stochastic, int options);
 const void* step_kernel_e4m3(int grad_dtype, int moment_dtype, int stochastic, int options);
+const void* step_kernel_e4m3b(int grad_dtype, int moment_dtype, int stochastic, int options);
 
 }  // namespace mpadam

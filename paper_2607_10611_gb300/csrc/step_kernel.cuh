@@ -100,6 +100,11 @@ __device__ __forceinline__ void lds4(uint32_t addr, uint32_t (&r)[4]) {
 __device__ __forceinline__ void lds2(uint32_t addr, uint32_t (&r)[2]) {
   asm volatile("ld.shared.v2.u32 {%0,%1}, [%2];" : "=r"(r[0]), "=r"(r[1]) : "r"(addr));
 }
+__device__ __forceinline__ uint32_t lds_u16(uint32_t addr) {
+  uint16_t h;
+  asm volatile("ld.shared.u16 %0, [%1];" : "=h"(h) : "r"(addr));
+  return h;
+}
 __device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
   asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
 }
@@ -248,6 +253,7 @@ __device__ __forceinline__ float div_approx(float a, float b) {
 
 struct CertUpd {
   float wn, lo, hi;  // fast weight and the interval holding the canonical one
+  float e;           // the bound: lo = wn - e rounded down, hi = wn + e rounded up
   float m, v, ve;    // exact moments
   bool ok;           // divisors in the documented range and wn' finite
 };
@@ -272,6 +278,7 @@ __device__ __forceinline__ CertUpd madam_update_cert(const StepScalars& s, float
   const float e = __fmaf_rn(__fadd_rn(fabsf(__fmul_rn(w, um)), fabsf(ua)), 7.62939453125e-06f /* 2^-17 */,
                             __fmaf_rn(__fadd_rn(fabsf(t), fabsf(o.wn)), 2.384185791015625e-07f /* 2^-22 */,
                                       1.2621774483536189e-29f /* 2^-96 */));
+  o.e = e;
   o.lo = __fsub_rd(o.wn, e);
   o.hi = __fadd_ru(o.wn, e);
   // divisors must stay below 2^125 (their lower bounds eps, tau >= 2^-125 are
@@ -412,6 +419,36 @@ __device__ __forceinline__ float pow2f(int32_t e) {
   return __uint_as_float(static_cast<uint32_t>(e + 127) << 23);
 }
 
+// Block scales (FP16 bit patterns).  A scale written by the step is 2^k with
+// k in [-24, 15]: every such power is an FP16 number (subnormal below 2^-14).
+__device__ __forceinline__ uint32_t fp16_pow2_bits(int32_t k) {
+  k = k < -24 ? -24 : (k > 15 ? 15 : k);
+  return k >= -14 ? static_cast<uint32_t>(k + 15) << 10 : 1u << (k + 24);
+}
+// Value of a scale (exact widening conversion).
+__device__ __forceinline__ float fp16_value(uint32_t h) {
+  return __half2float(__ushort_as_half(static_cast<unsigned short>(h)));
+}
+// Exponent of a scale: its exponent field minus the bias for normal scales,
+// floor(log2) of its subnormal value otherwise (-24 for zero); the sign is
+// ignored.  Exact for the powers of two the step writes.
+__device__ __forceinline__ int32_t fp16_pow2_exponent(uint32_t h) {
+  const int32_t e = static_cast<int32_t>((h >> 10) & 0x1Fu);
+  if (e != 0) return e - 15;
+  const int32_t k = 7 - __clz(static_cast<int32_t>(h & 0x3FFu));  // floor(log2 f) - 24
+  return k < -24 ? -24 : k;
+}
+// Block scale of the next encode: the smallest k with A <= 448 * 2^k (A as
+// binary32 bits, finite and >= 0), clamped to [-24, 15]; k_old when A = 0.
+// Non-decreasing in A, which the certified path relies on.
+__device__ __forceinline__ int32_t block_exponent(uint32_t a_bits, int32_t k_old) {
+  if (a_bits == 0u) return k_old;
+  const int32_t ef = static_cast<int32_t>(a_bits >> 23);
+  int32_t k = -24;
+  if (ef != 0) k = ef - 127 - 8 + ((a_bits & 0x7FFFFFu) > 0x600000u ? 1 : 0);
+  return k < -24 ? -24 : (k > 15 ? 15 : k);
+}
+
 __device__ __forceinline__ bool aligned(const void* p, uintptr_t bytes) {
   return (reinterpret_cast<uintptr_t>(p) & (bytes - 1)) == 0;
 }
@@ -525,6 +562,9 @@ struct TensorCtx {
   bool vec;            // all pointers aligned for vector access by whole groups
   bool fast;           // whole tiles are fully staged and stored with vector stores
   float dec_scale, enc_scale;
+  float cc_scale;      // E4M3 per-tensor: 2^e of the new encode (compute copy)
+  uint16_t* scale;     // kE4M3B block scales
+  uint16_t* cc;        // BF16 compute copy, or nullptr
 };
 
 template <int WD, int GD, int MD>
@@ -537,7 +577,75 @@ __device__ __forceinline__ void load_tensor(const StepArgs& a, int k, TensorCtx&
           aligned(c.d.ve, MD == kF32 ? 32 : 16);
   c.fast = c.vec && aligned(c.d.w, 16) && aligned(c.g, 16) && aligned(c.d.m, 16) && aligned(c.d.v, 16) &&
            aligned(c.d.ve, 16);
-  c.dec_scale = c.enc_scale = 1.0f;
+  c.dec_scale = c.enc_scale = c.cc_scale = 1.0f;
+  c.scale = c.cc = nullptr;
+  if (WD != kBF16 && a.aux) {
+    const TensorAux x = a.aux[k];
+    c.scale = x.scale;
+    c.cc = x.compute;
+    // the compute copy joins the vector path only when 16-byte aligned;
+    // block scales are staged (whole tiles: 240 bytes) only when 16-byte aligned
+    if (c.cc && !aligned(c.cc, 16)) c.vec = c.fast = false;
+    if (WD == kE4M3B && !aligned(c.scale, 16)) c.fast = false;
+  }
+}
+
+// BF16 compute copy of eight stored E4M3 codes: code value x scale (a power
+// of two, so exact), rounded to BF16 (exact as well inside BF16's range).
+__device__ __forceinline__ void put_compute(const uint32_t (&codes)[2], float scale, void* cc, int64_t e0,
+                                            int valid, bool vec) {
+  float xd[8];
+  e4m3x8_to_f32(codes, xd);
+  uint32_t o[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) o[i] = bf16x2_rn(__fmul_rn(xd[2 * i], scale), __fmul_rn(xd[2 * i + 1], scale));
+  put_bf16(o, cc, e0, valid, vec);
+}
+
+// Store the updated moments (BF16 moments nearest-even).
+template <int MD>
+__device__ __forceinline__ void put_moments(const TensorCtx& x, int64_t e0, int valid, const float (&m)[8],
+                                            const float (&v)[8], const float (&ve)[8]) {
+  if (MD == kF32) {
+    put_f32(m, x.d.m, e0, valid, x.vec);
+    put_f32(v, x.d.v, e0, valid, x.vec);
+    put_f32(ve, x.d.ve, e0, valid, x.vec);
+  } else {
+    uint32_t om[4], ov[4], oe[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      om[i] = bf16x2_rn(m[2 * i], m[2 * i + 1]);
+      ov[i] = bf16x2_rn(v[2 * i], v[2 * i + 1]);
+      oe[i] = bf16x2_rn(ve[2 * i], ve[2 * i + 1]);
+    }
+    put_bf16(om, x.d.m, e0, valid, x.vec);
+    put_bf16(ov, x.d.v, e0, valid, x.vec);
+    put_bf16(oe, x.d.ve, e0, valid, x.vec);
+  }
+}
+
+// Random bits of eight consecutive elements starting at global index gidx (a
+// multiple of 8): 16-bit lanes (complemented, see bf16_sr_sum) for BF16
+// storage, 32-bit lanes for E4M3 storage.
+template <int WD>
+__device__ __forceinline__ void group_random_bits(const StepArgs& a, uint64_t gidx, uint32_t (&rnd)[8]) {
+  const uint64_t gi = gidx >> 3;  // global group index
+  if (WD == kBF16) {
+    const uint4 r = philox4x32_10(static_cast<uint32_t>(gi), static_cast<uint32_t>(gi >> 32), a.t_lo, a.t_hi,
+                                  a.rk0, a.rk1);
+    rnd[0] = ~r.x & 0xFFFFu; rnd[1] = ~r.x >> 16;
+    rnd[2] = ~r.y & 0xFFFFu; rnd[3] = ~r.y >> 16;
+    rnd[4] = ~r.z & 0xFFFFu; rnd[5] = ~r.z >> 16;
+    rnd[6] = ~r.w & 0xFFFFu; rnd[7] = ~r.w >> 16;
+  } else {
+    const uint64_t b0 = 2ull * gi, b1 = b0 + 1ull;
+    const uint4 r0 = philox4x32_10(static_cast<uint32_t>(b0), static_cast<uint32_t>(b0 >> 32), a.t_lo, a.t_hi,
+                                   a.rk0, a.rk1);
+    const uint4 r1 = philox4x32_10(static_cast<uint32_t>(b1), static_cast<uint32_t>(b1 >> 32), a.t_lo, a.t_hi,
+                                   a.rk0, a.rk1);
+    rnd[0] = r0.x; rnd[1] = r0.y; rnd[2] = r0.z; rnd[3] = r0.w;
+    rnd[4] = r1.x; rnd[5] = r1.y; rnd[6] = r1.z; rnd[7] = r1.w;
+  }
 }
 
 // Update 8 loaded elements and store them (vector stores when `vec` and
@@ -548,25 +656,7 @@ __device__ __forceinline__ void finish_group(const StepArgs& a, const TensorCtx&
                                              float (&ve)[8], uint32_t& amax_bits) {
   // random bits: one Philox block per 8 BF16 lanes, two per 8 E4M3 lanes
   uint32_t rnd[8];
-  if (SR) {
-    const uint64_t gi = static_cast<uint64_t>(x.d.goff + e0) >> 3;  // global group index
-    if (WD == kBF16) {
-      const uint4 r = philox4x32_10(static_cast<uint32_t>(gi), static_cast<uint32_t>(gi >> 32), a.t_lo,
-                                    a.t_hi, a.rk0, a.rk1);
-      rnd[0] = ~r.x & 0xFFFFu; rnd[1] = ~r.x >> 16;
-      rnd[2] = ~r.y & 0xFFFFu; rnd[3] = ~r.y >> 16;
-      rnd[4] = ~r.z & 0xFFFFu; rnd[5] = ~r.z >> 16;
-      rnd[6] = ~r.w & 0xFFFFu; rnd[7] = ~r.w >> 16;
-    } else {
-      const uint64_t b0 = 2ull * gi, b1 = b0 + 1ull;
-      const uint4 r0 = philox4x32_10(static_cast<uint32_t>(b0), static_cast<uint32_t>(b0 >> 32), a.t_lo,
-                                     a.t_hi, a.rk0, a.rk1);
-      const uint4 r1 = philox4x32_10(static_cast<uint32_t>(b1), static_cast<uint32_t>(b1 >> 32), a.t_lo,
-                                     a.t_hi, a.rk0, a.rk1);
-      rnd[0] = r0.x; rnd[1] = r0.y; rnd[2] = r0.z; rnd[3] = r0.w;
-      rnd[4] = r1.x; rnd[5] = r1.y; rnd[6] = r1.z; rnd[7] = r1.w;
-    }
-  }
+  if (SR) group_random_bits<WD>(a, static_cast<uint64_t>(x.d.goff + e0), rnd);
 
   if (WD == kBF16 && !OPT && a.s.cert_ok) {  // certified fast path (see madam_update_cert)
     uint32_t out[8];
@@ -632,6 +722,7 @@ __device__ __forceinline__ void finish_group(const StepArgs& a, const TensorCtx&
     ow[0] = code[0] | (code[1] << 8) | (code[2] << 16) | (code[3] << 24);
     ow[1] = code[4] | (code[5] << 8) | (code[6] << 16) | (code[7] << 24);
     put_e4m3(ow, x.d.w, e0, valid, x.vec);
+    if (x.cc) put_compute(ow, x.cc_scale, x.cc, e0, valid, x.vec);
   } else {
   float wn[8];
 #pragma unroll
@@ -657,24 +748,10 @@ __device__ __forceinline__ void finish_group(const StepArgs& a, const TensorCtx&
       ow[j >> 2] |= e4m3_encode<SR>(__fmul_rn(wn[j], x.enc_scale), SR ? rnd[j] : 0u) << (8 * (j & 3));
     }
     put_e4m3(ow, x.d.w, e0, valid, x.vec);
+    if (x.cc) put_compute(ow, x.cc_scale, x.cc, e0, valid, x.vec);
   }
   }
-  if (MD == kF32) {
-    put_f32(m, x.d.m, e0, valid, x.vec);
-    put_f32(v, x.d.v, e0, valid, x.vec);
-    put_f32(ve, x.d.ve, e0, valid, x.vec);
-  } else {
-    uint32_t om[4], ov[4], oe[4];
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      om[i] = bf16x2_rn(m[2 * i], m[2 * i + 1]);
-      ov[i] = bf16x2_rn(v[2 * i], v[2 * i + 1]);
-      oe[i] = bf16x2_rn(ve[2 * i], ve[2 * i + 1]);
-    }
-    put_bf16(om, x.d.m, e0, valid, x.vec);
-    put_bf16(ov, x.d.v, e0, valid, x.vec);
-    put_bf16(oe, x.d.ve, e0, valid, x.vec);
-  }
+  put_moments<MD>(x, e0, valid, m, v, ve);
 }
 
 // One group of a partial tile, or of a tensor whose arrays are not all staged
@@ -713,6 +790,157 @@ __device__ __noinline__ void general_group(const StepArgs& a, const TensorCtx& x
 }
 
 // ---------------------------------------------------------------------------
+// Block-scaled E4M3 weights: the four threads of a quad hold one 32-element
+// block (8 elements each).  The stored codes decode with the block's old
+// scale; the block's new scale 2^k comes from the largest finite |w'| of the
+// block (current scaling); the codes re-encode x = w' 2^-k.  Every lane of the
+// warp must call this (the block maximum is a quad shuffle); elements j >=
+// valid are padding (valid may be 0) and neither count nor get stored.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint32_t quad_max(uint32_t x) {
+  x = max(x, __shfl_xor_sync(0xFFFFFFFFu, x, 1));
+  return max(x, __shfl_xor_sync(0xFFFFFFFFu, x, 2));
+}
+
+template <int GD, int MD, bool SR, bool OPT>
+__device__ __forceinline__ void finish_block(const StepArgs& a, const TensorCtx& x, int64_t e0, int valid,
+                                             uint32_t h_old, float (&w)[8], float (&g)[8], float (&m)[8],
+                                             float (&v)[8], float (&ve)[8]) {
+  uint32_t rnd[8];
+  if (SR) group_random_bits<kE4M3B>(a, static_cast<uint64_t>(x.d.goff + e0), rnd);
+  const int32_t k_old = fp16_pow2_exponent(h_old);
+  const uint32_t vmask = valid >= kGroup ? 0xFFu : (valid > 0 ? (1u << valid) - 1u : 0u);
+  uint32_t code[8];
+  int32_t k_new;
+  if (!OPT && a.s.cert_ok) {
+    // Certified path (see madam_update_cert).  Keep the fast weights and the
+    // thread's largest error bound et; the block maximum then lies in
+    // [max |w'| - et, max |w'| + et] (outward rounded).  When both ends give
+    // the same exponent (block_exponent is monotone) that is the exact one;
+    // otherwise the quad computes its exact maximum.  Each element's code is
+    // then taken from its interval [w' - et, w' + et] under the new scale
+    // where both ends agree, else from the exact weight.
+    float wf[8];
+    float et = 0.0f, am = 0.0f;
+    uint32_t bad = 0u;
+#pragma unroll
+    for (int j = 0; j < kGroup; ++j) {
+      const CertUpd u = madam_update_cert<false>(a.s, w[j], g[j], m[j], v[j], ve[j]);
+      wf[j] = u.wn;
+      m[j] = u.m; v[j] = u.v; ve[j] = u.ve;
+      if (!u.ok) {
+        bad |= 1u << j;
+      } else {
+        et = fmaxf(et, u.e);
+        if ((vmask >> j) & 1u) am = fmaxf(am, fabsf(u.wn));
+      }
+    }
+    bad &= vmask;
+    const float lo_t = bad ? 0.0f : fmaxf(__fsub_rd(am, et), 0.0f);
+    const float hi_t = bad ? INFINITY : __fadd_ru(am, et);
+    const uint32_t qlo = quad_max(__float_as_uint(lo_t));  // non-negative floats order as their bits
+    const uint32_t qhi = quad_max(__float_as_uint(hi_t));
+    const int32_t kl = block_exponent(qlo, k_old);
+    const bool certain = qlo != 0u && qhi < 0x7E800000u /* 2^126 */ && kl == block_exponent(qhi, k_old);
+    k_new = kl;
+    if (__any_sync(0xFFFFFFFFu, !certain)) {  // exact block maximum for the undecided quads
+      uint32_t amx = 0u;
+      if (!certain) {
+#pragma unroll
+        for (int j = 0; j < kGroup; ++j) {
+          if ((vmask >> j) & 1u) {
+            const uint32_t b = __float_as_uint(madam_wn_exact(a.s, w[j], g[j], m[j], v[j], ve[j])) & 0x7FFFFFFFu;
+            if (b < 0x7F800000u) amx = max(amx, b);
+          }
+        }
+      }
+      amx = quad_max(amx);
+      if (!certain) k_new = block_exponent(amx, k_old);
+    }
+    const float enc = pow2f(-k_new);
+    uint32_t redo = bad;
+#pragma unroll
+    for (int j = 0; j < kGroup; ++j) {
+      bool same;
+      code[j] = e4m3_pair_normal<SR>(__fmul_rd(__fsub_rd(wf[j], et), enc), __fmul_ru(__fadd_ru(wf[j], et), enc),
+                                     SR ? rnd[j] : 0u, same);
+      if (!same) redo |= 1u << j;
+    }
+    redo &= vmask;
+    if (redo) {  // rare: the canonical weight of the undecided elements
+#pragma unroll
+      for (int j = 0; j < kGroup; ++j) {
+        if ((redo >> j) & 1u) {
+          const float xe = madam_wn_exact(a.s, w[j], g[j], m[j], v[j], ve[j]);
+          code[j] = e4m3_encode<SR>(__fmul_rn(xe, enc), SR ? rnd[j] : 0u);
+        }
+      }
+    }
+  } else {
+    float wn[8];
+    uint32_t amx = 0u;
+#pragma unroll
+    for (int j = 0; j < kGroup; ++j) {
+      const Upd u = madam_update<OPT>(a.s, w[j], g[j], m[j], v[j], ve[j]);
+      wn[j] = u.wn; m[j] = u.m; v[j] = u.v; ve[j] = u.ve;
+      const uint32_t b = __float_as_uint(u.wn) & 0x7FFFFFFFu;
+      if (((vmask >> j) & 1u) && b < 0x7F800000u) amx = max(amx, b);
+    }
+    k_new = block_exponent(quad_max(amx), k_old);
+    const float enc = pow2f(-k_new);
+#pragma unroll
+    for (int j = 0; j < kGroup; ++j) code[j] = e4m3_encode<SR>(__fmul_rn(wn[j], enc), SR ? rnd[j] : 0u);
+  }
+  uint32_t ow[2];
+  ow[0] = code[0] | (code[1] << 8) | (code[2] << 16) | (code[3] << 24);
+  ow[1] = code[4] | (code[5] << 8) | (code[6] << 16) | (code[7] << 24);
+  put_e4m3(ow, x.d.w, e0, valid, x.vec);
+  const uint32_t h_new = fp16_pow2_bits(k_new);
+  if ((threadIdx.x & 3) == 0 && valid > 0) x.scale[e0 / kBlock] = static_cast<uint16_t>(h_new);
+  if (x.cc) put_compute(ow, fp16_value(h_new), x.cc, e0, valid, x.vec);
+  put_moments<MD>(x, e0, valid, m, v, ve);
+}
+
+// One group of a partial tile, or of a tensor whose arrays are not all
+// staged: every consumer lane calls this (lanes past the tile's end with no
+// elements), loading each array from the stage when its bytes were staged,
+// else from global memory.
+template <int GD, int MD, bool SR, bool OPT>
+__device__ __noinline__ void general_block_group(const StepArgs& a, const TensorCtx& x, int64_t tile_e0, int count,
+                                                 int c, uint32_t st) {
+  constexpr int GS = esize_of(GD), MS = esize_of(MD);
+  const int rem = count - kGroup * c;
+  const int valid = rem < 0 ? 0 : (rem < kGroup ? rem : kGroup);
+  const int64_t e0 = tile_e0 + kGroup * c;
+  const uint32_t end = static_cast<uint32_t>(kGroup * (c + 1));  // elements through this group
+  // the block's old scale: staged when the tile's scale bytes through this block were
+  const int nblk = (count + kBlock - 1) / kBlock, b = c >> 2;
+  uint32_t h = 0u;
+  if (static_cast<uint32_t>(2 * (b + 1)) <= staged_bytes(x.scale + tile_e0 / kBlock, nblk, 2))
+    h = lds_u16(st + a.off_s + 2 * b);
+  else if (b < nblk)
+    h = x.scale[(tile_e0 / kBlock) + b];
+  float w[8], g[8], m[8], v[8], ve[8];
+  get_e4m3(w, end <= staged_bytes(x.d.w, count, 1), st + kGroup * c, x.d.w, e0, valid, x.vec, fp16_value(h));
+  const bool g_st = end * GS <= staged_bytes(x.g, count, GS);
+  if (GD == kF32) get_f32<true>(g, g_st, st + a.off_g + kGroup * GS * c, x.g, e0, valid, x.vec);
+  else get_bf16<true>(g, g_st, st + a.off_g + kGroup * GS * c, x.g, e0, valid, x.vec);
+  const bool m_st = end * MS <= staged_bytes(x.d.m, count, MS);
+  const bool v_st = end * MS <= staged_bytes(x.d.v, count, MS);
+  const bool e_st = end * MS <= staged_bytes(x.d.ve, count, MS);
+  if (MD == kF32) {
+    get_f32<false>(m, m_st, st + a.off_m + kGroup * MS * c, x.d.m, e0, valid, x.vec);
+    get_f32<false>(v, v_st, st + a.off_v + kGroup * MS * c, x.d.v, e0, valid, x.vec);
+    get_f32<false>(ve, e_st, st + a.off_ve + kGroup * MS * c, x.d.ve, e0, valid, x.vec);
+  } else {
+    get_bf16<false>(m, m_st, st + a.off_m + kGroup * MS * c, x.d.m, e0, valid, x.vec);
+    get_bf16<false>(v, v_st, st + a.off_v + kGroup * MS * c, x.d.v, e0, valid, x.vec);
+    get_bf16<false>(ve, e_st, st + a.off_ve + kGroup * MS * c, x.d.ve, e0, valid, x.vec);
+  }
+  finish_block<GD, MD, SR, OPT>(a, x, e0, valid, h, w, g, m, v, ve);
+}
+
+// ---------------------------------------------------------------------------
 // The step kernel.
 // ---------------------------------------------------------------------------
 template <int WD, int GD, int MD, bool SR, bool OPT>
@@ -747,6 +975,7 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
     int k = a.cta_first[blockIdx.x];
     TensorDesc d = a.desc[k];
     const void* gp = a.grads[k];
+    const uint16_t* sp = WD == kE4M3B ? a.aux[k].scale : nullptr;
     int64_t tiles = (d.numel + kTile - 1) / kTile;
     int s = 0;
     uint32_t use = 0;
@@ -757,6 +986,7 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
         ++k;
         d = a.desc[k];
         gp = a.grads[k];
+        if (WD == kE4M3B) sp = a.aux[k].scale;
         tiles = (d.numel + kTile - 1) / kTile;
       }
       if (use > 0 && !mbar_wait(smem_addr(&empty_bar[s]), (use - 1) & 1u)) {
@@ -769,14 +999,16 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
       const uint32_t nw = staged_bytes(d.w, count, WS), ng = staged_bytes(gp, count, GS);
       const uint32_t nm = staged_bytes(d.m, count, MS), nv = staged_bytes(d.v, count, MS);
       const uint32_t nve = staged_bytes(d.ve, count, MS);
+      const uint32_t ns = WD == kE4M3B ? staged_bytes(sp + e0 / kBlock, (count + kBlock - 1) / kBlock, 2) : 0u;
       const uint32_t bar = smem_addr(&full_bar[s]);
       const uint32_t st = smem0 + static_cast<uint32_t>(s * a.stage_bytes);
-      mbar_arrive_expect_tx(bar, nw + ng + nm + nv + nve);
+      mbar_arrive_expect_tx(bar, nw + ng + nm + nv + nve + ns);
       if (nw) tma_load(st, static_cast<const uint8_t*>(d.w) + e0 * WS, nw, bar, pol);
       if (ng) tma_load(st + a.off_g, static_cast<const uint8_t*>(gp) + e0 * GS, ng, bar, pol);
       if (nm) tma_load(st + a.off_m, static_cast<const uint8_t*>(d.m) + e0 * MS, nm, bar, pol);
       if (nv) tma_load(st + a.off_v, static_cast<const uint8_t*>(d.v) + e0 * MS, nv, bar, pol);
       if (nve) tma_load(st + a.off_ve, static_cast<const uint8_t*>(d.ve) + e0 * MS, nve, bar, pol);
+      if (ns) tma_load(st + a.off_s, sp + e0 / kBlock, ns, bar, pol);
       ++issued;
       if (++s == S) { s = 0; ++use; }
     }
@@ -799,10 +1031,11 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
   load_tensor<WD, GD, MD>(a, k, x);
   int32_t e_next = 0;
   if (WD == kE4M3) {
-    const int32_t e_cur = a.fp8_exp[static_cast<int64_t>(a.e_cur_slot) * n + k];
-    e_next = fp8_next_exponent(a.fp8_amax[static_cast<int64_t>(a.a_cur_slot) * n + k], e_cur);
+    const int32_t e_cur = a.fp8_exp[static_cast<int64_t>(a.e_cur_slot) * n + x.d.ring];
+    e_next = fp8_next_exponent(a.fp8_amax[static_cast<int64_t>(a.a_cur_slot) * n + x.d.ring], e_cur);
     x.dec_scale = pow2f(e_cur);
     x.enc_scale = pow2f(-e_next);
+    x.cc_scale = pow2f(e_next);
   }
   uint32_t amax_bits = 0u;
   int s = 0;
@@ -811,21 +1044,23 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
     if (t >= x.d.tile_off + x.tiles) {  // next tensor: flush this one's E4M3 amax
       if (WD == kE4M3) {
         const uint32_t wmax = __reduce_max_sync(0xFFFFFFFFu, amax_bits);
-        if (lane == 0 && wmax != 0u) atomicMax(&a.fp8_amax[static_cast<int64_t>(a.a_next_slot) * n + k], wmax);
+        if (lane == 0 && wmax != 0u)
+          atomicMax(&a.fp8_amax[static_cast<int64_t>(a.a_next_slot) * n + x.d.ring], wmax);
         amax_bits = 0u;
       }
       do { ++k; load_tensor<WD, GD, MD>(a, k, x); } while (t >= x.d.tile_off + x.tiles);
       if (WD == kE4M3) {
-        const int32_t e_cur = a.fp8_exp[static_cast<int64_t>(a.e_cur_slot) * n + k];
-        e_next = fp8_next_exponent(a.fp8_amax[static_cast<int64_t>(a.a_cur_slot) * n + k], e_cur);
+        const int32_t e_cur = a.fp8_exp[static_cast<int64_t>(a.e_cur_slot) * n + x.d.ring];
+        e_next = fp8_next_exponent(a.fp8_amax[static_cast<int64_t>(a.a_cur_slot) * n + x.d.ring], e_cur);
         x.dec_scale = pow2f(e_cur);
         x.enc_scale = pow2f(-e_next);
+        x.cc_scale = pow2f(e_next);
       }
     }
     const int64_t tile_e0 = (t - x.d.tile_off) * kTile;
     if (WD == kE4M3 && tile_e0 == 0 && c == 0) {  // the CTA holding the tensor's first tile
-      a.fp8_exp[static_cast<int64_t>(a.e_next_slot) * n + k] = e_next;
-      a.fp8_amax[static_cast<int64_t>(a.a_zero_slot) * n + k] = 0u;
+      a.fp8_exp[static_cast<int64_t>(a.e_next_slot) * n + x.d.ring] = e_next;
+      a.fp8_amax[static_cast<int64_t>(a.a_zero_slot) * n + x.d.ring] = 0u;
     }
     if (!__all_sync(0xFFFFFFFFu, mbar_wait(smem_addr(&full_bar[s]), use & 1u))) {  // warp-uniform give-up
       if (a.err && lane == 0) atomicOr(a.err, kErrFullWait);
@@ -836,8 +1071,15 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
       const uint32_t st = smem0 + static_cast<uint32_t>(s * a.stage_bytes);
       const int64_t e0 = tile_e0 + kGroup * c;
       float w[8], g[8], m[8], v[8], ve[8];
-      if (WD == kBF16) get_bf16<false>(w, true, st + kGroup * WS * c, x.d.w, e0, kGroup, true);
-      else get_e4m3(w, true, st + kGroup * WS * c, x.d.w, e0, kGroup, true, x.dec_scale);
+      uint32_t h_old = 0u;
+      if (WD == kBF16) {
+        get_bf16<false>(w, true, st + kGroup * WS * c, x.d.w, e0, kGroup, true);
+      } else if (WD == kE4M3) {
+        get_e4m3(w, true, st + kGroup * WS * c, x.d.w, e0, kGroup, true, x.dec_scale);
+      } else {
+        h_old = lds_u16(st + a.off_s + 2 * (c >> 2));
+        get_e4m3(w, true, st + kGroup * WS * c, x.d.w, e0, kGroup, true, fp16_value(h_old));
+      }
       if (GD == kF32) get_f32<true>(g, true, st + a.off_g + kGroup * GS * c, x.g, e0, kGroup, true);
       else get_bf16<true>(g, true, st + a.off_g + kGroup * GS * c, x.g, e0, kGroup, true);
       if (MD == kF32) {
@@ -851,20 +1093,24 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
       }
       __syncwarp();
       if (lane == 0) mbar_arrive(smem_addr(&empty_bar[s]));
-      finish_group<WD, GD, MD, SR, OPT>(a, x, e0, kGroup, w, g, m, v, ve, amax_bits);
+      if constexpr (WD == kE4M3B) finish_block<GD, MD, SR, OPT>(a, x, e0, kGroup, h_old, w, g, m, v, ve);
+      else finish_group<WD, GD, MD, SR, OPT>(a, x, e0, kGroup, w, g, m, v, ve, amax_bits);
       if (++s == S) { s = 0; ++use; }
       continue;
     }
     // partial tile or unstaged arrays: element-wise fallback, out of line
-    general_group<WD, GD, MD, SR, OPT>(a, x, tile_e0, count, c, smem0 + static_cast<uint32_t>(s * a.stage_bytes),
-                                       amax_bits);
+    if constexpr (WD == kE4M3B)
+      general_block_group<GD, MD, SR, OPT>(a, x, tile_e0, count, c, smem0 + static_cast<uint32_t>(s * a.stage_bytes));
+    else
+      general_group<WD, GD, MD, SR, OPT>(a, x, tile_e0, count, c, smem0 + static_cast<uint32_t>(s * a.stage_bytes),
+                                         amax_bits);
     __syncwarp();
     if (lane == 0) mbar_arrive(smem_addr(&empty_bar[s]));
     if (++s == S) { s = 0; ++use; }
   }
   if (WD == kE4M3) {
     const uint32_t wmax = __reduce_max_sync(0xFFFFFFFFu, amax_bits);
-    if (lane == 0 && wmax != 0u) atomicMax(&a.fp8_amax[static_cast<int64_t>(a.a_next_slot) * n + k], wmax);
+    if (lane == 0 && wmax != 0u) atomicMax(&a.fp8_amax[static_cast<int64_t>(a.a_next_slot) * n + x.d.ring], wmax);
   }
 }
 

@@ -1,8 +1,12 @@
 """MPAdam: torch-tensor marshalling around the C ABI (no arithmetic here).
 
-Holds references to the caller's device tensors (weights, moments) so their
-memory outlives the native state, allocates the E4M3 scale rings with torch,
-and forwards every step to mpadam_step on the current torch stream.
+Holds references to the caller's device tensors (weights, moments, block
+scales, compute copies) so their memory outlives the native state, allocates
+the E4M3 scale rings with torch, and forwards every step to mpadam_step on
+the current torch stream.  `weight_dtype` is one format for the whole list
+("bf16", "e4m3") or a list with one format per tensor ("bf16", "e4m3",
+"e4m3_b32"); the latter, block scales or compute copies go through
+mpadam_create_ex.
 """
 from __future__ import annotations
 
@@ -12,38 +16,59 @@ import torch
 
 from . import _native as N
 
-_STORAGE = {"bf16": torch.bfloat16, "e4m3": torch.uint8, "f32": torch.float32}
+_STORAGE = {"bf16": torch.bfloat16, "e4m3": torch.uint8, "e4m3_b32": torch.uint8, "f32": torch.float32}
 
 
 class MPAdam:
     def __init__(self, w: Sequence[torch.Tensor], m: Sequence[torch.Tensor], v: Sequence[torch.Tensor],
-                 ve: Sequence[torch.Tensor], *, weight_dtype: str = "bf16", grad_dtype: str = "f32",
+                 ve: Sequence[torch.Tensor], *, weight_dtype="bf16", grad_dtype: str = "f32",
                  moment_dtype: str = "f32", rounding: str = "nearest", seed: int = 0,
-                 fp8_exp: Optional[Sequence[int]] = None, first_step: int = 1, **hparams):
+                 fp8_exp: Optional[Sequence[int]] = None, first_step: int = 1,
+                 block_scales: Optional[Sequence[Optional[torch.Tensor]]] = None,
+                 compute: Optional[Sequence[Optional[torch.Tensor]]] = None, **hparams):
         self.w, self.m, self.v, self.ve = list(w), list(m), list(v), list(ve)
+        self.n = len(self.w)
+        per_tensor = not isinstance(weight_dtype, str)
+        self.formats = list(weight_dtype) if per_tensor else [weight_dtype] * self.n
+        self.block_scales = list(block_scales) if block_scales is not None else [None] * self.n
+        self.compute = list(compute) if compute is not None else [None] * self.n
+        if not (len(self.formats) == len(self.block_scales) == len(self.compute) == self.n):
+            raise ValueError("one weight format, block-scale and compute entry per tensor")
         self.weight_dtype, self.grad_dtype, self.moment_dtype = weight_dtype, grad_dtype, moment_dtype
-        for t, dt in [(x, weight_dtype) for x in self.w] + \
-                     [(x, moment_dtype) for x in self.m + self.v + self.ve]:
+        for t, dt in [(x, f) for x, f in zip(self.w, self.formats)] + \
+                     [(x, moment_dtype) for x in self.m + self.v + self.ve] + \
+                     [(x, "bf16") for x in self.compute if x is not None]:
             if t.dtype != _STORAGE[dt] or not t.is_cuda or not t.is_contiguous():
                 raise ValueError(f"expected contiguous CUDA tensors of {_STORAGE[dt]}")
-        self.n = len(self.w)
-        self.cfg = N.make_config(weight_dtype=weight_dtype, grad_dtype=grad_dtype,
+        for x in self.block_scales:
+            if x is not None and (x.dtype != torch.float16 or not x.is_cuda or not x.is_contiguous()):
+                raise ValueError("block scales must be contiguous CUDA float16 tensors")
+        extended = per_tensor or any(x is not None for x in self.block_scales + self.compute)
+        uniform = weight_dtype if not per_tensor else "bf16"
+        self.cfg = N.make_config(weight_dtype="bf16" if extended else uniform, grad_dtype=grad_dtype,
                                  moment_dtype=moment_dtype, rounding=rounding, seed=seed, **hparams)
         dev = self.w[0].device if self.n else torch.device("cuda", torch.cuda.current_device())
         self.fp8_exp_ring = self.fp8_amax_ring = None
-        if weight_dtype == "e4m3":
+        any_e4m3 = "e4m3" in self.formats or (not self.n and weight_dtype == "e4m3")
+        if any_e4m3:
             self.fp8_exp_ring = torch.zeros(2 * max(1, self.n), dtype=torch.int32, device=dev)
             self.fp8_amax_ring = torch.zeros(3 * max(1, self.n), dtype=torch.int32, device=dev)
+        rings = (self.fp8_exp_ring.data_ptr() if any_e4m3 else 0, self.fp8_amax_ring.data_ptr() if any_e4m3 else 0)
+        ptr = lambda t: t.data_ptr() if t is not None else 0
         with torch.cuda.device(dev):
-            self.state = N.mpadam_create(
-                [(a.data_ptr(), b.data_ptr(), c.data_ptr(), d.data_ptr(), a.numel())
-                 for a, b, c, d in zip(self.w, self.m, self.v, self.ve)], self.cfg,
-                self.fp8_exp_ring.data_ptr() if self.fp8_exp_ring is not None else 0,
-                self.fp8_amax_ring.data_ptr() if self.fp8_amax_ring is not None else 0)
-            if weight_dtype == "e4m3":
+            if extended:
+                self.state = N.mpadam_create_ex(
+                    [(a.data_ptr(), b.data_ptr(), c.data_ptr(), d.data_ptr(), a.numel(), f, ptr(bs), ptr(cc))
+                     for a, b, c, d, f, bs, cc in zip(self.w, self.m, self.v, self.ve, self.formats,
+                                                      self.block_scales, self.compute)], self.cfg, *rings)
+            else:
+                self.state = N.mpadam_create(
+                    [(a.data_ptr(), b.data_ptr(), c.data_ptr(), d.data_ptr(), a.numel())
+                     for a, b, c, d in zip(self.w, self.m, self.v, self.ve)], self.cfg, *rings)
+            if "e4m3" in self.formats:
                 if fp8_exp is None:
                     raise ValueError("E4M3 weights need the exponents they are stored with (fp8_exp)")
-                N.mpadam_fp8_init(self.state, list(fp8_exp), first_step,
+                N.mpadam_fp8_init(self.state, [int(e) for e in fp8_exp], first_step,
                                   torch.cuda.current_stream().cuda_stream)
         self.device = dev
 

@@ -3,8 +3,9 @@ step (through the C ABI) and the oracle on the same seeded inputs and compare
 every stored bit.
 
 Tolerance: the library and the oracle follow the same binary32 operation
-sequence, so stored weights, moments and E4M3 scale state must agree bit for
-bit (NaN compares equal to NaN).  That is stricter than the bar of the
+sequence, so stored weights, moments, E4M3 scale state (per-tensor rings and
+FP16 block scales) and BF16 compute copies must agree bit for bit (NaN
+compares equal to NaN).  That is stricter than the bar of the
 method's parity contract (weights within 1 storage ulp on at most 1e-4 of
 elements where rounding is stochastic, binary32 moments within relative
 1e-5); `contract_ok` checks that weaker bar too, for reporting.
@@ -21,7 +22,7 @@ import oracle
 import workloads as W
 from paper_2607_10611_gb300.optimizer import MPAdam
 
-ODT = {"f32": oracle.F32, "bf16": oracle.BF16, "e4m3": oracle.E4M3}
+ODT = {"f32": oracle.F32, "bf16": oracle.BF16, "e4m3": oracle.E4M3, "e4m3_b32": oracle.E4M3_B32}
 HP_KEYS = ("lr_add", "lr_mul", "beta1", "beta2", "eps", "tau", "rmax_pos", "rmax_neg", "g_max",
            "dmult_max", "w_max", "wd_add", "bias_correction")
 
@@ -32,8 +33,14 @@ def oracle_hparams(wl: W.Workload, hp: Dict):
 
 
 def host_tensors(mt: W.Materialized) -> List[dict]:
-    return [dict(w=W.to_numpy_bits(mt.w[k]), g=W.to_numpy_bits(mt.g[k]), m=W.to_numpy_bits(mt.m[k]),
-                 v=W.to_numpy_bits(mt.v[k]), ve=W.to_numpy_bits(mt.ve[k])) for k in range(len(mt.w))]
+    out = []
+    for k in range(len(mt.w)):
+        d = dict(w=W.to_numpy_bits(mt.w[k]), g=W.to_numpy_bits(mt.g[k]), m=W.to_numpy_bits(mt.m[k]),
+                 v=W.to_numpy_bits(mt.v[k]), ve=W.to_numpy_bits(mt.ve[k]))
+        if mt.bscale and mt.bscale[k] is not None:
+            d["bscale"] = W.to_numpy_bits(mt.bscale[k])
+        out.append(d)
+    return out
 
 
 def device_copy(mt: W.Materialized, layout: str = "separate", misalign: int = 0) -> Dict[str, list]:
@@ -42,7 +49,7 @@ def device_copy(mt: W.Materialized, layout: str = "separate", misalign: int = 0)
     out = {}
     for key in ("w", "g", "m", "v", "ve"):
         src = getattr(mt, key)
-        if layout == "flat" and mt.flat:
+        if layout == "flat" and key in mt.flat:
             base = mt.flat[key].to("cuda")
             out[key] = [base[o:o + t.numel()] for o, t in zip(mt.offsets, src)]
         elif misalign:
@@ -55,6 +62,18 @@ def device_copy(mt: W.Materialized, layout: str = "separate", misalign: int = 0)
             out[key] = views
         else:
             out[key] = [t.to("cuda") for t in src]
+    for key, src in (("bscale", mt.bscale), ("cc", mt.cc)):
+        views = []
+        for t in (src or [None] * len(mt.w)):
+            if t is None:
+                views.append(None)
+            elif misalign:
+                buf = torch.zeros(t.numel() + misalign, dtype=t.dtype, device="cuda")
+                views.append(buf[misalign:])
+                views[-1].copy_(t)
+            else:
+                views.append(t.to("cuda"))
+        out[key] = views
     return out
 
 
@@ -99,24 +118,46 @@ class Run:
         self.dev = device_copy(self.mt, layout, misalign)
         self.ohp = oracle_hparams(wl, self.hp)
         gkw = {k: v for k, v in self.hp.items() if k in HP_KEYS}
+        self.formats = list(self.mt.formats) if self.mt.formats else [wl.weight_dtype] * len(self.mt.w)
+        extended = wl.weight_dtype not in ("bf16", "e4m3") or bool(wl.format_list) or \
+            any(x is not None for x in self.dev["cc"])
         self.opt = MPAdam(self.dev["w"], self.dev["m"], self.dev["v"], self.dev["ve"],
-                          weight_dtype=wl.weight_dtype, grad_dtype=wl.grad_dtype,
+                          weight_dtype=self.formats if extended else wl.weight_dtype, grad_dtype=wl.grad_dtype,
                           moment_dtype=wl.moment_dtype, rounding=wl.rounding, seed=wl.seed,
-                          fp8_exp=self.mt.fp8_exp, **gkw)
-        self.fp8 = oracle.fp8_init(self.host, self.mt.fp8_exp) if wl.weight_dtype == "e4m3" else None
-        self.wdt, self.gdt, self.mdt = ODT[wl.weight_dtype], ODT[wl.grad_dtype], ODT[wl.moment_dtype]
+                          fp8_exp=self.mt.fp8_exp,
+                          block_scales=self.dev["bscale"] if extended else None,
+                          compute=self.dev["cc"] if extended else None, **gkw)
+        self.e4m3 = [k for k, f in enumerate(self.formats) if f == "e4m3"]
+        self.fp8 = None
+        if self.e4m3:
+            self.fp8 = [None] * len(self.host)
+            for k in self.e4m3:
+                self.fp8[k] = oracle.fp8_init([self.host[k]], [self.mt.fp8_exp[k]])[0]
+        self.wdt = [ODT[f] for f in self.formats]
+        self.gdt, self.mdt = ODT[wl.grad_dtype], ODT[wl.moment_dtype]
+        self.stepped = False
 
     def step(self, t: int):
         self.opt.step(self.dev["g"], t)
         oracle.step(self.host, wdt=self.wdt, gdt=self.gdt, mdt=self.mdt, hp=self.ohp, t=t,
                     fp8_state=self.fp8)
         torch.cuda.synchronize()
+        self.stepped = True
         assert self.opt.device_status() == 0, "a bounded wait in the step kernel gave up"
 
 
-    def compare(self, t_next: int) -> Dict[str, int]:
-        """Mismatch counts per array (and the E4M3 scale state read for step t_next)."""
-        res = {"w": 0, "m": 0, "v": 0, "ve": 0, "elements": 0, "contract_ok": True}
+    def expected_compute_copy(self, k: int) -> np.ndarray:
+        """The oracle's BF16 compute copy of tensor k's current stored weights."""
+        h = self.host[k]
+        if self.formats[k] == "e4m3_b32":
+            return oracle.dequant_bf16(h["w"], bscale=h["bscale"])
+        return oracle.dequant_bf16(h["w"], e=self.fp8[k][0])
+
+    def compare(self, t_next: int, compute_copy: bool = True) -> Dict[str, int]:
+        """Mismatch counts per array (and the E4M3 scale state read for step
+        t_next); compute copies are checked when compute_copy, once a step has
+        written them."""
+        res = {"w": 0, "m": 0, "v": 0, "ve": 0, "bscale": 0, "cc": 0, "elements": 0, "contract_ok": True}
         for k in range(len(self.host)):
             h = self.host[k]
             res["elements"] += h["w"].size
@@ -126,14 +167,19 @@ class Run:
             res["m"] += mismatches(gm, h["m"])
             res["v"] += mismatches(W.to_numpy_bits(self.dev["v"][k]), h["v"])
             res["ve"] += mismatches(W.to_numpy_bits(self.dev["ve"][k]), h["ve"])
-            if h["w"].size and not contract_ok(gw, h["w"], gm, h["m"], self.wl.weight_dtype):
+            if "bscale" in h:
+                res["bscale"] += mismatches(W.to_numpy_bits(self.dev["bscale"][k]), h["bscale"])
+            if compute_copy and self.stepped and self.dev["cc"][k] is not None and h["w"].size:
+                res["cc"] += mismatches(W.to_numpy_bits(self.dev["cc"][k]), self.expected_compute_copy(k))
+            fmt = "bf16" if self.formats[k] == "bf16" else "e4m3"
+            if h["w"].size and not contract_ok(gw, h["w"], gm, h["m"], fmt):
                 res["contract_ok"] = False
         if self.fp8 is not None:
             exps = self.opt.fp8_exponents(t_next)
             amax = self.opt.fp8_amax(t_next).cpu().numpy()
-            res["fp8_exp"] = sum(int(e != s[0]) for e, s in zip(exps, self.fp8))
-            res["fp8_amax"] = sum(int(np.float32(a).view(np.uint32) != np.float32(s[1]).view(np.uint32))
-                                  for a, s in zip(amax, self.fp8))
+            res["fp8_exp"] = sum(int(exps[k] != self.fp8[k][0]) for k in self.e4m3)
+            res["fp8_amax"] = sum(int(np.float32(amax[k]).view(np.uint32) != np.float32(self.fp8[k][1]).view(np.uint32))
+                                  for k in self.e4m3)
         return res
 
     def close(self):

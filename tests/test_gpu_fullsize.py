@@ -178,3 +178,68 @@ def test_llama_1p5b_e4m3():
     opt.close()
     del mt, opt
     _free()
+
+
+def test_llama_1p5b_mixed_sampled_blocks_two_steps():
+    """The paper's FP8 regime at full size (linears block-scaled E4M3 with
+    BF16 compute copies, the rest BF16): whole sampled 32-element blocks of
+    every linear (a block's new scale depends on all of it) and sampled
+    elements of every BF16 tensor, two steps, in the benchmark's launch
+    configuration."""
+    from paper_2607_10611_gb300.optimizer import MPAdam
+    wl = W.CONFIGS["llama_1p5b_mixed"]
+    mt = W.materialize(wl, "cuda", layout="flat")
+    opt = MPAdam(mt.w, mt.m, mt.v, mt.ve, weight_dtype=mt.formats, grad_dtype=wl.grad_dtype,
+                 moment_dtype=wl.moment_dtype, rounding=wl.rounding, seed=wl.seed,
+                 block_scales=mt.bscale, compute=mt.cc)
+    hp = oracle.hparams(stochastic=1, seed=wl.seed)
+    gd, md = ODT[wl.grad_dtype], ODT[wl.moment_dtype]
+    rng = np.random.default_rng(17)
+    keys = ("w", "g", "m", "v", "ve")
+    picks = []  # (k, element indices, block indices or None)
+    for k, (n, f) in enumerate(zip(wl.numels, mt.formats)):
+        if f == "e4m3_b32":
+            nb = (n + 31) // 32
+            blocks = np.unique(np.concatenate([[0, nb - 1], rng.integers(0, nb, 150)]))
+            idx = np.concatenate([np.arange(32 * b, min(n, 32 * b + 32)) for b in blocks])
+            picks.append((k, idx, blocks))
+        else:
+            idx = np.unique(np.concatenate([[0, n - 1], rng.integers(0, n, 4000)]))
+            picks.append((k, idx, None))
+
+    def gather(k, idx, blocks):
+        p = torch.from_numpy(idx).to("cuda")
+        d = {key: _bits(getattr(mt, key)[k].index_select(0, p)) for key in keys}
+        if blocks is not None:
+            d["bscale"] = W.to_numpy_bits(mt.bscale[k].index_select(0, torch.from_numpy(blocks).to("cuda")))
+            d["cc"] = _bits(mt.cc[k].index_select(0, p))
+        return d
+
+    host = [gather(*pk) for pk in picks]
+    for t in (1, 2):
+        opt.step(mt.g, t)
+        torch.cuda.synchronize()
+        for (k, idx, blocks), h in zip(picks, host):
+            goff = mt.offsets[k]
+            if blocks is None:
+                oracle.step_elements(hp, t, oracle.BF16, gd, md, h["w"], h["g"], h["m"], h["v"], h["ve"],
+                                     gidx=goff + idx)
+            else:
+                pos = 0
+                for j, b in enumerate(blocks):
+                    ln = min(32, wl.numels[k] - 32 * int(b))
+                    sl = slice(pos, pos + ln)
+                    arrs = [h[key][sl] for key in keys]
+                    bs = h["bscale"][j:j + 1]
+                    oracle.step_block_e4m3(hp, t, gd, md, arrs[0], bs, *arrs[1:], gidx0=goff + 32 * int(b))
+                    h["cc"][sl] = oracle.dequant_bf16(arrs[0], bscale=bs)
+                    pos += ln
+            got = gather(k, idx, blocks)
+            _assert_same(got, h, f"llama_1p5b_mixed tensor {k} step {t}")
+            if blocks is not None:
+                assert np.array_equal(got["bscale"], h["bscale"]), f"tensor {k} step {t}: block scales"
+                assert np.array_equal(got["cc"], h["cc"]), f"tensor {k} step {t}: compute copy"
+    assert opt.device_status() == 0
+    opt.close()
+    del mt, opt
+    _free()

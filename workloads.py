@@ -5,8 +5,10 @@ tests/benchmark.  It draws weights, gradients and optimizer states; it holds
 none of the M+Adam arithmetic (no moment update, no rounding rule, no scale
 rule).  The FP8 initial weights are produced with torch's own float8_e4m3fn
 cast of a pre-scaled draw, with a per-role power-of-two exponent chosen from
-the draw's standard deviation: an input recipe, not the optimizer's delayed
-scale rule.
+the draw's standard deviation (per-tensor scaling), or per 32-element block
+the power of two at or above the block's largest |w| / 448 computed with
+torch in binary64 (block scaling): an input recipe, not the optimizer's
+scale rules.
 
 Stand-ins: the paper trains LLaMA-style decoders on C4/EN (Sec. 5.2, the
 model-architecture table of Appendix C).  An optimizer step needs no data, so
@@ -35,14 +37,14 @@ ALIGN = 8  # elements; tensor starts in the global index space
 class TensorSpec:
     name: str
     numel: int
-    role: str  # "matrix" | "embedding" | "bias" | "norm" | "flat"
+    role: str  # "matrix" | "head" | "embedding" | "bias" | "norm" | "flat"
 
 
 @dataclass(frozen=True)
 class Workload:
     name: str
     specs: tuple
-    weight_dtype: str          # "bf16" | "e4m3"
+    weight_dtype: str          # "bf16" | "e4m3" | "e4m3_b32" | "mixed_b32" (see format_of)
     grad_dtype: str            # "f32" | "bf16"
     moment_dtype: str          # "f32" | "bf16"
     rounding: str              # "nearest" | "stochastic"
@@ -53,7 +55,23 @@ class Workload:
     grad: tuple = ("normal", 1e-3)  # ("normal", s) | ("normal_logu", lo, hi) | ("student_t_logu", nu, lo, hi)
     norm_gain: float = 1.0     # initial value of norm gains
     bias_zero: bool = True     # biases start at exactly 0
+    compute_copy: bool = False  # E4M3 tensors also get a BF16 compute copy
+    format_list: tuple = ()    # explicit weight format per tensor (overrides weight_dtype)
     description: str = ""
+
+    def format_of(self, spec: "TensorSpec") -> str:
+        """Weight format of one tensor.  "mixed_b32" is the paper's FP8 regime
+        (Sec. 5.2): linear layers block-scaled E4M3, embeddings, norms, biases
+        and the LM head BF16."""
+        if self.weight_dtype == "mixed_b32":
+            return "e4m3_b32" if spec.role == "matrix" else "bf16"
+        return self.weight_dtype
+
+    @property
+    def formats(self) -> List[str]:
+        if self.format_list:
+            return list(self.format_list)
+        return [self.format_of(s) for s in self.specs]
 
     @property
     def numels(self) -> List[int]:
@@ -121,7 +139,7 @@ def llama_specs(layers, d, ffn, vocab) -> tuple:
             TensorSpec(p + "input_layernorm", d, "norm"),
             TensorSpec(p + "post_attention_layernorm", d, "norm"),
         ]
-    s += [TensorSpec("norm", d, "norm"), TensorSpec("lm_head", vocab * d, "matrix")]
+    s += [TensorSpec("norm", d, "norm"), TensorSpec("lm_head", vocab * d, "head")]
     return tuple(s)
 
 
@@ -161,6 +179,17 @@ def _llama15(layers=24, d=2048, ffn=5632, vocab=32000, name="llama_1p5b"):
                     "(std log-uniform [1e-5,1e-2]), fp32 moments, stochastic rounding")
 
 
+def _llama15_mixed(layers=24, d=2048, ffn=5632, vocab=32000, name="llama_1p5b_mixed"):
+    return Workload(
+        name=name, specs=llama_specs(layers, d, ffn, vocab),
+        weight_dtype="mixed_b32", grad_dtype="bf16", moment_dtype="f32", rounding="stochastic",
+        steps=10, grad=("student_t_logu", 3.0, 1e-5, 1e-2), compute_copy=True,
+        description="LLaMA-style 1.5B list in the paper's FP8 regime: linear layers E4M3 with one "
+                    "FP16 power-of-two scale per 32 weights and a BF16 compute copy written by the "
+                    "step, embeddings / norms / LM head BF16; bf16 Student-t(3) grads scaled per "
+                    "tensor, fp32 moments, stochastic rounding")
+
+
 def _llama7(layers=32, d=4096, ffn=11008, vocab=32000, name="llama_7b"):
     return Workload(
         name=name, specs=llama_specs(layers, d, ffn, vocab),
@@ -186,6 +215,7 @@ CONFIGS: Dict[str, Workload] = {
     "llama_1p5b": _llama15(),
     "llama_7b": _llama7(),
     "ragged_20k": _ragged(),
+    "llama_1p5b_mixed": _llama15_mixed(),
 }
 
 # Same distributions and formats at sizes the oracle finishes in seconds,
@@ -196,13 +226,15 @@ SMALL: Dict[str, Workload] = {
     "llama_1p5b": _llama15(layers=2, d=128, ffn=344, vocab=517, name="llama15_small"),
     "llama_7b": _llama7(layers=2, d=128, ffn=344, vocab=517, name="llama7_small"),
     "ragged_20k": _ragged(n=300, max_log2=13, name="ragged_small"),
+    "llama_1p5b_mixed": _llama15_mixed(layers=2, d=128, ffn=344, vocab=517, name="llama15_mixed_small"),
 }
 
 
 # ---------------------------------------------------------------------------
 # Materialisation
 # ---------------------------------------------------------------------------
-_TORCH = {"f32": torch.float32, "bf16": torch.bfloat16, "e4m3": torch.uint8}
+_TORCH = {"f32": torch.float32, "bf16": torch.bfloat16, "e4m3": torch.uint8, "e4m3_b32": torch.uint8}
+BLOCK = 32  # elements per block scale (block-scaled E4M3)
 
 
 def _gen(device, seed, k, salt):
@@ -218,6 +250,21 @@ def _grad_std(wl: Workload, k: int) -> float:
     lo, hi = (wl.grad[1], wl.grad[2]) if kind == "normal_logu" else (wl.grad[2], wl.grad[3])
     u = torch.rand(1, generator=_gen("cpu", wl.seed, k, 5), dtype=torch.float64).item()
     return math.exp(math.log(lo) + u * (math.log(hi) - math.log(lo)))
+
+
+def block_initial_scales(wf: torch.Tensor, default_exp: int) -> torch.Tensor:
+    """Float16 power-of-two scale per 32-element block: 2^k with k the
+    smallest integer such that the block's largest |w| fits under 448 * 2^k
+    (evaluated in binary64 by torch), clamped to [-24, 15]; all-zero blocks
+    take 2^default_exp."""
+    n = wf.numel()
+    nb = (n + BLOCK - 1) // BLOCK
+    pad = torch.zeros(nb * BLOCK, dtype=torch.float64, device=wf.device)
+    pad[:n] = wf.to(torch.float64).abs()
+    amax = pad.view(nb, BLOCK).amax(dim=1)
+    k = torch.ceil(torch.log2(amax / 448.0))
+    k = torch.where(amax > 0, k, torch.full_like(k, float(default_exp))).clamp_(-24, 15)
+    return torch.exp2(k).to(torch.float16)
 
 
 def fp8_initial_exponent(role: str, w_std: float, norm_gain: float) -> int:
@@ -241,6 +288,9 @@ class Materialized:
     ve: List[torch.Tensor]
     fp8_exp: Optional[List[int]] = None
     flat: Dict[str, torch.Tensor] = field(default_factory=dict)
+    formats: List[str] = field(default_factory=list)
+    bscale: List[Optional[torch.Tensor]] = field(default_factory=list)  # float16 block scales
+    cc: List[Optional[torch.Tensor]] = field(default_factory=list)      # BF16 compute copies
 
 
 def _alloc(kind_dtype, numels, offsets, length, device, layout):
@@ -257,19 +307,32 @@ def materialize(wl: Workload, device="cpu", layout="separate", warm_state=False)
     numels = wl.numels
     offsets = global_offsets(numels)
     length = global_length(numels)
-    wdt, gdt, mdt = _TORCH[wl.weight_dtype], _TORCH[wl.grad_dtype], _TORCH[wl.moment_dtype]
+    formats = wl.formats
+    uniform = len(set(formats)) <= 1
+    wdt = _TORCH[formats[0]] if formats else torch.bfloat16
+    gdt, mdt = _TORCH[wl.grad_dtype], _TORCH[wl.moment_dtype]
     flat = {}
-    fw, w = _alloc(wdt, numels, offsets, length, device, layout)
+    if uniform:
+        fw, w = _alloc(wdt, numels, offsets, length, device, layout)
+    else:  # weights of different element sizes: one allocation per tensor
+        fw, w = None, [torch.zeros(n, dtype=_TORCH[f], device=device) for n, f in zip(numels, formats)]
     fg, g = _alloc(gdt, numels, offsets, length, device, layout)
     fm, m = _alloc(mdt, numels, offsets, length, device, layout)
     fv, v = _alloc(mdt, numels, offsets, length, device, layout)
     fve, ve = _alloc(mdt, numels, offsets, length, device, layout)
     if layout == "flat":
-        flat = {"w": fw, "g": fg, "m": fm, "v": fv, "ve": fve}
-    fp8_exp = [] if wl.weight_dtype == "e4m3" else None
+        flat = {"g": fg, "m": fm, "v": fv, "ve": fve}
+        if uniform:
+            flat["w"] = fw
+    fp8_exp = [] if "e4m3" in formats else None
+    bscale = [torch.ones((n + BLOCK - 1) // BLOCK, dtype=torch.float16, device=device) if f == "e4m3_b32" else None
+              for n, f in zip(numels, formats)]
+    cc = [torch.zeros(n, dtype=torch.bfloat16, device=device) if wl.compute_copy and f != "bf16" else None
+          for n, f in zip(numels, formats)]
 
     for k, spec in enumerate(wl.specs):
         n = spec.numel
+        fmt = formats[k]
         if n == 0:
             if fp8_exp is not None:
                 fp8_exp.append(0)
@@ -285,13 +348,20 @@ def materialize(wl: Workload, device="cpu", layout="separate", warm_state=False)
             if wl.zero_frac > 0:
                 z = torch.rand(n, generator=gw, device=device) < wl.zero_frac
                 wf[z] = 0.0
-        if wl.weight_dtype == "e4m3":
-            e0 = fp8_initial_exponent(spec.role, wl.w_std, wl.norm_gain)
-            fp8_exp.append(e0)
+        if fp8_exp is not None:
+            fp8_exp.append(fp8_initial_exponent(spec.role, wl.w_std, wl.norm_gain) if fmt == "e4m3" else 0)
+        if fmt == "e4m3":
+            e0 = fp8_exp[-1]
             q = (wf * (2.0 ** -e0)).clamp_(-448.0, 448.0).to(torch.float8_e4m3fn)
             w[k].copy_(q.view(torch.uint8))
+        elif fmt == "e4m3_b32":
+            sc = block_initial_scales(wf, fp8_initial_exponent(spec.role, wl.w_std, wl.norm_gain))
+            bscale[k].copy_(sc)
+            per = sc.to(torch.float32).repeat_interleave(BLOCK)[:n]
+            q = (wf / per).clamp_(-448.0, 448.0).to(torch.float8_e4m3fn)
+            w[k].copy_(q.view(torch.uint8))
         else:
-            w[k].copy_(wf.to(wdt))
+            w[k].copy_(wf.to(torch.bfloat16))
         # gradients
         gg = _gen(device, wl.seed, k, 2)
         sd = _grad_std(wl, k)
@@ -315,13 +385,13 @@ def materialize(wl: Workload, device="cpu", layout="separate", warm_state=False)
             m[k].copy_(mf.to(mdt))
             v[k].copy_(vf.to(mdt))
             ve[k].copy_(vef.to(mdt))
-    return Materialized(wl, offsets, length, w, g, m, v, ve, fp8_exp, flat)
+    return Materialized(wl, offsets, length, w, g, m, v, ve, fp8_exp, flat, formats, bscale, cc)
 
 
 def to_numpy_bits(t: torch.Tensor):
-    """Host numpy view: float32 stays float32, bfloat16 becomes uint16 bits,
-    uint8 (E4M3 codes) stays uint8."""
+    """Host numpy view: float32 stays float32, bfloat16 and float16 become
+    uint16 bits, uint8 (E4M3 codes) stays uint8."""
     t = t.detach().to("cpu").contiguous()
-    if t.dtype == torch.bfloat16:
+    if t.dtype in (torch.bfloat16, torch.float16):
         return t.view(torch.int16).numpy().view("uint16").copy()
     return t.numpy().copy()
