@@ -269,12 +269,38 @@ def run_gpu(wl, steps: int, warmup: int, rank: int, e2e_steps: int):
         res["e2e_ms"] = e0.elapsed_time(e1) / e2e_steps
         res["h2d"] = sum(x.numel() for x in mt.g) * BYTES[wl.grad_dtype]
         res["d2h"] = sum(x.numel() for x in mt.w) * BYTES[wl.weight_dtype]
+        res["link_ms"] = host_link_ms(hg, mt.flat["g"], hw, mt.flat["w"], stream)
         del hg, hw, hgs, hws
     opt.close()
     del mt, opt
     torch.cuda.synchronize()
     torch.cuda.empty_cache()
     return res
+
+
+def host_link_ms(h_src, d_dst, h_dst, d_src, stream, reps: int = 3) -> float:
+    """The host link alone: the same bytes the end-to-end step moves (pinned
+    host -> device and device -> host, concurrently on two streams), best of
+    `reps`, in ms.  d_dst is rewritten with the values it already holds."""
+    import torch
+    up, down = torch.cuda.Stream(), torch.cuda.Stream()
+    best = float("inf")
+    for _ in range(reps):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize()
+        a.record(stream)
+        up.wait_event(a)
+        down.wait_event(a)
+        with torch.cuda.stream(up):
+            d_dst.copy_(h_src, non_blocking=True)
+        with torch.cuda.stream(down):
+            h_dst.copy_(d_src, non_blocking=True)
+        stream.wait_stream(up)
+        stream.wait_stream(down)
+        b.record(stream)
+        torch.cuda.synchronize()
+        best = min(best, a.elapsed_time(b))
+    return best
 
 
 def max_over_ranks(ms: float, device: str) -> float:
@@ -312,7 +338,10 @@ def summarize(wl, res, n_gpus, peak, peak_kind):
     if "e2e_ms" in res:
         out["e2e"] = {"value": n_gpus * n / (res["e2e_ms"] * 1e-3) / 1e9, "unit": UNIT,
                       "h2d_bytes_per_step": res["h2d"], "d2h_bytes_per_step": res["d2h"],
-                      "ms_per_step": res["e2e_ms"]}
+                      "ms_per_step": res["e2e_ms"],
+                      "host_link_ms": res["link_ms"],
+                      "host_link_gbs": (res["h2d"] + res["d2h"]) / (res["link_ms"] * 1e-3) / 1e9,
+                      "frac_of_host_link_bound": res["link_ms"] / res["e2e_ms"]}
     return out
 
 
