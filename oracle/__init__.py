@@ -20,10 +20,11 @@ import numpy as np
 
 from . import build as _build
 
-F32, BF16, E4M3, E4M3_B32 = 0, 1, 2, 3
-DTYPES = {"f32": F32, "bf16": BF16, "e4m3": E4M3, "e4m3_b32": E4M3_B32}
+F32, BF16, E4M3, E4M3_B32, NVFP4 = 0, 1, 2, 3, 4
+DTYPES = {"f32": F32, "bf16": BF16, "e4m3": E4M3, "e4m3_b32": E4M3_B32, "nvfp4": NVFP4}
 ALIGN = 8
 BLOCK = 32
+FP4_BLOCK = 16
 
 _LIB = None
 
@@ -96,6 +97,14 @@ def lib() -> ctypes.CDLL:
         L.orc_step_block_e4m3.argtypes = [i64, i64, i32, i32, P, P, P, P, P, P, P, i64]
         L.orc_step_block_e4m3.restype = i32
         L.orc_dequant_bf16.argtypes = [i64, P, i32, P, P]
+        L.orc_e2m1_rne.argtypes = [ctypes.c_float]; L.orc_e2m1_rne.restype = ctypes.c_uint8
+        L.orc_e2m1_sr.argtypes = [ctypes.c_float, ctypes.c_uint32]; L.orc_e2m1_sr.restype = ctypes.c_uint8
+        L.orc_e2m1_decode.argtypes = [ctypes.c_uint8]; L.orc_e2m1_decode.restype = ctypes.c_float
+        L.orc_nvfp4_scale_code.argtypes = [ctypes.c_float, ctypes.c_float, i32]
+        L.orc_nvfp4_scale_code.restype = i32
+        L.orc_step_nvfp4.argtypes = [i64, i64, i32, i32, P, P, ctypes.c_float, P, P, P, P, P, i64]
+        L.orc_step_nvfp4.restype = i32
+        L.orc_dequant_nvfp4_bf16.argtypes = [i64, P, P, ctypes.c_float, P]
         _LIB = L
     return _LIB
 
@@ -242,6 +251,61 @@ def dequant_bf16(q, e: int = 0, bscale=None) -> np.ndarray:
     return out
 
 
+def e2m1_rne(x) -> np.ndarray:
+    return np.array([lib().orc_e2m1_rne(float(v)) for v in np.atleast_1d(np.asarray(x, np.float32))], np.uint8)
+
+
+def e2m1_sr(x, r32) -> np.ndarray:
+    xs = np.atleast_1d(np.asarray(x, np.float32))
+    rs = np.atleast_1d(np.asarray(r32, np.uint32))
+    return np.array([lib().orc_e2m1_sr(float(v), int(r)) for v, r in zip(xs, rs)], np.uint8)
+
+
+def e2m1_decode(c) -> np.ndarray:
+    return np.array([lib().orc_e2m1_decode(int(v)) for v in np.atleast_1d(c)], np.float32)
+
+
+def nvfp4_scale_code(amax: float, G: float, c_old: int) -> int:
+    return int(lib().orc_nvfp4_scale_code(ctypes.c_float(amax), ctypes.c_float(G), int(c_old)))
+
+
+def nvfp4_unpack(q, n: int) -> np.ndarray:
+    """Codes of n elements from packed bytes (even element in the low nibble)."""
+    q = np.asarray(q, np.uint8)
+    out = np.empty(2 * q.size, np.uint8)
+    out[0::2] = q & 0x0F
+    out[1::2] = q >> 4
+    return out[:n]
+
+
+def nvfp4_pack(codes) -> np.ndarray:
+    c = np.asarray(codes, np.uint8)
+    if c.size % 2:
+        c = np.concatenate([c, np.zeros(1, np.uint8)])
+    return (c[0::2] & 0x0F) | (c[1::2] << 4)
+
+
+def step_nvfp4(hp: HParams, t: int, gdt: int, mdt: int, n: int, q, bscale, G: float, g, m, v, ve,
+               gidx0: int = 0) -> None:
+    """One step of a whole NVFP4 tensor of n elements: q (packed codes),
+    bscale (E4M3 block-scale codes) and the moments update in place."""
+    for a in (q, bscale, g, m, v, ve):
+        assert a.flags.c_contiguous
+    assert q.size == (n + 1) // 2 and bscale.size == -(-n // FP4_BLOCK)
+    rc = lib().orc_step_nvfp4(n, gidx0, gdt, mdt, _p(q), _p(bscale), ctypes.c_float(G), _p(g), _p(m), _p(v),
+                              _p(ve), ctypes.byref(hp), t)
+    if rc != 0:
+        raise ValueError("invalid arguments")
+
+
+def dequant_nvfp4_bf16(n: int, q, bscale, G: float) -> np.ndarray:
+    q = _c(q, np.uint8)
+    bs = _c(bscale, np.uint8)
+    out = np.zeros(n, np.uint16)
+    lib().orc_dequant_nvfp4_bf16(n, _p(q), _p(bs), ctypes.c_float(G), _p(out))
+    return out
+
+
 def global_offsets(numels) -> List[int]:
     """First global element index of each tensor: the previous tensor's end
     rounded up to a multiple of 8."""
@@ -267,7 +331,8 @@ def step(tensors, *, wdt, gdt: int, mdt: int, hp: HParams, t: int,
     step]; it is advanced in place: the weights are re-encoded with the
     exponent chosen from that largest |w|, and the new largest |w| is recorded.
     For E4M3_B32 storage the dict also holds "bscale" (FP16 block scales,
-    updated in place)."""
+    updated in place); for NVFP4 storage "w" holds packed codes, "bscale" the
+    E4M3 block-scale codes (updated in place) and "gscale" the tensor scale."""
     offs = global_offsets([d["w"].size for d in tensors])
     formats = list(wdt) if isinstance(wdt, (list, tuple)) else [wdt] * len(tensors)
     for k, d in enumerate(tensors):
@@ -277,6 +342,9 @@ def step(tensors, *, wdt, gdt: int, mdt: int, hp: HParams, t: int,
         if wdt == E4M3_B32:
             step_block_e4m3(hp, t, gdt, mdt, d["w"], d["bscale"], d["g"], d["m"], d["v"], d["ve"],
                             gidx0=offs[k])
+        elif wdt == NVFP4:
+            step_nvfp4(hp, t, gdt, mdt, d["g"].size, d["w"], d["bscale"], d["gscale"], d["g"], d["m"],
+                       d["v"], d["ve"], gidx0=offs[k])
         elif wdt == E4M3:
             e_cur, a_cur = fp8_state[k]
             e_next = fp8_next_exponent(a_cur, e_cur)

@@ -447,6 +447,118 @@ void orc_dequant_bf16(int64_t n, const uint8_t* q, int32_t e, const uint16_t* bs
 }
 
 /* ------------------------------------------------------------------------ */
+/* NVFP4: E2M1 payload, E4M3 block scales (16 elements), binary32 tensor     */
+/* scale.  The paper stores master weights in NVFP4 (Sec. 5.2, the results   */
+/* table's NVFP4/FP8 rows) and writes a block's weights as payload times     */
+/* block scale (the FP4 block-scale paragraph of the ablation appendix).     */
+/* ------------------------------------------------------------------------ */
+static const float e2m1_grid[8] = {0.0f, 0.5f, 1.0f, 1.5f, 2.0f, 3.0f, 4.0f, 6.0f};
+
+float orc_e2m1_decode(uint8_t c) {
+  float v = e2m1_grid[c & 7u];
+  return (c & 8u) ? -v : v;
+}
+
+/* Magnitude index of the grid point at or below a (a in [0, 6)), and the
+ * fraction of the way to the next grid point, in binary64 (exact). */
+static uint32_t e2m1_floor(float a, double* frac) {
+  uint32_t i = 0;
+  while (i < 6 && (double)e2m1_grid[i + 1] <= (double)a) ++i;
+  *frac = ((double)a - (double)e2m1_grid[i]) / ((double)e2m1_grid[i + 1] - (double)e2m1_grid[i]);
+  return i;
+}
+
+uint8_t orc_e2m1_rne(float x) {
+  if (isnan(x)) return 0;
+  uint32_t sign = signbit(x) ? 8u : 0u;
+  float a = fabsf(x);
+  if (a >= 6.0f) return (uint8_t)(sign | 7u);
+  double frac;
+  uint32_t i = e2m1_floor(a, &frac);
+  if (frac > 0.5 || (frac == 0.5 && (i & 1u))) i += 1;   /* ties to the even code (mantissa 0) */
+  return (uint8_t)(sign | i);
+}
+
+uint8_t orc_e2m1_sr(float x, uint32_t r32) {
+  if (isnan(x)) return 0;
+  uint32_t sign = signbit(x) ? 8u : 0u;
+  float a = fabsf(x);
+  if (a >= 6.0f) return (uint8_t)(sign | 7u);
+  double frac;
+  uint32_t i = e2m1_floor(a, &frac);
+  double thr = floor(frac * 4294967296.0);                /* exact: frac has few bits */
+  if ((double)r32 < thr) i += 1;
+  return (uint8_t)(sign | i);
+}
+
+int32_t orc_nvfp4_scale_code(float amax, float G, int32_t c_old) {
+  if (!(amax > 0.0f)) return c_old;
+  for (int32_t c = 1; c <= 126; ++c) {
+    float d = orc_e4m3_decode((uint8_t)c) * G;
+    float top = 6.0f * d;
+    if (top >= amax) return c;
+  }
+  return 126;
+}
+
+static uint8_t nvfp4_get(const uint8_t* q, int64_t k) {
+  return (uint8_t)((k & 1) ? (q[k >> 1] >> 4) : (q[k >> 1] & 0x0Fu));
+}
+
+static void nvfp4_put(uint8_t* q, int64_t k, uint8_t c) {
+  if (k & 1) q[k >> 1] = (uint8_t)((q[k >> 1] & 0x0Fu) | (c << 4));
+  else q[k >> 1] = (uint8_t)((q[k >> 1] & 0xF0u) | (c & 0x0Fu));
+}
+
+int32_t orc_step_nvfp4(int64_t n, int64_t gidx0, int32_t gdt, int32_t mdt, uint8_t* q, uint8_t* bscale,
+                       float G, const void* g, void* m, void* v, void* ve, const orc_hparams* hp, int64_t t) {
+  if (gdt != ORC_F32 && gdt != ORC_BF16) return -1;
+  if (mdt != ORC_F32 && mdt != ORC_BF16) return -1;
+  if (!(G > 0.0f) || isinf(G)) return -1;
+  orc_scalars s;
+  if (orc_scalars_for_step(hp, t, &s) != 0) return -1;
+  for (int64_t b0 = 0; b0 < n; b0 += ORC_FP4_BLOCK) {
+    const int64_t bn = (n - b0 < ORC_FP4_BLOCK) ? n - b0 : ORC_FP4_BLOCK;
+    const int64_t blk = b0 / ORC_FP4_BLOCK;
+    const float d_old = orc_e4m3_decode(bscale[blk]) * G;
+    float wn[ORC_FP4_BLOCK];
+    float amax = 0.0f;
+    for (int64_t j = 0; j < bn; ++j) {
+      const int64_t k = b0 + j;
+      float wk = orc_e2m1_decode(nvfp4_get(q, k)) * d_old;
+      float gk = load_elem(g, k, gdt), mk = load_elem(m, k, mdt), vk = load_elem(v, k, mdt);
+      float vek = load_elem(ve, k, mdt);
+      float m1, v1, ve1;
+      orc_update_element(&s, wk, gk, mk, vk, vek, &wn[j], &m1, &v1, &ve1);
+      if (isfinite(wn[j]) && fabsf(wn[j]) > amax) amax = fabsf(wn[j]);
+      store_moment(m, k, mdt, m1);
+      store_moment(v, k, mdt, v1);
+      store_moment(ve, k, mdt, ve1);
+    }
+    /* current scaling: the block's new scale covers its largest updated |w| */
+    const int32_t c_new = orc_nvfp4_scale_code(amax, G, bscale[blk]);
+    bscale[blk] = (uint8_t)c_new;
+    const float d_new = orc_e4m3_decode((uint8_t)c_new) * G;
+    for (int64_t j = 0; j < bn; ++j) {
+      const int64_t k = b0 + j;
+      const float x = wn[j] / d_new;
+      const uint8_t c = hp->stochastic
+          ? orc_e2m1_sr(x, orc_rng_lane(hp->seed, (uint64_t)t, (uint64_t)(gidx0 + k), ORC_E4M3))
+          : orc_e2m1_rne(x);
+      nvfp4_put(q, k, c);
+    }
+  }
+  return 0;
+}
+
+void orc_dequant_nvfp4_bf16(int64_t n, const uint8_t* q, const uint8_t* bscale, float G, uint16_t* out) {
+  for (int64_t k = 0; k < n; ++k) {
+    const float d = orc_e4m3_decode(bscale[k / ORC_FP4_BLOCK]) * G;
+    out[k] = orc_bf16_rne(orc_e2m1_decode(nvfp4_get(q, k)) * d);
+  }
+}
+
+/* ------------------------------------------------------------------------ */
 /* Array helpers for the tests: plain loops over the scalar functions above. */
 /* ------------------------------------------------------------------------ */
 void orc_bf16_rne_n(int64_t n, const float* x, uint16_t* out) {

@@ -24,9 +24,11 @@ extern "C" {
 #endif
 
 /* Element formats.  ORC_E4M3_B32: E4M3 codes with one power-of-two scale
- * per 32 consecutive elements, stored as FP16 bits. */
-enum { ORC_F32 = 0, ORC_BF16 = 1, ORC_E4M3 = 2, ORC_E4M3_B32 = 3 };
-enum { ORC_BLOCK = 32 };
+ * per 32 consecutive elements, stored as FP16 bits.  ORC_NVFP4: E2M1 codes
+ * (two per byte, the even element in the low nibble) with one E4M3 scale per
+ * 16 consecutive elements and one binary32 scale per tensor. */
+enum { ORC_F32 = 0, ORC_BF16 = 1, ORC_E4M3 = 2, ORC_E4M3_B32 = 3, ORC_NVFP4 = 4 };
+enum { ORC_BLOCK = 32, ORC_FP4_BLOCK = 16 };
 
 /* Hyper-parameters (Algorithm 1 inputs; Algorithm 2 optional clips). */
 typedef struct {
@@ -117,6 +119,32 @@ int32_t orc_step_block_e4m3(int64_t n, int64_t gidx0, int32_t gdt, int32_t mdt,
 /* BF16 compute copy of stored E4M3 weights: bf16(decode(q) * scale), exact.
  * Per-tensor scale 2^e (bscale NULL) or per-32-block FP16 scales. */
 void orc_dequant_bf16(int64_t n, const uint8_t* q, int32_t e, const uint16_t* bscale, uint16_t* out);
+
+/* E2M1 (OCP FP4: sign, 2 exponent bits with bias 1, 1 mantissa bit; values
+ * +-{0, 0.5, 1, 1.5, 2, 3, 4, 6}, no infinity or NaN) codes in the low 4
+ * bits.  Nearest-even or stochastic (away from zero iff r32 < floor(fraction
+ * * 2^32)); |x| >= 6 and infinities saturate to +-6; NaN gives +0. */
+uint8_t orc_e2m1_rne(float x);
+uint8_t orc_e2m1_sr(float x, uint32_t r32);
+float   orc_e2m1_decode(uint8_t c);
+
+/* NVFP4 block scale: the smallest E4M3 code c in [1, 126] whose block range
+ * covers amax, i.e. 6 * (value(c) * G) >= amax with both products rounded to
+ * binary32; 126 when none does; c_old when amax is 0. */
+int32_t orc_nvfp4_scale_code(float amax, float G, int32_t c_old);
+
+/* One optimizer step over a whole NVFP4 tensor (current block scaling).
+ * q: ceil(n/2) bytes of codes, bscale: ceil(n/16) E4M3 scale codes (both
+ * updated in place), G the tensor scale (> 0, finite).  Element j decodes as
+ * q_j * d_b with d_b = value(bscale[b]) * G (rounded to binary32), and
+ * re-encodes x_j = w'_j / d_b' (rounded to binary32) with the block's new
+ * scale.  Element j has global index gidx0 + j (32-bit random lanes, as for
+ * E4M3).  Returns 0 or -1. */
+int32_t orc_step_nvfp4(int64_t n, int64_t gidx0, int32_t gdt, int32_t mdt, uint8_t* q, uint8_t* bscale,
+                       float G, const void* g, void* m, void* v, void* ve, const orc_hparams* hp, int64_t t);
+
+/* BF16 compute copy of NVFP4 weights: bf16(q_j * d_b) with d_b as above. */
+void orc_dequant_nvfp4_bf16(int64_t n, const uint8_t* q, const uint8_t* bscale, float G, uint16_t* out);
 
 /* Array forms of the scalar functions (plain loops), for the tests. */
 void orc_bf16_rne_n(int64_t n, const float* x, uint16_t* out);
