@@ -37,19 +37,22 @@ sys.path.insert(0, str(ROOT))
 
 METRIC = "fused M+Adam step Gparams/s and HBM GB/s as % of GB300 peak (1 GPU)"
 UNIT = "Gparams/s"
-BYTES = {"f32": 4, "bf16": 2, "e4m3": 1, "e4m3_b32": 1}
+BYTES = {"f32": 4, "bf16": 2, "e4m3": 1, "e4m3_b32": 1, "nvfp4": 0.5}
 
 
 def algorithmic_bytes(wl) -> float:
     """Reads + writes of one step over the list: per element w (r+w), g (r),
     mu, nu, nu_e (r+w); per 32-element block of block-scaled E4M3 its FP16
-    scale (r+w); per element of a BF16 compute copy 2 bytes (w)."""
+    scale (r+w); per 16-element block of NVFP4 its E4M3 scale (r+w); per
+    element of a BF16 compute copy 2 bytes (w)."""
     total = 0
     for spec, fmt in zip(wl.specs, wl.formats):
         n = spec.numel
         total += n * (2 * BYTES[fmt] + BYTES[wl.grad_dtype] + 6 * BYTES[wl.moment_dtype])
         if fmt == "e4m3_b32":
             total += 4 * ((n + 31) // 32)
+        if fmt == "nvfp4":
+            total += 2 * ((n + 15) // 16)
         if wl.compute_copy and fmt != "bf16":
             total += 2 * n
     return float(total)
@@ -165,6 +168,8 @@ def host_lists(mt):
     for k, b in enumerate(mt.bscale or []):
         if b is not None:
             tensors[k]["bscale"] = W.to_numpy_bits(b)
+        if mt.gscale and mt.gscale[k]:
+            tensors[k]["gscale"] = float(mt.gscale[k])
     fp8 = None
     if mt.fp8_exp is not None:
         fp8 = [oracle.fp8_init([tensors[k]], [mt.fp8_exp[k]])[0] if f == "e4m3" else None
@@ -189,7 +194,10 @@ def time_oracle(wl, target_s: float, t_step: int = 1):
         oracle.step(tensors, **kw)
         for k, x in enumerate(mt.cc or []):  # the compute copy the step also writes
             if x is not None:
-                if "bscale" in tensors[k]:
+                if "gscale" in tensors[k]:
+                    oracle.dequant_nvfp4_bf16(tensors[k]["g"].size, tensors[k]["w"], tensors[k]["bscale"],
+                                              tensors[k]["gscale"])
+                elif "bscale" in tensors[k]:
                     oracle.dequant_bf16(tensors[k]["w"], bscale=tensors[k]["bscale"])
                 else:
                     oracle.dequant_bf16(tensors[k]["w"], e=fp8[k][0])
@@ -216,7 +224,7 @@ def run_gpu(wl, steps: int, warmup: int, rank: int, e2e_steps: int):
     opt = MPAdam(mt.w, mt.m, mt.v, mt.ve, weight_dtype=mt.formats if extended else wl.weight_dtype,
                  grad_dtype=wl.grad_dtype, moment_dtype=wl.moment_dtype, rounding=wl.rounding,
                  seed=wl.seed + rank, fp8_exp=mt.fp8_exp, block_scales=mt.bscale if extended else None,
-                 compute=mt.cc if extended else None)
+                 compute=mt.cc if extended else None, global_scales=mt.gscale if extended else None)
     launches_per_step = len(set(mt.formats))
     stream = torch.cuda.current_stream(dev)
     gptrs = [g.data_ptr() for g in mt.g]
@@ -351,11 +359,13 @@ def main():
     ap.add_argument("--steps", type=int, default=50)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--config", default="llama_7b")
-    ap.add_argument("--secondary", default="llama_1p5b,llama_1p5b_mixed,gpt2_124m,ragged_20k",
+    ap.add_argument("--secondary", default="llama_1p5b,llama_1p5b_mixed,llama_1p5b_nvfp4,gpt2_124m,ragged_20k",
                     help="'' to skip")
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--e2e-steps", type=int, default=5)
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    ap.add_argument("--rounding", default=None, choices=["nearest", "stochastic"],
+                    help="override the workload's weight rounding")
     ap.add_argument("--max-params", type=int, default=0,
                     help="truncate the list to its first N params (small profiling cases)")
     args = ap.parse_args()
@@ -363,6 +373,8 @@ def main():
 
     import workloads as W
     wl = W.CONFIGS[args.config]
+    if args.rounding:
+        wl = W.replace(wl, rounding=args.rounding)
     if args.max_params:
         wl, got = oracle_sample(wl, args.max_params)
         wl = W.replace(wl, name=f"{wl.name}[:{got}]")

@@ -95,8 +95,12 @@ typedef enum {
 } mpadam_status;
 
 /* MPADAM_E4M3_B32: E4M3 codes with one FP16 power-of-two scale per 32
- * consecutive elements (block scaling; weights only, mpadam_create_ex). */
-typedef enum { MPADAM_F32 = 0, MPADAM_BF16 = 1, MPADAM_E4M3 = 2, MPADAM_E4M3_B32 = 3 } mpadam_dtype;
+ * consecutive elements.  MPADAM_NVFP4: E2M1 codes (OCP FP4), two per byte,
+ * with one E4M3 scale per 16 consecutive elements and one binary32 scale per
+ * tensor.  Both are block-scaled weight formats (mpadam_create_ex). */
+typedef enum {
+  MPADAM_F32 = 0, MPADAM_BF16 = 1, MPADAM_E4M3 = 2, MPADAM_E4M3_B32 = 3, MPADAM_NVFP4 = 4
+} mpadam_dtype;
 typedef enum { MPADAM_ROUND_NEAREST = 0, MPADAM_ROUND_STOCHASTIC = 1 } mpadam_rounding;
 
 /* One parameter tensor (Algorithm 1's state per parameter: w, mu, nu, nu_e),
@@ -146,9 +150,10 @@ typedef struct mpadam_state mpadam_state;
  * FP16 block scales, BF16 embeddings, norms and head).  w, m, v, ve, numel
  * as in mpadam_tensor (m, v, ve of the config's moment_dtype).
  *   weight_dtype: MPADAM_BF16, MPADAM_E4M3 (per-tensor scale, delayed, held
- *     in the fp8 rings as described above) or MPADAM_E4M3_B32;
- *   block_scale: E4M3_B32 only (else NULL): device array of ceil(numel/32)
- *     FP16 bit patterns, the scale of elements [32b, 32b + 32) at index b,
+ *     in the fp8 rings as described above), MPADAM_E4M3_B32 or MPADAM_NVFP4;
+ *   block_scale: E4M3_B32 and NVFP4 only (else NULL).  For E4M3_B32, a
+ *     device array of ceil(numel/32) FP16 bit patterns, the scale of
+ *     elements [32b, 32b + 32) at index b,
  *     2-byte aligned (16-byte aligned for the staged fast path).  Stored
  *     weights decode as code * scale.  A step rewrites every block's scale
  *     with 2^k, k the smallest integer with A <= 448 * 2^k (A = the block's
@@ -157,14 +162,27 @@ typedef struct mpadam_state mpadam_state;
  *     keeps the exponent of its old scale.  The new codes encode w' * 2^-k
  *     (nearest-even or stochastic, saturating at +-448, as for E4M3).
  *     Scales should be powers of two; another FP16 value decodes as itself
- *     and counts as the power of two at or below it;
- *   compute: optional (NULL = none; E4M3 formats only): device array of
- *     numel BF16 values, 2-byte aligned (16-byte for the vector path),
- *     overwritten every step with the dequantised updated weights
- *     bf16(code * scale) -- exact, since every E4M3 value times a scale is a
- *     BF16 number -- from the same kernel pass that writes the codes
- *     (Sec. 5.2's low-precision master weights feed a BF16 forward pass).
- *   reserved: must be 0. */
+ *     and counts as the power of two at or below it.  For NVFP4, a device
+ *     array of ceil(numel/16) E4M3 codes, the scale s of elements
+ *     [16b, 16b + 16) at index b (16-byte aligned for the staged fast path);
+ *     w holds ceil(numel/2) bytes, element 2i in the low nibble of byte i
+ *     (the spare high nibble of an odd-length tensor is written 0).  A
+ *     weight decodes as q * d with d = s * G (G = global_scale; both
+ *     products rounded to binary32).  A step rewrites every block's scale
+ *     with the smallest E4M3 code c in [1, 126] such that 6 * (value(c) * G)
+ *     (products rounded) >= A, the block's largest finite |w'| (126 when
+ *     none; kept when A = 0), and the codes with E2M1(w' / d') (quotient
+ *     rounded to binary32; nearest-even, or stochastic: away from zero iff
+ *     R32 < floor(fraction * 2^32), with the E4M3 random lanes; |x| >= 6
+ *     saturates, NaN stores +0);
+ *   compute: optional (NULL = none; E4M3, E4M3_B32 and NVFP4 only): device
+ *     array of numel BF16 values, 2-byte aligned (16-byte for the vector
+ *     path), overwritten every step with the dequantised updated weights
+ *     bf16(decoded weight) from the same kernel pass that writes the codes
+ *     (Sec. 5.2's low-precision master weights feed a BF16 forward pass);
+ *     for the E4M3 formats this is exact (code * scale is a BF16 number);
+ *   global_scale: NVFP4 only, the tensor's binary32 scale G (finite, > 0),
+ *     held fixed by the step; 0 for every other format. */
 typedef struct {
   void* w;
   void* m;
@@ -172,8 +190,8 @@ typedef struct {
   void* ve;
   int64_t numel;
   int32_t weight_dtype;
-  int32_t reserved;
-  uint16_t* block_scale;
+  float global_scale;
+  void* block_scale;
   uint16_t* compute;
 } mpadam_tensor_ex;
 
@@ -189,7 +207,7 @@ int32_t mpadam_create(const mpadam_tensor* tensors, int32_t n, const mpadam_conf
 /* The same for a list whose tensors each name their weight format (and
  * carry block scales and compute copies, see mpadam_tensor_ex); cfg's
  * weight_dtype is not used.  The tensors are stepped by one kernel launch
- * per format present, in the order BF16, E4M3, E4M3_B32, all on the stream
+ * per format present, in the order BF16, E4M3, E4M3_B32, NVFP4, all on the stream
  * given to mpadam_step; global element indices (stochastic rounding) are
  * those of the whole list, and the fp8 rings (required when any tensor is
  * E4M3, else may be NULL) are indexed by list position k over all n
@@ -220,9 +238,10 @@ int32_t mpadam_step(mpadam_state* s, const void* const* grads, int64_t step,
 /* The same step with gradients and weights in host memory: copies
  * host_grads[k] (numel[k] gradients each) to library-owned device staging,
  * runs the step, and copies every updated weight tensor back to
- * host_w_out[k] (numel[k] weights of its weight format each; block scales
- * and compute copies stay in device memory).  The host buffers should be
- * pinned.  When the list has one weight format and host_grads, host_w_out
+ * host_w_out[k] (numel[k] weights of its weight format each, NVFP4 packed
+ * two per byte; block scales and compute copies stay in device memory).  The host buffers should be
+ * pinned.  When the list has one weight format other than NVFP4 and
+ * host_grads, host_w_out
  * and the device weights each follow the global-index layout of one flat
  * allocation (pointer k = base + off[k] * element size), the step is
  * pipelined in up to 8 chunks of whole
@@ -265,7 +284,7 @@ int32_t mpadam_device_status(mpadam_state* s, int32_t* code);
 /* Diagnostics: the random bits the step draws.  Writes into out (device,
  * uint32[n]) the lane of global element indices first, ..., first + n - 1 at
  * step `step` for weight storage `weight_dtype` (16-bit lanes for BF16,
- * 32-bit for both E4M3 formats), on `stream`.  Errors: EINVAL, ECUDA. */
+ * 32-bit for the E4M3 formats and NVFP4), on `stream`.  Errors: EINVAL, ECUDA. */
 int32_t mpadam_rng_lanes(uint64_t seed, int64_t step, int32_t weight_dtype, int64_t first,
                          int64_t n, uint32_t* out, struct CUstream_st* stream);
 

@@ -333,11 +333,11 @@ def step(tensors, *, wdt, gdt: int, mdt: int, hp: HParams, t: int,
     For E4M3_B32 storage the dict also holds "bscale" (FP16 block scales,
     updated in place); for NVFP4 storage "w" holds packed codes, "bscale" the
     E4M3 block-scale codes (updated in place) and "gscale" the tensor scale."""
-    offs = global_offsets([d["w"].size for d in tensors])
+    offs = global_offsets([d["g"].size for d in tensors])   # element counts (NVFP4 "w" is packed)
     formats = list(wdt) if isinstance(wdt, (list, tuple)) else [wdt] * len(tensors)
     for k, d in enumerate(tensors):
         wdt = formats[k]
-        if d["w"].size == 0:
+        if d["g"].size == 0:
             continue
         if wdt == E4M3_B32:
             step_block_e4m3(hp, t, gdt, mdt, d["w"], d["bscale"], d["g"], d["m"], d["v"], d["ve"],

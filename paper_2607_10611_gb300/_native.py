@@ -14,9 +14,10 @@ from typing import Optional, Sequence
 from . import builder as _build
 
 MPADAM_OK, MPADAM_EINVAL, MPADAM_EALLOC, MPADAM_ECUDA, MPADAM_EUNSUPPORTED = 0, 1, 2, 3, 4
-MPADAM_F32, MPADAM_BF16, MPADAM_E4M3, MPADAM_E4M3_B32 = 0, 1, 2, 3
+MPADAM_F32, MPADAM_BF16, MPADAM_E4M3, MPADAM_E4M3_B32, MPADAM_NVFP4 = 0, 1, 2, 3, 4
 MPADAM_ROUND_NEAREST, MPADAM_ROUND_STOCHASTIC = 0, 1
-DTYPE = {"f32": MPADAM_F32, "bf16": MPADAM_BF16, "e4m3": MPADAM_E4M3, "e4m3_b32": MPADAM_E4M3_B32}
+DTYPE = {"f32": MPADAM_F32, "bf16": MPADAM_BF16, "e4m3": MPADAM_E4M3, "e4m3_b32": MPADAM_E4M3_B32,
+         "nvfp4": MPADAM_NVFP4}
 ROUNDING = {"nearest": MPADAM_ROUND_NEAREST, "stochastic": MPADAM_ROUND_STOCHASTIC}
 
 EXPORTED = ["mpadam_create", "mpadam_create_ex", "mpadam_fp8_init", "mpadam_step", "mpadam_step_host",
@@ -38,7 +39,7 @@ class mpadam_tensor(ctypes.Structure):
 class mpadam_tensor_ex(ctypes.Structure):
     _fields_ = [("w", ctypes.c_void_p), ("m", ctypes.c_void_p), ("v", ctypes.c_void_p),
                 ("ve", ctypes.c_void_p), ("numel", ctypes.c_int64), ("weight_dtype", ctypes.c_int32),
-                ("reserved", ctypes.c_int32), ("block_scale", ctypes.c_void_p), ("compute", ctypes.c_void_p)]
+                ("global_scale", ctypes.c_float), ("block_scale", ctypes.c_void_p), ("compute", ctypes.c_void_p)]
 
 
 class mpadam_config(ctypes.Structure):
@@ -140,11 +141,14 @@ def mpadam_create(tensors: Sequence[tuple], cfg: mpadam_config, fp8_exp: int = 0
 
 
 def mpadam_create_ex(tensors: Sequence[tuple], cfg: mpadam_config, fp8_exp: int = 0, fp8_amax: int = 0) -> int:
-    """tensors: (w, m, v, ve, numel, weight_dtype, block_scale, compute) per tensor,
-    pointers as ints (0 = NULL), weight_dtype an MPADAM_* value or its name."""
+    """tensors: (w, m, v, ve, numel, weight_dtype, block_scale, compute[, global_scale]) per
+    tensor, pointers as ints (0 = NULL), weight_dtype an MPADAM_* value or its name,
+    global_scale the NVFP4 tensor scale (0 for other formats)."""
     arr = (mpadam_tensor_ex * max(1, len(tensors)))()
-    for i, (w, m, v, ve, n, wd, bs, cc) in enumerate(tensors):
-        arr[i] = mpadam_tensor_ex(w, m, v, ve, n, DTYPE[wd] if isinstance(wd, str) else wd, 0, bs or None,
+    for i, t in enumerate(tensors):
+        w, m, v, ve, n, wd, bs, cc = t[:8]
+        gs = float(t[8]) if len(t) > 8 else 0.0
+        arr[i] = mpadam_tensor_ex(w, m, v, ve, n, DTYPE[wd] if isinstance(wd, str) else wd, gs, bs or None,
                                   cc or None)
     out = ctypes.c_void_p()
     _check(lib().mpadam_create_ex(arr, len(tensors), ctypes.byref(cfg), fp8_exp or None, fp8_amax or None,

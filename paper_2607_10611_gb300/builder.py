@@ -18,7 +18,7 @@ INCLUDE = ROOT / "include"
 OUT_DIR = PKG / "_build"
 LIB = OUT_DIR / "libmpadam.so"
 
-SOURCES = ["mpadam_api.cu", "step_bf16.cu", "step_e4m3.cu", "step_e4m3b.cu"]
+SOURCES = ["mpadam_api.cu", "step_bf16.cu", "step_e4m3.cu", "step_e4m3b.cu", "step_nvfp4.cu"]
 HEADERS = ["step_args.h", "step_kernel.cuh"]
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]

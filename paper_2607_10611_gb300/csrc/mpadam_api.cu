@@ -43,6 +43,11 @@ int32_t cuda_fail(cudaError_t e, const char* what) {
 
 size_t elem_size(int32_t dt) { return dt == MPADAM_F32 ? 4 : (dt == MPADAM_BF16 ? 2 : 1); }
 
+// Bytes of n stored weights (NVFP4: two per byte).
+size_t weight_bytes(int32_t wd, int64_t n) {
+  return wd == MPADAM_NVFP4 ? (size_t)((n + 1) / 2) : (size_t)n * elem_size(wd);
+}
+
 bool is_aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
 // Per-step binary32 scalars of the canonical update, from binary64.
@@ -109,8 +114,8 @@ bool kernel_options(const mpadam_config& c) {
 // (mpadam_create_ex) and cfg->weight_dtype is not used.
 int32_t check_config(const mpadam_config* c, bool per_tensor_weights = false) {
   if (!c) return fail(MPADAM_EINVAL, "config is NULL");
-  if (!per_tensor_weights && c->weight_dtype == MPADAM_E4M3_B32)
-    return fail(MPADAM_EINVAL, "block-scaled E4M3 weights need their scale arrays: use mpadam_create_ex");
+  if (!per_tensor_weights && (c->weight_dtype == MPADAM_E4M3_B32 || c->weight_dtype == MPADAM_NVFP4))
+    return fail(MPADAM_EINVAL, "block-scaled weights need their scale arrays: use mpadam_create_ex");
   if (!per_tensor_weights && c->weight_dtype != MPADAM_BF16 && c->weight_dtype != MPADAM_E4M3)
     return fail(MPADAM_EINVAL, "weight_dtype must be MPADAM_BF16 or MPADAM_E4M3 (got %d)", c->weight_dtype);
   if (c->grad_dtype != MPADAM_F32 && c->grad_dtype != MPADAM_BF16)
@@ -140,10 +145,12 @@ int32_t check_config(const mpadam_config* c, bool per_tensor_weights = false) {
 }
 
 int32_t make_geometry(const mpadam_config& c, int32_t wd, int dev, Geometry* g) {
-  const int32_t rw = mpadam::kTile * (int32_t)elem_size(wd);
+  const int32_t rw = (int32_t)weight_bytes(wd, mpadam::kTile);
   const int32_t rg = mpadam::kTile * (int32_t)elem_size(c.grad_dtype);
   const int32_t rm = mpadam::kTile * (int32_t)elem_size(c.moment_dtype);
-  const int32_t rs = wd == MPADAM_E4M3_B32 ? mpadam::kTileBlocks * 2 : 0;  // 240 bytes, a 16-byte multiple
+  const int32_t rs = wd == MPADAM_E4M3_B32 ? mpadam::kTileBlocks * 2           // 240 bytes, a 16-byte multiple
+                   : wd == MPADAM_NVFP4    ? mpadam::kTileFp4Blocks               // 240 bytes
+                                           : 0;
   g->off_g = rw;
   g->off_m = rw + rg;
   g->off_v = g->off_m + rm;
@@ -397,6 +404,7 @@ const void* select_kernel(const mpadam_config& c, int32_t wd) {
   if (wd == MPADAM_BF16) return mpadam::step_kernel_bf16(c.grad_dtype, c.moment_dtype, c.rounding, opt);
   if (wd == MPADAM_E4M3) return mpadam::step_kernel_e4m3(c.grad_dtype, c.moment_dtype, c.rounding, opt);
   if (wd == MPADAM_E4M3_B32) return mpadam::step_kernel_e4m3b(c.grad_dtype, c.moment_dtype, c.rounding, opt);
+  if (wd == MPADAM_NVFP4) return mpadam::step_kernel_nvfp4(c.grad_dtype, c.moment_dtype, c.rounding, opt);
   return nullptr;
 }
 
@@ -426,8 +434,9 @@ struct TensorIn {
   void *w, *m, *v, *ve;
   int64_t numel;
   int32_t wd;
-  uint16_t* scale;
+  void* scale;
   uint16_t* compute;
+  float gscale;
 };
 
 // Validate a tensor list, lay out its global index and format groups, and
@@ -441,8 +450,12 @@ int32_t create_state(const std::vector<TensorIn>& t, const mpadam_config* cfg, i
   int64_t off = 0;
   for (int32_t k = 0; k < n; ++k) {
     const TensorIn& x = t[k];
-    if (x.wd != MPADAM_BF16 && x.wd != MPADAM_E4M3 && x.wd != MPADAM_E4M3_B32)
-      return fail(MPADAM_EINVAL, "tensor %d: weight_dtype must be BF16, E4M3 or E4M3_B32 (got %d)", k, x.wd);
+    if (x.wd != MPADAM_BF16 && x.wd != MPADAM_E4M3 && x.wd != MPADAM_E4M3_B32 && x.wd != MPADAM_NVFP4)
+      return fail(MPADAM_EINVAL, "tensor %d: weight_dtype must be BF16, E4M3, E4M3_B32 or NVFP4 (got %d)", k, x.wd);
+    if (x.wd == MPADAM_NVFP4 && !(std::isfinite(x.gscale) && x.gscale > 0.0f))
+      return fail(MPADAM_EINVAL, "tensor %d: NVFP4 weights need a finite global_scale > 0", k);
+    if (x.wd != MPADAM_NVFP4 && x.gscale != 0.0f)
+      return fail(MPADAM_EINVAL, "tensor %d: global_scale is only for NVFP4 weights (must be 0)", k);
     if (x.numel < 0) return fail(MPADAM_EINVAL, "tensor %d: numel < 0", k);
     any_e4m3 = any_e4m3 || x.wd == MPADAM_E4M3;
     if (x.numel > 0) {
@@ -452,11 +465,13 @@ int32_t create_state(const std::vector<TensorIn>& t, const mpadam_config* cfg, i
         return fail(MPADAM_EINVAL, "tensor %d: pointer not aligned to its element size", k);
       if (x.wd == MPADAM_E4M3_B32 && (!x.scale || !is_aligned(x.scale, 2)))
         return fail(MPADAM_EINVAL, "tensor %d: block-scaled weights need a 2-byte aligned block_scale array", k);
+      if (x.wd == MPADAM_NVFP4 && !x.scale)
+        return fail(MPADAM_EINVAL, "tensor %d: NVFP4 weights need their block_scale array", k);
       if (x.compute && !is_aligned(x.compute, 2))
         return fail(MPADAM_EINVAL, "tensor %d: compute copy not 2-byte aligned", k);
     }
-    if (x.wd != MPADAM_E4M3_B32 && x.scale)
-      return fail(MPADAM_EINVAL, "tensor %d: block_scale is only for E4M3_B32 weights", k);
+    if (x.wd != MPADAM_E4M3_B32 && x.wd != MPADAM_NVFP4 && x.scale)
+      return fail(MPADAM_EINVAL, "tensor %d: block_scale is only for E4M3_B32 and NVFP4 weights", k);
     if (x.wd == MPADAM_BF16 && x.compute)
       return fail(MPADAM_EINVAL, "tensor %d: BF16 weights are their own compute copy (compute must be NULL)", k);
     if (x.numel > (int64_t(1) << 56) || off > (int64_t(1) << 58))
@@ -492,11 +507,11 @@ int32_t create_state(const std::vector<TensorIn>& t, const mpadam_config* cfg, i
     s->fp8_exp = fp8_exp;
     s->fp8_amax = fp8_amax;
 
-    // format groups, in the fixed order BF16, E4M3, E4M3_B32
+    // format groups, in the fixed order BF16, E4M3, E4M3_B32, NVFP4
     std::vector<TensorDesc> desc;
     std::vector<TensorAux> aux;
     bool any_aux = false;
-    for (int32_t wd : {MPADAM_BF16, MPADAM_E4M3, MPADAM_E4M3_B32}) {
+    for (int32_t wd : {MPADAM_BF16, MPADAM_E4M3, MPADAM_E4M3_B32, MPADAM_NVFP4}) {
       Group g;
       g.wd = wd;
       g.first = (int32_t)s->order.size();
@@ -504,7 +519,7 @@ int32_t create_state(const std::vector<TensorIn>& t, const mpadam_config* cfg, i
         if (t[k].wd != wd) continue;
         s->tile_off[k] = g.tiles;
         desc.push_back(TensorDesc{t[k].w, t[k].m, t[k].v, t[k].ve, t[k].numel, s->goff[k], g.tiles, k, 0});
-        aux.push_back(TensorAux{t[k].scale, t[k].compute});
+        aux.push_back(TensorAux{t[k].scale, t[k].compute, t[k].gscale, 0});
         g.aux = g.aux || t[k].scale != nullptr || t[k].compute != nullptr;
         g.numel.push_back(t[k].numel);
         g.tiles += tiles_of(t[k].numel);
@@ -668,7 +683,7 @@ int32_t mpadam_create(const mpadam_tensor* tensors, int32_t n, const mpadam_conf
     std::vector<TensorIn> t(n);
     for (int32_t k = 0; k < n; ++k)
       t[k] = TensorIn{tensors[k].w, tensors[k].m, tensors[k].v, tensors[k].ve, tensors[k].numel, cfg->weight_dtype,
-                      nullptr, nullptr};
+                      nullptr, nullptr, 0.0f};
     return create_state(t, cfg, cfg->weight_dtype, fp8_exp, fp8_amax, out);
   } catch (const std::bad_alloc&) {
     return fail(MPADAM_EALLOC, "host allocation failed");
@@ -687,8 +702,7 @@ int32_t mpadam_create_ex(const mpadam_tensor_ex* tensors, int32_t n, const mpada
     std::vector<TensorIn> t(n);
     for (int32_t k = 0; k < n; ++k) {
       const mpadam_tensor_ex& x = tensors[k];
-      if (x.reserved != 0) return fail(MPADAM_EINVAL, "tensor %d: reserved must be 0", k);
-      t[k] = TensorIn{x.w, x.m, x.v, x.ve, x.numel, x.weight_dtype, x.block_scale, x.compute};
+      t[k] = TensorIn{x.w, x.m, x.v, x.ve, x.numel, x.weight_dtype, x.block_scale, x.compute, x.global_scale};
     }
     return create_state(t, cfg, MPADAM_BF16, fp8_exp, fp8_amax, out);
   } catch (const std::bad_alloc&) {
@@ -812,8 +826,9 @@ int32_t mpadam_fp8_init(mpadam_state* s, const int32_t* init_exp, int64_t first_
 int32_t mpadam_rng_lanes(uint64_t seed, int64_t step, int32_t weight_dtype, int64_t first, int64_t n,
                          uint32_t* out, cudaStream_t stream) {
   if (step < 0) return fail(MPADAM_EINVAL, "step must be >= 0");
-  if (weight_dtype != MPADAM_BF16 && weight_dtype != MPADAM_E4M3 && weight_dtype != MPADAM_E4M3_B32)
-    return fail(MPADAM_EINVAL, "weight_dtype must be MPADAM_BF16, MPADAM_E4M3 or MPADAM_E4M3_B32");
+  if (weight_dtype != MPADAM_BF16 && weight_dtype != MPADAM_E4M3 && weight_dtype != MPADAM_E4M3_B32 &&
+      weight_dtype != MPADAM_NVFP4)
+    return fail(MPADAM_EINVAL, "weight_dtype must be MPADAM_BF16, MPADAM_E4M3, MPADAM_E4M3_B32 or MPADAM_NVFP4");
   if (first < 0 || n < 0) return fail(MPADAM_EINVAL, "first and n must be >= 0");
   if (n == 0) return MPADAM_OK;
   if (!out || !is_aligned(out, 4)) return fail(MPADAM_EINVAL, "out is NULL or misaligned");
@@ -872,7 +887,7 @@ int32_t mpadam_step_host(mpadam_state* s, const void* const* host_grads, void* c
   if (first > last) return MPADAM_OK;
   const size_t lo_e = (size_t)s->goff[first], hi_e = (size_t)(s->goff[last] + s->numel[last]);
   // one weight format for the whole list?  (then wsz is its element size)
-  const bool single = s->groups.size() == 1;
+  const bool single = s->groups.size() == 1 && s->groups[0].wd != MPADAM_NVFP4;
   const size_t wsz = elem_size(s->groups[0].wd);
 
   const char* hb = nullptr;
@@ -939,7 +954,7 @@ int32_t mpadam_step_host(mpadam_state* s, const void* const* host_grads, void* c
   } else {
     for (int32_t k = 0; k < s->n; ++k) {
       if (s->numel[k] == 0) continue;
-      e = cudaMemcpyAsync(host_w_out[k], s->w[k], (size_t)s->numel[k] * elem_size(s->wdt[k]), cudaMemcpyDeviceToHost,
+      e = cudaMemcpyAsync(host_w_out[k], s->w[k], weight_bytes(s->wdt[k], s->numel[k]), cudaMemcpyDeviceToHost,
                           stream);
       if (e != cudaSuccess) return cuda_fail(e, "weight download");
     }

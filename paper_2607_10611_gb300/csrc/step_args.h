@@ -37,9 +37,14 @@ constexpr int kPhiloxRounds = 10;
 constexpr int kBlock = 32;                          // elements per block scale (block-scaled E4M3)
 constexpr int kTileBlocks = kTile / kBlock;         // 120 block scales per tile (240 bytes)
 static_assert(kTile % kBlock == 0 && kBlock == 4 * kGroup, "a block is one quad of consumer threads");
+constexpr int kFp4Block = 16;                       // elements per NVFP4 block scale
+constexpr int kTileFp4Blocks = kTile / kFp4Block;   // 240 E4M3 block scales per tile (240 bytes)
+static_assert(kTile % kFp4Block == 0 && kFp4Block == 2 * kGroup, "an NVFP4 block is a pair of consumer threads");
 
 // kE4M3B: E4M3 codes with FP16 block scales (one per kBlock elements).
-enum Dtype : int { kF32 = 0, kBF16 = 1, kE4M3 = 2, kE4M3B = 3 };
+// kNVFP4: E2M1 codes, two per byte (even element in the low nibble), with an
+// E4M3 scale per kFp4Block elements and a binary32 scale per tensor.
+enum Dtype : int { kF32 = 0, kBF16 = 1, kE4M3 = 2, kE4M3B = 3, kNVFP4 = 4 };
 
 // Error bits a step kernel may set in *err (bounded waits that gave up).
 enum DeviceError : int32_t { kErrFullWait = 1, kErrEmptyWait = 2, kErrDrainWait = 4 };
@@ -62,8 +67,11 @@ static_assert(sizeof(TensorDesc) == 64, "TensorDesc must stay 64 bytes");
 // Per-tensor extras of the E4M3 formats; one entry per descriptor, or no
 // table at all when no tensor of the launch has any.
 struct TensorAux {
-  uint16_t* scale;    // kE4M3B: ceil(numel / kBlock) FP16 block scales, updated in place
+  void* scale;        // kE4M3B: ceil(numel / kBlock) FP16 block scales; kNVFP4: ceil(numel / kFp4Block)
+                      // E4M3 block scales; updated in place
   uint16_t* compute;  // BF16 copy of the updated stored weights (dequantised), or nullptr
+  float gscale;       // kNVFP4: the tensor's binary32 scale
+  int32_t pad;
 };
 
 // Per-step binary32 scalars of the canonical update (computed on the host in
@@ -94,7 +102,7 @@ struct StepArgs {
   int32_t stages;            // shared-memory pipeline depth (2..kMaxStages)
   int32_t stage_bytes;       // bytes of one stage: w | g | m | v | ve | block-scale regions
   int32_t off_g, off_m, off_v, off_ve;  // region offsets inside a stage (w at 0)
-  int32_t off_s;             // block scales (kE4M3B only)
+  int32_t off_s;             // block scales (kE4M3B, kNVFP4)
   StepScalars s;
   uint32_t rk0[kPhiloxRounds], rk1[kPhiloxRounds];  // Philox round keys: seed + r * Weyl
   uint32_t t_lo, t_hi;       // step number (Philox counter words 2, 3)
@@ -113,5 +121,6 @@ struct StepArgs {
 const void* step_kernel_bf16(int grad_dtype, int moment_dtype, int stochastic, int options);
 const void* step_kernel_e4m3(int grad_dtype, int moment_dtype, int stochastic, int options);
 const void* step_kernel_e4m3b(int grad_dtype, int moment_dtype, int stochastic, int options);
+const void* step_kernel_nvfp4(int grad_dtype, int moment_dtype, int stochastic, int options);
 
 }  // namespace mpadam

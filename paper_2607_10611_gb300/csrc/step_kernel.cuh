@@ -105,6 +105,16 @@ __device__ __forceinline__ uint32_t lds_u16(uint32_t addr) {
   asm volatile("ld.shared.u16 %0, [%1];" : "=h"(h) : "r"(addr));
   return h;
 }
+__device__ __forceinline__ uint32_t lds_u8(uint32_t addr) {
+  uint32_t v;
+  asm volatile("ld.shared.u8 %0, [%1];" : "=r"(v) : "r"(addr));
+  return v;
+}
+__device__ __forceinline__ uint32_t lds_u32(uint32_t addr) {
+  uint32_t v;
+  asm volatile("ld.shared.u32 %0, [%1];" : "=r"(v) : "r"(addr));
+  return v;
+}
 __device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
   asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
 }
@@ -563,8 +573,9 @@ struct TensorCtx {
   bool fast;           // whole tiles are fully staged and stored with vector stores
   float dec_scale, enc_scale;
   float cc_scale;      // E4M3 per-tensor: 2^e of the new encode (compute copy)
-  uint16_t* scale;     // kE4M3B block scales
+  void* scale;         // kE4M3B (FP16) / kNVFP4 (E4M3) block scales
   uint16_t* cc;        // BF16 compute copy, or nullptr
+  float gscale;        // kNVFP4 tensor scale
 };
 
 template <int WD, int GD, int MD>
@@ -572,21 +583,24 @@ __device__ __forceinline__ void load_tensor(const StepArgs& a, int k, TensorCtx&
   c.d = a.desc[k];
   c.g = a.grads[k];
   c.tiles = (c.d.numel + kTile - 1) / kTile;
-  c.vec = aligned(c.d.w, WD == kBF16 ? 16 : 8) && aligned(c.g, GD == kF32 ? 32 : 16) &&
+  c.vec = aligned(c.d.w, WD == kBF16 ? 16 : (WD == kNVFP4 ? 4 : 8)) && aligned(c.g, GD == kF32 ? 32 : 16) &&
           aligned(c.d.m, MD == kF32 ? 32 : 16) && aligned(c.d.v, MD == kF32 ? 32 : 16) &&
           aligned(c.d.ve, MD == kF32 ? 32 : 16);
   c.fast = c.vec && aligned(c.d.w, 16) && aligned(c.g, 16) && aligned(c.d.m, 16) && aligned(c.d.v, 16) &&
            aligned(c.d.ve, 16);
   c.dec_scale = c.enc_scale = c.cc_scale = 1.0f;
-  c.scale = c.cc = nullptr;
+  c.scale = nullptr;
+  c.cc = nullptr;
+  c.gscale = 1.0f;
   if (WD != kBF16 && a.aux) {
     const TensorAux x = a.aux[k];
     c.scale = x.scale;
     c.cc = x.compute;
+    c.gscale = x.gscale;
     // the compute copy joins the vector path only when 16-byte aligned;
     // block scales are staged (whole tiles: 240 bytes) only when 16-byte aligned
     if (c.cc && !aligned(c.cc, 16)) c.vec = c.fast = false;
-    if (WD == kE4M3B && !aligned(c.scale, 16)) c.fast = false;
+    if ((WD == kE4M3B || WD == kNVFP4) && !aligned(c.scale, 16)) c.fast = false;
   }
 }
 
@@ -896,7 +910,7 @@ __device__ __forceinline__ void finish_block(const StepArgs& a, const TensorCtx&
   ow[1] = code[4] | (code[5] << 8) | (code[6] << 16) | (code[7] << 24);
   put_e4m3(ow, x.d.w, e0, valid, x.vec);
   const uint32_t h_new = fp16_pow2_bits(k_new);
-  if ((threadIdx.x & 3) == 0 && valid > 0) x.scale[e0 / kBlock] = static_cast<uint16_t>(h_new);
+  if ((threadIdx.x & 3) == 0 && valid > 0) static_cast<uint16_t*>(x.scale)[e0 / kBlock] = static_cast<uint16_t>(h_new);
   if (x.cc) put_compute(ow, fp16_value(h_new), x.cc, e0, valid, x.vec);
   put_moments<MD>(x, e0, valid, m, v, ve);
 }
@@ -916,10 +930,11 @@ __device__ __noinline__ void general_block_group(const StepArgs& a, const Tensor
   // the block's old scale: staged when the tile's scale bytes through this block were
   const int nblk = (count + kBlock - 1) / kBlock, b = c >> 2;
   uint32_t h = 0u;
-  if (static_cast<uint32_t>(2 * (b + 1)) <= staged_bytes(x.scale + tile_e0 / kBlock, nblk, 2))
+  const uint16_t* sc = static_cast<const uint16_t*>(x.scale);
+  if (static_cast<uint32_t>(2 * (b + 1)) <= staged_bytes(sc + tile_e0 / kBlock, nblk, 2))
     h = lds_u16(st + a.off_s + 2 * b);
   else if (b < nblk)
-    h = x.scale[(tile_e0 / kBlock) + b];
+    h = sc[(tile_e0 / kBlock) + b];
   float w[8], g[8], m[8], v[8], ve[8];
   get_e4m3(w, end <= staged_bytes(x.d.w, count, 1), st + kGroup * c, x.d.w, e0, valid, x.vec, fp16_value(h));
   const bool g_st = end * GS <= staged_bytes(x.g, count, GS);
@@ -938,6 +953,321 @@ __device__ __noinline__ void general_block_group(const StepArgs& a, const Tensor
     get_bf16<false>(ve, e_st, st + a.off_ve + kGroup * MS * c, x.d.ve, e0, valid, x.vec);
   }
   finish_block<GD, MD, SR, OPT>(a, x, e0, valid, h, w, g, m, v, ve);
+}
+
+// ---------------------------------------------------------------------------
+// NVFP4 weights: E2M1 codes (OCP FP4: sign, 2 exponent bits with bias 1, one
+// mantissa bit; +-{0, 0.5, 1, 1.5, 2, 3, 4, 6}), an E4M3 scale s per 16
+// elements and a binary32 tensor scale G.  A weight decodes as q * d with
+// d = s * G (both products rounded to binary32); a step re-encodes
+// x = w' / d' (correctly rounded) under the block's new scale.  The two
+// threads of a pair (lanes 2p, 2p+1) hold one block.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ float e2m1_value(uint32_t c) {
+  const uint32_t mag = c & 7u;
+  const uint32_t b = mag >= 2u ? ((((mag >> 1) + 126u) << 23) | ((mag & 1u) << 22)) : (mag ? 0x3F000000u : 0u);
+  return __uint_as_float(b | ((c & 8u) << 28));
+}
+
+// binary32 -> E2M1 code: nearest-even, or stochastic (away from zero iff
+// r < floor(fraction * 2^32)); |x| >= 6 and infinities saturate; NaN -> +0.
+// Branch-free: with the grid spacing sp = 0.5, 1 or 2 of |x|'s binade
+// ([0, 2), [2, 4), [4, 6]), q = |x| / sp is exact, its integer part k and
+// fraction f give the code k + (0, 2 or 4) and the step up.
+template <bool SR>
+__device__ __forceinline__ uint32_t e2m1_encode(float x, uint32_t r) {
+  const float a = fminf(fabsf(x), 6.0f);
+  const float sp = a < 2.0f ? 0.5f : (a < 4.0f ? 1.0f : 2.0f);
+  const uint32_t off = a < 2.0f ? 0u : (a < 4.0f ? 2u : 4u);
+  const float q = __fdiv_rn(a, sp);  // a power-of-two divisor: exact
+  const float kf = truncf(q);
+  const float f = __fsub_rn(q, kf);  // exact
+  const uint32_t k = __float2uint_rz(kf);
+  uint32_t up;
+  if (SR) up = r < __float2uint_rz(__fmul_rn(f, 4294967296.0f)) ? 1u : 0u;
+  else up = (f > 0.5f || (f == 0.5f && (k & 1u))) ? 1u : 0u;
+  const uint32_t code = ((__float_as_uint(x) >> 28) & 8u) | (k + off + up);
+  return x != x ? 0u : code;
+}
+
+// Eight packed E2M1 codes (element j in bits [4j, 4j + 4)) -> binary32, with
+// the hardware E2M1 -> FP16 conversion (exact) and FP16 -> binary32.
+__device__ __forceinline__ void e2m1x8_to_f32(uint32_t packed, float (&x)[8]) {
+  uint32_t h[4];
+  asm("{\n .reg .b8 b0, b1, b2, b3;\n mov.b32 {b0, b1, b2, b3}, %4;\n"
+      " cvt.rn.f16x2.e2m1x2 %0, b0;\n cvt.rn.f16x2.e2m1x2 %1, b1;\n"
+      " cvt.rn.f16x2.e2m1x2 %2, b2;\n cvt.rn.f16x2.e2m1x2 %3, b3;\n}"
+      : "=r"(h[0]), "=r"(h[1]), "=r"(h[2]), "=r"(h[3])
+      : "r"(packed));
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&h[i]));
+    x[2 * i] = f.x;
+    x[2 * i + 1] = f.y;
+  }
+}
+
+// Eight binary32 -> packed E2M1 codes, nearest-even with saturation at +-6
+// (the hardware conversion; used only on finite values).
+__device__ __forceinline__ uint32_t e2m1x8_rn(const float (&x)[8]) {
+  uint32_t p;
+  asm("{\n .reg .b8 b0, b1, b2, b3;\n"
+      " cvt.rn.satfinite.e2m1x2.f32 b0, %2, %1;\n cvt.rn.satfinite.e2m1x2.f32 b1, %4, %3;\n"
+      " cvt.rn.satfinite.e2m1x2.f32 b2, %6, %5;\n cvt.rn.satfinite.e2m1x2.f32 b3, %8, %7;\n"
+      " mov.b32 %0, {b0, b1, b2, b3};\n}"
+      : "=r"(p)
+      : "f"(x[0]), "f"(x[1]), "f"(x[2]), "f"(x[3]), "f"(x[4]), "f"(x[5]), "f"(x[6]), "f"(x[7]));
+  return p;
+}
+
+// Stochastic E2M1 codes of both ends of an interval [xl, xh] (the same
+// random bits), sharing the binade of xl: the code of xl, and whether xh has
+// the same code (an end in another binade or sign reports false).
+__device__ __forceinline__ uint32_t e2m1_pair_sr(float xl, float xh, uint32_t r, bool& same) {
+  const float al = fminf(fabsf(xl), 6.0f), ah = fminf(fabsf(xh), 6.0f);
+  const float sp = al < 2.0f ? 0.5f : (al < 4.0f ? 1.0f : 2.0f);
+  const uint32_t off = al < 2.0f ? 0u : (al < 4.0f ? 2u : 4u);
+  const float ql = __fdiv_rn(al, sp), qh = __fdiv_rn(ah, sp);  // exact
+  const float kl = truncf(ql), kh = truncf(qh);
+  const uint32_t ul = r < __float2uint_rz(__fmul_rn(__fsub_rn(ql, kl), 4294967296.0f)) ? 1u : 0u;
+  const uint32_t uh = r < __float2uint_rz(__fmul_rn(__fsub_rn(qh, kh), 4294967296.0f)) ? 1u : 0u;
+  same = kl == kh && ul == uh && ((__float_as_uint(xl) ^ __float_as_uint(xh)) >> 31) == 0u && xl == xl && xh == xh;
+  return ((__float_as_uint(xl) >> 28) & 8u) | (__float2uint_rz(kl) + off + ul);
+}
+
+// Does E4M3 scale code c cover A (6 * (s * G) >= A, products rounded)?
+__device__ __forceinline__ bool fp4_covers(uint32_t c, float G, float A) {
+  return __fmul_rn(6.0f, __fmul_rn(e4m3_value(c), G)) >= A;
+}
+
+// Block scale code of the next encode: the smallest code in [1, 126] that
+// covers A (finite, >= 0), 126 when none does, c_old when A = 0.  Starts at
+// the E4M3 code of an estimate of A / (6 G) and steps to the smallest
+// covering code (covering is monotone in the code).
+__device__ __forceinline__ uint32_t nvfp4_scale_code(float A, float G, uint32_t c_old) {
+  if (!(A > 0.0f)) return c_old;
+  const float est = div_approx<false>(A, __fmul_rn(6.0f, G));
+  int32_t c = static_cast<int32_t>(e4m3_encode<false>(est, 0u) & 0x7Fu);
+  c = c < 1 ? 1 : (c > 126 ? 126 : c);
+  for (int i = 0; i < 126 && c > 1 && fp4_covers(static_cast<uint32_t>(c - 1), G, A); ++i) --c;
+  for (int i = 0; i < 126 && c < 126 && !fp4_covers(static_cast<uint32_t>(c), G, A); ++i) ++c;
+  return static_cast<uint32_t>(c);
+}
+
+// Eight packed codes (element j in bits [4j, 4j + 4)) -> the group's bytes.
+__device__ __forceinline__ void put_fp4(uint32_t packed, void* w, int64_t e0, int valid, bool vec) {
+  uint8_t* p = static_cast<uint8_t*>(w) + e0 / 2;
+  if (vec && valid == kGroup) {
+    asm volatile("st.global.L1::no_allocate.u32 [%0], %1;" ::"l"(p), "r"(packed) : "memory");
+  } else {
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      if (2 * k < valid) {
+        uint32_t byte = (packed >> (8 * k)) & 0xFFu;
+        if (2 * k + 1 >= valid) byte &= 0x0Fu;  // past the tensor's end: the spare nibble is 0
+        p[k] = static_cast<uint8_t>(byte);
+      }
+    }
+  }
+}
+
+__device__ __forceinline__ uint32_t pair_max(uint32_t x) {
+  return max(x, __shfl_xor_sync(0xFFFFFFFFu, x, 1));
+}
+
+template <int GD, int MD, bool SR, bool OPT>
+__device__ __forceinline__ void finish_fp4(const StepArgs& a, const TensorCtx& x, int64_t e0, int valid,
+                                           uint32_t c_old, float (&w)[8], float (&g)[8], float (&m)[8],
+                                           float (&v)[8], float (&ve)[8]) {
+  const float G = x.gscale;
+  const uint64_t gi = static_cast<uint64_t>(x.d.goff + e0) >> 3;  // global group index (random lanes)
+  uint32_t rnd[8];
+  if (SR) group_random_bits<kNVFP4>(a, gi << 3, rnd);
+  const uint32_t vmask = valid >= kGroup ? 0xFFu : (valid > 0 ? (1u << valid) - 1u : 0u);
+  uint32_t code[8];
+  uint32_t c_new;
+  float d;
+  if (!OPT && a.s.cert_ok) {
+    // Certified path, as for block-scaled E4M3: fast weights and one error
+    // bound et; the pair's maximum bounds decide the scale code (exact
+    // maximum where they do not); then each element's interval, divided by
+    // d through an approximate reciprocal and widened by 2^-20 relative and
+    // 2^-126 absolute (beyond the approximation's error), is encoded at both
+    // ends.
+    float wf[8];
+    float et = 0.0f, am = 0.0f;
+    uint32_t bad = 0u;
+#pragma unroll
+    for (int j = 0; j < kGroup; ++j) {
+      const CertUpd u = madam_update_cert<false>(a.s, w[j], g[j], m[j], v[j], ve[j]);
+      wf[j] = u.wn;
+      m[j] = u.m; v[j] = u.v; ve[j] = u.ve;
+      if (!u.ok) {
+        bad |= 1u << j;
+      } else {
+        et = fmaxf(et, u.e);
+        if ((vmask >> j) & 1u) am = fmaxf(am, fabsf(u.wn));
+      }
+    }
+    bad &= vmask;
+    const float lo_t = bad ? 0.0f : fmaxf(__fsub_rd(am, et), 0.0f);
+    const float hi_t = bad ? INFINITY : __fadd_ru(am, et);
+    const uint32_t plo = pair_max(__float_as_uint(lo_t));
+    const uint32_t phi = pair_max(__float_as_uint(hi_t));
+    const uint32_t cl = nvfp4_scale_code(__uint_as_float(plo), G, c_old);
+    // the upper bound has the same code iff that code still covers it (or is the top one)
+    const bool certain = plo != 0u && phi < 0x7E800000u /* 2^126 */ &&
+                         (cl == 126u || fp4_covers(cl, G, __uint_as_float(phi)));
+    c_new = cl;
+    if (__any_sync(0xFFFFFFFFu, !certain)) {  // exact block maximum for the undecided pairs
+      uint32_t amx = 0u;
+      if (!certain) {
+#pragma unroll
+        for (int j = 0; j < kGroup; ++j) {
+          if ((vmask >> j) & 1u) {
+            const uint32_t bb = __float_as_uint(madam_wn_exact(a.s, w[j], g[j], m[j], v[j], ve[j])) & 0x7FFFFFFFu;
+            if (bb < 0x7F800000u) amx = max(amx, bb);
+          }
+        }
+      }
+      amx = pair_max(amx);
+      if (!certain) c_new = nvfp4_scale_code(__uint_as_float(amx), G, c_old);
+    }
+    d = __fmul_rn(e4m3_value(c_new), G);
+    uint32_t redo = bad;
+    if (d >= 1.1754943508222875e-38f /* 2^-126 */ && d <= 8.507059173023462e+37f /* 2^126 */) {
+      // w' / d bounded through one approximate reciprocal (1 ulp) and a
+      // product (half an ulp): within 2^-22 relative, widened to 2^-20
+      float inv;
+      asm("rcp.approx.f32 %0, %1;" : "=f"(inv) : "f"(d));
+      if (SR) {
+#pragma unroll
+        for (int j = 0; j < kGroup; ++j) {
+          const float ql = __fmul_rn(__fsub_rd(wf[j], et), inv);
+          const float qh = __fmul_rn(__fadd_ru(wf[j], et), inv);
+          const float xl = __fsub_rd(ql, __fmaf_ru(fabsf(ql), 9.5367431640625e-07f /* 2^-20 */, 1.1754943508222875e-38f));
+          const float xh = __fadd_ru(qh, __fmaf_ru(fabsf(qh), 9.5367431640625e-07f, 1.1754943508222875e-38f));
+          bool same;
+          code[j] = e2m1_pair_sr(xl, xh, rnd[j], same);
+          if (!same) redo |= 1u << j;
+        }
+      } else {
+        float xl[8], xh[8];
+#pragma unroll
+        for (int j = 0; j < kGroup; ++j) {
+          const float ql = __fmul_rn(__fsub_rd(wf[j], et), inv);
+          const float qh = __fmul_rn(__fadd_ru(wf[j], et), inv);
+          xl[j] = __fsub_rd(ql, __fmaf_ru(fabsf(ql), 9.5367431640625e-07f /* 2^-20 */, 1.1754943508222875e-38f));
+          xh[j] = __fadd_ru(qh, __fmaf_ru(fabsf(qh), 9.5367431640625e-07f, 1.1754943508222875e-38f));
+        }
+        const uint32_t pl = e2m1x8_rn(xl), diff = pl ^ e2m1x8_rn(xh);
+#pragma unroll
+        for (int j = 0; j < kGroup; ++j) {
+          code[j] = (pl >> (4 * j)) & 0xFu;
+          if ((diff >> (4 * j)) & 0xFu) redo |= 1u << j;
+        }
+      }
+    } else {
+      redo = 0xFFu;
+    }
+    redo &= vmask;
+    if (redo) {  // rare: the canonical weight of the undecided elements
+#pragma unroll
+      for (int j = 0; j < kGroup; ++j) {
+        if ((redo >> j) & 1u) {
+          const float xe = __fdiv_rn(madam_wn_exact(a.s, w[j], g[j], m[j], v[j], ve[j]), d);
+          code[j] = e2m1_encode<SR>(xe, SR ? rnd[j] : 0u);
+        }
+      }
+    }
+  } else {
+    float wn[8];
+    uint32_t amx = 0u;
+#pragma unroll
+    for (int j = 0; j < kGroup; ++j) {
+      const Upd u = madam_update<OPT>(a.s, w[j], g[j], m[j], v[j], ve[j]);
+      wn[j] = u.wn; m[j] = u.m; v[j] = u.v; ve[j] = u.ve;
+      const uint32_t bb = __float_as_uint(u.wn) & 0x7FFFFFFFu;
+      if (((vmask >> j) & 1u) && bb < 0x7F800000u) amx = max(amx, bb);
+    }
+    c_new = nvfp4_scale_code(__uint_as_float(pair_max(amx)), G, c_old);
+    d = __fmul_rn(e4m3_value(c_new), G);
+#pragma unroll
+    for (int j = 0; j < kGroup; ++j) code[j] = e2m1_encode<SR>(__fdiv_rn(wn[j], d), SR ? rnd[j] : 0u);
+  }
+  uint32_t packed = 0u;
+#pragma unroll
+  for (int j = 0; j < kGroup; ++j) packed |= (code[j] & 0xFu) << (4 * j);
+  put_fp4(packed, x.d.w, e0, valid, x.vec);
+  if ((threadIdx.x & 1) == 0 && valid > 0) static_cast<uint8_t*>(x.scale)[e0 / kFp4Block] = static_cast<uint8_t>(c_new);
+  if (x.cc) {
+    float q[8];
+    e2m1x8_to_f32(packed, q);
+    uint32_t o[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) o[i] = bf16x2_rn(__fmul_rn(q[2 * i], d), __fmul_rn(q[2 * i + 1], d));
+    put_bf16(o, x.cc, e0, valid, x.vec);
+  }
+  put_moments<MD>(x, e0, valid, m, v, ve);
+}
+
+// Eight NVFP4 weights decoded with d: from the stage or global memory as one
+// 32-bit word when whole, else nibble by nibble.
+__device__ __forceinline__ void get_fp4(float (&w)[8], bool staged, uint32_t saddr, const void* gw, int64_t e0,
+                                        int valid, bool vec, float d) {
+  if (staged || (vec && valid == kGroup)) {
+    uint32_t r;
+    if (staged) r = lds_u32(saddr);
+    else asm("ld.global.L1::no_allocate.u32 %0, [%1];" : "=r"(r) : "l"(static_cast<const uint8_t*>(gw) + e0 / 2));
+    e2m1x8_to_f32(r, w);
+#pragma unroll
+    for (int j = 0; j < kGroup; ++j) w[j] = __fmul_rn(w[j], d);
+  } else {
+    const uint8_t* p = static_cast<const uint8_t*>(gw);
+#pragma unroll
+    for (int j = 0; j < kGroup; ++j) {
+      const int64_t k = e0 + j;
+      w[j] = j < valid ? __fmul_rn(e2m1_value((k & 1) ? (p[k >> 1] >> 4) : (p[k >> 1] & 0xFu)), d) : 0.0f;
+    }
+  }
+}
+
+// One NVFP4 group of a partial tile or of a tensor whose arrays are not all
+// staged; every consumer lane calls this (the block maximum is a pair shuffle).
+template <int GD, int MD, bool SR, bool OPT>
+__device__ __noinline__ void general_fp4_group(const StepArgs& a, const TensorCtx& x, int64_t tile_e0, int count,
+                                               int c, uint32_t st) {
+  constexpr int GS = esize_of(GD), MS = esize_of(MD);
+  const int rem = count - kGroup * c;
+  const int valid = rem < 0 ? 0 : (rem < kGroup ? rem : kGroup);
+  const int64_t e0 = tile_e0 + kGroup * c;
+  const uint32_t end = static_cast<uint32_t>(kGroup * (c + 1));  // elements through this group
+  const int nblk = (count + kFp4Block - 1) / kFp4Block, b = c >> 1;
+  const uint8_t* sc = static_cast<const uint8_t*>(x.scale);
+  uint32_t s_old = 0u;
+  if (static_cast<uint32_t>(b + 1) <= staged_bytes(sc + tile_e0 / kFp4Block, nblk, 1))
+    s_old = lds_u8(st + a.off_s + b);
+  else if (b < nblk)
+    s_old = sc[(tile_e0 / kFp4Block) + b];
+  const float d_old = __fmul_rn(e4m3_value(s_old), x.gscale);
+  float w[8], g[8], m[8], v[8], ve[8];
+  get_fp4(w, end / 2 <= staged_bytes(x.d.w, (count + 1) / 2, 1), st + 4 * c, x.d.w, e0, valid, x.vec, d_old);
+  const bool g_st = end * GS <= staged_bytes(x.g, count, GS);
+  if (GD == kF32) get_f32<true>(g, g_st, st + a.off_g + kGroup * GS * c, x.g, e0, valid, x.vec);
+  else get_bf16<true>(g, g_st, st + a.off_g + kGroup * GS * c, x.g, e0, valid, x.vec);
+  const bool m_st = end * MS <= staged_bytes(x.d.m, count, MS);
+  const bool v_st = end * MS <= staged_bytes(x.d.v, count, MS);
+  const bool e_st = end * MS <= staged_bytes(x.d.ve, count, MS);
+  if (MD == kF32) {
+    get_f32<false>(m, m_st, st + a.off_m + kGroup * MS * c, x.d.m, e0, valid, x.vec);
+    get_f32<false>(v, v_st, st + a.off_v + kGroup * MS * c, x.d.v, e0, valid, x.vec);
+    get_f32<false>(ve, e_st, st + a.off_ve + kGroup * MS * c, x.d.ve, e0, valid, x.vec);
+  } else {
+    get_bf16<false>(m, m_st, st + a.off_m + kGroup * MS * c, x.d.m, e0, valid, x.vec);
+    get_bf16<false>(v, v_st, st + a.off_v + kGroup * MS * c, x.d.v, e0, valid, x.vec);
+    get_bf16<false>(ve, e_st, st + a.off_ve + kGroup * MS * c, x.d.ve, e0, valid, x.vec);
+  }
+  finish_fp4<GD, MD, SR, OPT>(a, x, e0, valid, s_old, w, g, m, v, ve);
 }
 
 // ---------------------------------------------------------------------------
@@ -975,7 +1305,7 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
     int k = a.cta_first[blockIdx.x];
     TensorDesc d = a.desc[k];
     const void* gp = a.grads[k];
-    const uint16_t* sp = WD == kE4M3B ? a.aux[k].scale : nullptr;
+    const uint8_t* sp = (WD == kE4M3B || WD == kNVFP4) ? static_cast<const uint8_t*>(a.aux[k].scale) : nullptr;
     int64_t tiles = (d.numel + kTile - 1) / kTile;
     int s = 0;
     uint32_t use = 0;
@@ -986,7 +1316,7 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
         ++k;
         d = a.desc[k];
         gp = a.grads[k];
-        if (WD == kE4M3B) sp = a.aux[k].scale;
+        if (WD == kE4M3B || WD == kNVFP4) sp = static_cast<const uint8_t*>(a.aux[k].scale);
         tiles = (d.numel + kTile - 1) / kTile;
       }
       if (use > 0 && !mbar_wait(smem_addr(&empty_bar[s]), (use - 1) & 1u)) {
@@ -996,19 +1326,24 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
       }
       const int64_t e0 = (t - d.tile_off) * kTile;
       const int count = static_cast<int>(d.numel - e0 < kTile ? d.numel - e0 : kTile);
-      const uint32_t nw = staged_bytes(d.w, count, WS), ng = staged_bytes(gp, count, GS);
+      // NVFP4 weights: half a byte per element (tile starts stay 16-byte aligned: 1920 bytes per tile)
+      const uint32_t nw = WD == kNVFP4 ? staged_bytes(d.w, (count + 1) / 2, 1) : staged_bytes(d.w, count, WS);
+      const uint32_t ng = staged_bytes(gp, count, GS);
       const uint32_t nm = staged_bytes(d.m, count, MS), nv = staged_bytes(d.v, count, MS);
       const uint32_t nve = staged_bytes(d.ve, count, MS);
-      const uint32_t ns = WD == kE4M3B ? staged_bytes(sp + e0 / kBlock, (count + kBlock - 1) / kBlock, 2) : 0u;
+      const int64_t s0 = WD == kE4M3B ? 2 * (e0 / kBlock) : e0 / kFp4Block;  // the tile's first scale byte
+      const uint32_t ns = WD == kE4M3B   ? staged_bytes(sp + s0, 2 * ((count + kBlock - 1) / kBlock), 1)
+                          : WD == kNVFP4 ? staged_bytes(sp + s0, (count + kFp4Block - 1) / kFp4Block, 1)
+                                         : 0u;
       const uint32_t bar = smem_addr(&full_bar[s]);
       const uint32_t st = smem0 + static_cast<uint32_t>(s * a.stage_bytes);
       mbar_arrive_expect_tx(bar, nw + ng + nm + nv + nve + ns);
-      if (nw) tma_load(st, static_cast<const uint8_t*>(d.w) + e0 * WS, nw, bar, pol);
+      if (nw) tma_load(st, static_cast<const uint8_t*>(d.w) + (WD == kNVFP4 ? e0 / 2 : e0 * WS), nw, bar, pol);
       if (ng) tma_load(st + a.off_g, static_cast<const uint8_t*>(gp) + e0 * GS, ng, bar, pol);
       if (nm) tma_load(st + a.off_m, static_cast<const uint8_t*>(d.m) + e0 * MS, nm, bar, pol);
       if (nv) tma_load(st + a.off_v, static_cast<const uint8_t*>(d.v) + e0 * MS, nv, bar, pol);
       if (nve) tma_load(st + a.off_ve, static_cast<const uint8_t*>(d.ve) + e0 * MS, nve, bar, pol);
-      if (ns) tma_load(st + a.off_s, sp + e0 / kBlock, ns, bar, pol);
+      if (ns) tma_load(st + a.off_s, sp + s0, ns, bar, pol);
       ++issued;
       if (++s == S) { s = 0; ++use; }
     }
@@ -1076,9 +1411,12 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
         get_bf16<false>(w, true, st + kGroup * WS * c, x.d.w, e0, kGroup, true);
       } else if (WD == kE4M3) {
         get_e4m3(w, true, st + kGroup * WS * c, x.d.w, e0, kGroup, true, x.dec_scale);
-      } else {
+      } else if (WD == kE4M3B) {
         h_old = lds_u16(st + a.off_s + 2 * (c >> 2));
         get_e4m3(w, true, st + kGroup * WS * c, x.d.w, e0, kGroup, true, fp16_value(h_old));
+      } else {
+        h_old = lds_u8(st + a.off_s + (c >> 1));
+        get_fp4(w, true, st + 4 * c, x.d.w, e0, kGroup, true, __fmul_rn(e4m3_value(h_old), x.gscale));
       }
       if (GD == kF32) get_f32<true>(g, true, st + a.off_g + kGroup * GS * c, x.g, e0, kGroup, true);
       else get_bf16<true>(g, true, st + a.off_g + kGroup * GS * c, x.g, e0, kGroup, true);
@@ -1094,6 +1432,7 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
       __syncwarp();
       if (lane == 0) mbar_arrive(smem_addr(&empty_bar[s]));
       if constexpr (WD == kE4M3B) finish_block<GD, MD, SR, OPT>(a, x, e0, kGroup, h_old, w, g, m, v, ve);
+      else if constexpr (WD == kNVFP4) finish_fp4<GD, MD, SR, OPT>(a, x, e0, kGroup, h_old, w, g, m, v, ve);
       else finish_group<WD, GD, MD, SR, OPT>(a, x, e0, kGroup, w, g, m, v, ve, amax_bits);
       if (++s == S) { s = 0; ++use; }
       continue;
@@ -1101,6 +1440,8 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
     // partial tile or unstaged arrays: element-wise fallback, out of line
     if constexpr (WD == kE4M3B)
       general_block_group<GD, MD, SR, OPT>(a, x, tile_e0, count, c, smem0 + static_cast<uint32_t>(s * a.stage_bytes));
+    else if constexpr (WD == kNVFP4)
+      general_fp4_group<GD, MD, SR, OPT>(a, x, tile_e0, count, c, smem0 + static_cast<uint32_t>(s * a.stage_bytes));
     else
       general_group<WD, GD, MD, SR, OPT>(a, x, tile_e0, count, c, smem0 + static_cast<uint32_t>(s * a.stage_bytes),
                                          amax_bits);

@@ -5,8 +5,9 @@ scales, compute copies) so their memory outlives the native state, allocates
 the E4M3 scale rings with torch, and forwards every step to mpadam_step on
 the current torch stream.  `weight_dtype` is one format for the whole list
 ("bf16", "e4m3") or a list with one format per tensor ("bf16", "e4m3",
-"e4m3_b32"); the latter, block scales or compute copies go through
-mpadam_create_ex.
+"e4m3_b32", "nvfp4"); the latter, block scales or compute copies go through
+mpadam_create_ex.  NVFP4 weights are packed bytes (two codes each), so the
+element count of every tensor is taken from its first moment.
 """
 from __future__ import annotations
 
@@ -16,7 +17,9 @@ import torch
 
 from . import _native as N
 
-_STORAGE = {"bf16": torch.bfloat16, "e4m3": torch.uint8, "e4m3_b32": torch.uint8, "f32": torch.float32}
+_STORAGE = {"bf16": torch.bfloat16, "e4m3": torch.uint8, "e4m3_b32": torch.uint8, "nvfp4": torch.uint8,
+            "f32": torch.float32}
+_SCALES = {"e4m3_b32": torch.float16, "nvfp4": torch.uint8}
 
 
 class MPAdam:
@@ -25,14 +28,16 @@ class MPAdam:
                  moment_dtype: str = "f32", rounding: str = "nearest", seed: int = 0,
                  fp8_exp: Optional[Sequence[int]] = None, first_step: int = 1,
                  block_scales: Optional[Sequence[Optional[torch.Tensor]]] = None,
-                 compute: Optional[Sequence[Optional[torch.Tensor]]] = None, **hparams):
+                 compute: Optional[Sequence[Optional[torch.Tensor]]] = None,
+                 global_scales: Optional[Sequence[float]] = None, **hparams):
         self.w, self.m, self.v, self.ve = list(w), list(m), list(v), list(ve)
         self.n = len(self.w)
         per_tensor = not isinstance(weight_dtype, str)
         self.formats = list(weight_dtype) if per_tensor else [weight_dtype] * self.n
         self.block_scales = list(block_scales) if block_scales is not None else [None] * self.n
         self.compute = list(compute) if compute is not None else [None] * self.n
-        if not (len(self.formats) == len(self.block_scales) == len(self.compute) == self.n):
+        self.global_scales = [float(x or 0.0) for x in global_scales] if global_scales is not None else [0.0] * self.n
+        if not (len(self.formats) == len(self.block_scales) == len(self.compute) == len(self.global_scales) == self.n):
             raise ValueError("one weight format, block-scale and compute entry per tensor")
         self.weight_dtype, self.grad_dtype, self.moment_dtype = weight_dtype, grad_dtype, moment_dtype
         for t, dt in [(x, f) for x, f in zip(self.w, self.formats)] + \
@@ -40,9 +45,10 @@ class MPAdam:
                      [(x, "bf16") for x in self.compute if x is not None]:
             if t.dtype != _STORAGE[dt] or not t.is_cuda or not t.is_contiguous():
                 raise ValueError(f"expected contiguous CUDA tensors of {_STORAGE[dt]}")
-        for x in self.block_scales:
-            if x is not None and (x.dtype != torch.float16 or not x.is_cuda or not x.is_contiguous()):
-                raise ValueError("block scales must be contiguous CUDA float16 tensors")
+        for x, f in zip(self.block_scales, self.formats):
+            if x is not None and (x.dtype != _SCALES.get(f) or not x.is_cuda or not x.is_contiguous()):
+                raise ValueError("block scales must be contiguous CUDA tensors (float16 for e4m3_b32, "
+                                 "uint8 E4M3 codes for nvfp4)")
         extended = per_tensor or any(x is not None for x in self.block_scales + self.compute)
         uniform = weight_dtype if not per_tensor else "bf16"
         self.cfg = N.make_config(weight_dtype="bf16" if extended else uniform, grad_dtype=grad_dtype,
@@ -58,9 +64,10 @@ class MPAdam:
         with torch.cuda.device(dev):
             if extended:
                 self.state = N.mpadam_create_ex(
-                    [(a.data_ptr(), b.data_ptr(), c.data_ptr(), d.data_ptr(), a.numel(), f, ptr(bs), ptr(cc))
-                     for a, b, c, d, f, bs, cc in zip(self.w, self.m, self.v, self.ve, self.formats,
-                                                      self.block_scales, self.compute)], self.cfg, *rings)
+                    [(a.data_ptr(), b.data_ptr(), c.data_ptr(), d.data_ptr(), b.numel(), f, ptr(bs), ptr(cc), gs)
+                     for a, b, c, d, f, bs, cc, gs in zip(self.w, self.m, self.v, self.ve, self.formats,
+                                                          self.block_scales, self.compute, self.global_scales)],
+                    self.cfg, *rings)
             else:
                 self.state = N.mpadam_create(
                     [(a.data_ptr(), b.data_ptr(), c.data_ptr(), d.data_ptr(), a.numel())

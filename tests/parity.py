@@ -22,7 +22,8 @@ import oracle
 import workloads as W
 from paper_2607_10611_gb300.optimizer import MPAdam
 
-ODT = {"f32": oracle.F32, "bf16": oracle.BF16, "e4m3": oracle.E4M3, "e4m3_b32": oracle.E4M3_B32}
+ODT = {"f32": oracle.F32, "bf16": oracle.BF16, "e4m3": oracle.E4M3, "e4m3_b32": oracle.E4M3_B32,
+       "nvfp4": oracle.NVFP4}
 HP_KEYS = ("lr_add", "lr_mul", "beta1", "beta2", "eps", "tau", "rmax_pos", "rmax_neg", "g_max",
            "dmult_max", "w_max", "wd_add", "bias_correction")
 
@@ -39,6 +40,8 @@ def host_tensors(mt: W.Materialized) -> List[dict]:
                  v=W.to_numpy_bits(mt.v[k]), ve=W.to_numpy_bits(mt.ve[k]))
         if mt.bscale and mt.bscale[k] is not None:
             d["bscale"] = W.to_numpy_bits(mt.bscale[k])
+        if mt.gscale and mt.gscale[k]:
+            d["gscale"] = float(mt.gscale[k])
         out.append(d)
     return out
 
@@ -126,7 +129,8 @@ class Run:
                           moment_dtype=wl.moment_dtype, rounding=wl.rounding, seed=wl.seed,
                           fp8_exp=self.mt.fp8_exp,
                           block_scales=self.dev["bscale"] if extended else None,
-                          compute=self.dev["cc"] if extended else None, **gkw)
+                          compute=self.dev["cc"] if extended else None,
+                          global_scales=self.mt.gscale if extended else None, **gkw)
         self.e4m3 = [k for k, f in enumerate(self.formats) if f == "e4m3"]
         self.fp8 = None
         if self.e4m3:
@@ -151,6 +155,8 @@ class Run:
         h = self.host[k]
         if self.formats[k] == "e4m3_b32":
             return oracle.dequant_bf16(h["w"], bscale=h["bscale"])
+        if self.formats[k] == "nvfp4":
+            return oracle.dequant_nvfp4_bf16(h["g"].size, h["w"], h["bscale"], h["gscale"])
         return oracle.dequant_bf16(h["w"], e=self.fp8[k][0])
 
     def compare(self, t_next: int, compute_copy: bool = True) -> Dict[str, int]:
@@ -160,7 +166,7 @@ class Run:
         res = {"w": 0, "m": 0, "v": 0, "ve": 0, "bscale": 0, "cc": 0, "elements": 0, "contract_ok": True}
         for k in range(len(self.host)):
             h = self.host[k]
-            res["elements"] += h["w"].size
+            res["elements"] += h["g"].size
             gw = W.to_numpy_bits(self.dev["w"][k])
             gm = W.to_numpy_bits(self.dev["m"][k])
             res["w"] += mismatches(gw, h["w"])
@@ -169,9 +175,15 @@ class Run:
             res["ve"] += mismatches(W.to_numpy_bits(self.dev["ve"][k]), h["ve"])
             if "bscale" in h:
                 res["bscale"] += mismatches(W.to_numpy_bits(self.dev["bscale"][k]), h["bscale"])
-            if compute_copy and self.stepped and self.dev["cc"][k] is not None and h["w"].size:
+            if compute_copy and self.stepped and self.dev["cc"][k] is not None and h["g"].size:
                 res["cc"] += mismatches(W.to_numpy_bits(self.dev["cc"][k]), self.expected_compute_copy(k))
             fmt = "bf16" if self.formats[k] == "bf16" else "e4m3"
+            if self.formats[k] == "nvfp4":   # codes compared through their nibbles
+                gw = oracle.nvfp4_unpack(gw, h["g"].size)
+                hw = oracle.nvfp4_unpack(h["w"], h["g"].size)
+                if hw.size and not contract_ok(gw, hw, gm, h["m"], "e4m3"):
+                    res["contract_ok"] = False
+                continue
             if h["w"].size and not contract_ok(gw, h["w"], gm, h["m"], fmt):
                 res["contract_ok"] = False
         if self.fp8 is not None:

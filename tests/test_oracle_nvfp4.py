@@ -178,3 +178,26 @@ def test_nvfp4_dequant_is_payload_times_block_scale():
     w = pay * np.repeat((vals[bs] * G).astype(F), 16)[:n]
     want = torch.from_numpy(w.astype(F)).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
     np.testing.assert_array_equal(got, want)
+
+
+def test_list_step_indexes_nvfp4_tensors_by_element_count():
+    """Global indices follow element counts: an NVFP4 tensor of n elements
+    (n/2 packed bytes) moves the next tensor's first index by n rounded up
+    to a multiple of 8, so the next tensor draws the same random lanes as
+    when stepped alone at that offset."""
+    rng = np.random.default_rng(6)
+    G = F(2.0 ** -12)
+    mk = lambda n: dict(g=(rng.standard_normal(n) * 1e-3).astype(F), m=np.zeros(n, F), v=np.zeros(n, F),
+                        ve=np.zeros(n, F))
+    a = mk(37)
+    a["bscale"] = np.full(3, 90, np.uint8)
+    a["gscale"] = float(G)
+    a["w"] = oracle.nvfp4_pack(rng.integers(0, 16, 37).astype(np.uint8))
+    b = mk(50)
+    b["w"] = oracle.bf16_rne((rng.standard_normal(50) * 0.02).astype(F))
+    ref = {k: v.copy() if isinstance(v, np.ndarray) else v for k, v in b.items()}
+    hp = oracle.hparams(stochastic=1, seed=9)
+    oracle.step([a, b], wdt=[oracle.NVFP4, oracle.BF16], gdt=F32, mdt=F32, hp=hp, t=1)
+    assert oracle.global_offsets([37, 50]) == [0, 40]
+    oracle.step_elements(hp, 1, oracle.BF16, F32, F32, ref["w"], ref["g"], ref["m"], ref["v"], ref["ve"], gidx0=40)
+    np.testing.assert_array_equal(b["w"], ref["w"])

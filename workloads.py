@@ -7,8 +7,10 @@ rule).  The FP8 initial weights are produced with torch's own float8_e4m3fn
 cast of a pre-scaled draw, with a per-role power-of-two exponent chosen from
 the draw's standard deviation (per-tensor scaling), or per 32-element block
 the power of two at or above the block's largest |w| / 448 computed with
-torch in binary64 (block scaling): an input recipe, not the optimizer's
-scale rules.
+torch in binary64 (block scaling).  NVFP4 weights take a power-of-two tensor
+scale per role, per 16-element block the smallest E4M3 value whose range
+covers the block (binary64), and the nearest E2M1 code (torch bucketize):
+input recipes, not the optimizer's scale or rounding rules.
 
 Stand-ins: the paper trains LLaMA-style decoders on C4/EN (Sec. 5.2, the
 model-architecture table of Appendix C).  An optimizer step needs no data, so
@@ -44,7 +46,7 @@ class TensorSpec:
 class Workload:
     name: str
     specs: tuple
-    weight_dtype: str          # "bf16" | "e4m3" | "e4m3_b32" | "mixed_b32" (see format_of)
+    weight_dtype: str          # "bf16" | "e4m3" | "e4m3_b32" | "nvfp4" | "mixed_b32" | "mixed_fp4" (see format_of)
     grad_dtype: str            # "f32" | "bf16"
     moment_dtype: str          # "f32" | "bf16"
     rounding: str              # "nearest" | "stochastic"
@@ -65,6 +67,8 @@ class Workload:
         and the LM head BF16."""
         if self.weight_dtype == "mixed_b32":
             return "e4m3_b32" if spec.role == "matrix" else "bf16"
+        if self.weight_dtype == "mixed_fp4":
+            return "nvfp4" if spec.role == "matrix" else "bf16"
         return self.weight_dtype
 
     @property
@@ -190,6 +194,18 @@ def _llama15_mixed(layers=24, d=2048, ffn=5632, vocab=32000, name="llama_1p5b_mi
                     "tensor, fp32 moments, stochastic rounding")
 
 
+def _llama15_nvfp4(layers=24, d=2048, ffn=5632, vocab=32000, name="llama_1p5b_nvfp4"):
+    return Workload(
+        name=name, specs=llama_specs(layers, d, ffn, vocab),
+        weight_dtype="mixed_fp4", grad_dtype="bf16", moment_dtype="f32", rounding="nearest",
+        steps=10, grad=("student_t_logu", 3.0, 1e-5, 1e-2), compute_copy=True,
+        description="LLaMA-style 1.5B list in the paper's NVFP4 regime: linear layers NVFP4 (E2M1 "
+                    "codes, an E4M3 scale per 16 weights, a tensor scale) with a BF16 compute copy "
+                    "written by the step, embeddings / norms / LM head BF16; bf16 Student-t(3) grads "
+                    "scaled per tensor, fp32 moments, round-to-nearest (the paper trains M+Adam "
+                    "without stochastic rounding)")
+
+
 def _llama7(layers=32, d=4096, ffn=11008, vocab=32000, name="llama_7b"):
     return Workload(
         name=name, specs=llama_specs(layers, d, ffn, vocab),
@@ -216,6 +232,7 @@ CONFIGS: Dict[str, Workload] = {
     "llama_7b": _llama7(),
     "ragged_20k": _ragged(),
     "llama_1p5b_mixed": _llama15_mixed(),
+    "llama_1p5b_nvfp4": _llama15_nvfp4(),
 }
 
 # Same distributions and formats at sizes the oracle finishes in seconds,
@@ -227,14 +244,18 @@ SMALL: Dict[str, Workload] = {
     "llama_7b": _llama7(layers=2, d=128, ffn=344, vocab=517, name="llama7_small"),
     "ragged_20k": _ragged(n=300, max_log2=13, name="ragged_small"),
     "llama_1p5b_mixed": _llama15_mixed(layers=2, d=128, ffn=344, vocab=517, name="llama15_mixed_small"),
+    "llama_1p5b_nvfp4": _llama15_nvfp4(layers=2, d=128, ffn=344, vocab=517, name="llama15_nvfp4_small"),
 }
 
 
 # ---------------------------------------------------------------------------
 # Materialisation
 # ---------------------------------------------------------------------------
-_TORCH = {"f32": torch.float32, "bf16": torch.bfloat16, "e4m3": torch.uint8, "e4m3_b32": torch.uint8}
-BLOCK = 32  # elements per block scale (block-scaled E4M3)
+_TORCH = {"f32": torch.float32, "bf16": torch.bfloat16, "e4m3": torch.uint8, "e4m3_b32": torch.uint8,
+          "nvfp4": torch.uint8}
+BLOCK = 32      # elements per block scale (block-scaled E4M3)
+FP4_BLOCK = 16  # elements per block scale (NVFP4)
+_E2M1_MIDPOINTS = (0.25, 0.75, 1.25, 1.75, 2.5, 3.5, 5.0)  # between the grid values 0 .. 6
 
 
 def _gen(device, seed, k, salt):
@@ -267,6 +288,39 @@ def block_initial_scales(wf: torch.Tensor, default_exp: int) -> torch.Tensor:
     return torch.exp2(k).to(torch.float16)
 
 
+def nvfp4_initial(wf: torch.Tensor, G: float):
+    """Packed E2M1 codes and E4M3 block-scale codes of a draw (input recipe):
+    per 16-element block the smallest positive E4M3 value v with
+    6 v G >= the block's largest |w| (binary64; code 56 = 1.0 for all-zero
+    blocks, 126 when none), then per element the nearest E2M1 value of
+    w / (v G)."""
+    dev = wf.device
+    n = wf.numel()
+    nb = (n + FP4_BLOCK - 1) // FP4_BLOCK
+    vals = torch.arange(1, 127, dtype=torch.uint8).view(torch.float8_e4m3fn).to(torch.float64).to(dev)
+    pad = torch.zeros(nb * FP4_BLOCK, dtype=torch.float64, device=dev)
+    pad[:n] = wf.to(torch.float64)
+    amax = pad.abs().view(nb, FP4_BLOCK).amax(dim=1)
+    idx = torch.searchsorted(vals, amax / (6.0 * G)).clamp_(max=125)
+    codes_s = torch.where(amax > 0, idx + 1, torch.full_like(idx, 56)).to(torch.uint8)
+    d = vals[codes_s.long() - 1].repeat_interleave(FP4_BLOCK) * G
+    x = pad / d
+    mag = torch.bucketize(x.abs(), torch.tensor(_E2M1_MIDPOINTS, dtype=torch.float64, device=dev))
+    c = (mag + 8 * (x < 0).to(mag.dtype)).to(torch.uint8)[:n]
+    if n % 2:
+        c = torch.cat([c, torch.zeros(1, dtype=torch.uint8, device=dev)])
+    packed = (c[0::2] & 0x0F) | (c[1::2] << 4)
+    return packed, codes_s
+
+
+def nvfp4_tensor_scale(role: str, w_std: float, norm_gain: float) -> float:
+    """Power-of-two tensor scale G putting the block scales of a draw near
+    112 of E4M3's 448 (room for 4x growth): top / (6 * 112), rounded up to a
+    power of two, top = 6 sigma (or the norm gain)."""
+    top = norm_gain if role == "norm" else 6.0 * w_std
+    return 2.0 ** math.ceil(math.log2(top / (6.0 * 112.0)))
+
+
 def fp8_initial_exponent(role: str, w_std: float, norm_gain: float) -> int:
     """Power-of-two exponent the synthetic FP8 weights are first stored with:
     6 sigma (or the norm gain) fits under E4M3's largest finite value 448."""
@@ -289,8 +343,9 @@ class Materialized:
     fp8_exp: Optional[List[int]] = None
     flat: Dict[str, torch.Tensor] = field(default_factory=dict)
     formats: List[str] = field(default_factory=list)
-    bscale: List[Optional[torch.Tensor]] = field(default_factory=list)  # float16 block scales
+    bscale: List[Optional[torch.Tensor]] = field(default_factory=list)  # float16 / E4M3-code block scales
     cc: List[Optional[torch.Tensor]] = field(default_factory=list)      # BF16 compute copies
+    gscale: List[float] = field(default_factory=list)                   # NVFP4 tensor scales (else 0)
 
 
 def _alloc(kind_dtype, numels, offsets, length, device, layout):
@@ -312,21 +367,25 @@ def materialize(wl: Workload, device="cpu", layout="separate", warm_state=False)
     wdt = _TORCH[formats[0]] if formats else torch.bfloat16
     gdt, mdt = _TORCH[wl.grad_dtype], _TORCH[wl.moment_dtype]
     flat = {}
-    if uniform:
+    wbytes = [(n + 1) // 2 if f == "nvfp4" else n for n, f in zip(numels, formats)]
+    if uniform and "nvfp4" not in formats:
         fw, w = _alloc(wdt, numels, offsets, length, device, layout)
-    else:  # weights of different element sizes: one allocation per tensor
-        fw, w = None, [torch.zeros(n, dtype=_TORCH[f], device=device) for n, f in zip(numels, formats)]
+    else:  # weights of different element sizes (or packed): one allocation per tensor
+        fw, w = None, [torch.zeros(b, dtype=_TORCH[f], device=device) for b, f in zip(wbytes, formats)]
     fg, g = _alloc(gdt, numels, offsets, length, device, layout)
     fm, m = _alloc(mdt, numels, offsets, length, device, layout)
     fv, v = _alloc(mdt, numels, offsets, length, device, layout)
     fve, ve = _alloc(mdt, numels, offsets, length, device, layout)
     if layout == "flat":
         flat = {"g": fg, "m": fm, "v": fv, "ve": fve}
-        if uniform:
+        if fw is not None:
             flat["w"] = fw
     fp8_exp = [] if "e4m3" in formats else None
-    bscale = [torch.ones((n + BLOCK - 1) // BLOCK, dtype=torch.float16, device=device) if f == "e4m3_b32" else None
+    bscale = [torch.ones((n + BLOCK - 1) // BLOCK, dtype=torch.float16, device=device) if f == "e4m3_b32" else
+              torch.zeros((n + FP4_BLOCK - 1) // FP4_BLOCK, dtype=torch.uint8, device=device) if f == "nvfp4" else None
               for n, f in zip(numels, formats)]
+    gscale = [nvfp4_tensor_scale(s.role, wl.w_std, wl.norm_gain) if f == "nvfp4" else 0.0
+              for s, f in zip(wl.specs, formats)]
     cc = [torch.zeros(n, dtype=torch.bfloat16, device=device) if wl.compute_copy and f != "bf16" else None
           for n, f in zip(numels, formats)]
 
@@ -354,6 +413,10 @@ def materialize(wl: Workload, device="cpu", layout="separate", warm_state=False)
             e0 = fp8_exp[-1]
             q = (wf * (2.0 ** -e0)).clamp_(-448.0, 448.0).to(torch.float8_e4m3fn)
             w[k].copy_(q.view(torch.uint8))
+        elif fmt == "nvfp4":
+            packed, sc = nvfp4_initial(wf, gscale[k])
+            w[k].copy_(packed)
+            bscale[k].copy_(sc)
         elif fmt == "e4m3_b32":
             sc = block_initial_scales(wf, fp8_initial_exponent(spec.role, wl.w_std, wl.norm_gain))
             bscale[k].copy_(sc)
@@ -385,7 +448,7 @@ def materialize(wl: Workload, device="cpu", layout="separate", warm_state=False)
             m[k].copy_(mf.to(mdt))
             v[k].copy_(vf.to(mdt))
             ve[k].copy_(vef.to(mdt))
-    return Materialized(wl, offsets, length, w, g, m, v, ve, fp8_exp, flat, formats, bscale, cc)
+    return Materialized(wl, offsets, length, w, g, m, v, ve, fp8_exp, flat, formats, bscale, cc, gscale)
 
 
 def to_numpy_bits(t: torch.Tensor):
