@@ -105,6 +105,8 @@ def lib() -> ctypes.CDLL:
         L.orc_step_nvfp4.argtypes = [i64, i64, i32, i32, P, P, ctypes.c_float, P, P, P, P, P, i64]
         L.orc_step_nvfp4.restype = i32
         L.orc_dequant_nvfp4_bf16.argtypes = [i64, P, P, ctypes.c_float, P]
+        L.orc_tree_sum.argtypes = [i64, P]; L.orc_tree_sum.restype = ctypes.c_double
+        L.orc_toy_step.argtypes = [P, i64, P, P, i64]; L.orc_toy_step.restype = ctypes.c_double
         _LIB = L
     return _LIB
 
@@ -304,6 +306,38 @@ def dequant_nvfp4_bf16(n: int, q, bscale, G: float) -> np.ndarray:
     out = np.zeros(n, np.uint16)
     lib().orc_dequant_nvfp4_bf16(n, _p(q), _p(bs), ctypes.c_float(G), _p(out))
     return out
+
+
+class ToyConfig(ctypes.Structure):
+    _fields_ = [("mode", ctypes.c_int32), ("split", ctypes.c_int32), ("batch", ctypes.c_int32),
+                ("pad", ctypes.c_int32), ("lr_add", ctypes.c_float), ("lr_mul", ctypes.c_float),
+                ("rmax", ctypes.c_float), ("tau", ctypes.c_float), ("c_lo", ctypes.c_float),
+                ("c_hi", ctypes.c_float), ("seed", ctypes.c_uint64)]
+
+
+TOY_MODES = {"additive": 0, "multiplicative": 1, "combined": 2}
+
+
+def toy_config(mode, *, lr_add=0.0, lr_mul=0.0, batch=65536, c_lo=1.0, c_hi=None, split=False, seed=0,
+               rmax=0.75, tau=1e-8) -> ToyConfig:
+    return ToyConfig(TOY_MODES[mode] if isinstance(mode, str) else mode, int(split), batch, 0, lr_add, lr_mul,
+                     rmax, tau, c_lo, c_lo if c_hi is None else c_hi, seed)
+
+
+def tree_sum(x) -> float:
+    x = _c(x, np.float64)
+    return float(lib().orc_tree_sum(x.size, _p(x)))
+
+
+def toy_step(cfg: ToyConfig, w, wstar, t: int) -> float:
+    """One toy-diagnostic step: w (uint16 BF16 bits) updated in place; returns
+    the minibatch loss before the update."""
+    assert w.dtype == np.uint16 and w.flags.c_contiguous
+    n, B = w.size, cfg.batch
+    if n & (n - 1) or B & (B - 1) or B < 64 or cfg.mode not in (0, 1, 2) or cfg.split not in (0, 1):
+        raise ValueError("invalid arguments")
+    ws = _c(wstar, np.float32)
+    return float(lib().orc_toy_step(ctypes.byref(cfg), n, _p(w), _p(ws), t))
 
 
 def global_offsets(numels) -> List[int]:

@@ -44,6 +44,7 @@
 #include "mpadam_oracle.h"
 
 #include <math.h>
+#include <stdlib.h>
 #include <string.h>
 
 static float f_from_bits(uint32_t b) { float f; memcpy(&f, &b, sizeof f); return f; }
@@ -556,6 +557,84 @@ void orc_dequant_nvfp4_bf16(int64_t n, const uint8_t* q, const uint8_t* bscale, 
     const float d = orc_e4m3_decode(bscale[k / ORC_FP4_BLOCK]) * G;
     out[k] = orc_bf16_rne(orc_e2m1_decode(nvfp4_get(q, k)) * d);
   }
+}
+
+/* ------------------------------------------------------------------------ */
+/* BF16-stored matrix fitting (the toy diagnostic of Sec. 5.1; its appendix  */
+/* gives the loss c ||W - W*||^4 estimated on sampled entries, the three     */
+/* update rules without moments, r_max = 0.75, tau = 1e-8, and the regimes). */
+/* ------------------------------------------------------------------------ */
+double orc_tree_sum(int64_t n, const double* x) {
+  double* v = (double*)malloc(sizeof(double) * (size_t)(n > 0 ? n : 1));
+  if (!v) return NAN;
+  memcpy(v, x, sizeof(double) * (size_t)n);
+  for (int64_t len = n; len > 1; len /= 2)
+    for (int64_t i = 0; i < len / 2; ++i) v[i] = v[2 * i] + v[2 * i + 1];
+  double r = n > 0 ? v[0] : 0.0;
+  free(v);
+  return r;
+}
+
+static int is_pow2(int64_t x) { return x > 0 && (x & (x - 1)) == 0; }
+
+double orc_toy_step(const orc_toy_config* c, int64_t n, uint16_t* w, const float* wstar, int64_t t) {
+  if (!c || !w || !wstar || !is_pow2(n) || !is_pow2(c->batch) || c->batch < 64) return NAN;
+  if (c->mode < 0 || c->mode > 2 || (c->split != 0 && c->split != 1)) return NAN;
+  if (c->split && n < 2) return NAN;
+  const int64_t B = c->batch, halves = c->split ? 2 : 1, Bh = B / halves, range = n / halves;
+  int64_t* idx = (int64_t*)malloc(sizeof(int64_t) * (size_t)B);
+  float* r = (float*)malloc(sizeof(float) * (size_t)B);
+  double* sq = (double*)malloc(sizeof(double) * (size_t)Bh);
+  int32_t* cnt = (int32_t*)calloc((size_t)n, sizeof(int32_t));
+  int64_t* first = (int64_t*)calloc((size_t)n, sizeof(int64_t));   /* first sample + 1, 0 = none */
+  if (!idx || !r || !sq || !cnt || !first) { free(idx); free(r); free(sq); free(cnt); free(first); return NAN; }
+
+  /* sample with replacement; residuals of the stored weights */
+  for (int64_t s = 0; s < B; ++s) {
+    const int64_t h = c->split ? s / Bh : 0;
+    const uint32_t lane = orc_rng_lane(c->seed, (uint64_t)t, (uint64_t)s, ORC_E4M3);
+    idx[s] = h * range + (int64_t)((uint64_t)lane & (uint64_t)(range - 1));
+    r[s] = orc_bf16_decode(w[idx[s]]) - wstar[idx[s]];
+  }
+  /* loss and gradient scale per half: M = mean r^2, L = c M^2, dL/dr_s = 4 c M r_s / B_h */
+  double loss = 0.0;
+  float alpha[2] = {0.0f, 0.0f};
+  for (int64_t h = 0; h < halves; ++h) {
+    for (int64_t i = 0; i < Bh; ++i) sq[i] = (double)r[h * Bh + i] * (double)r[h * Bh + i];
+    const double M = orc_tree_sum(Bh, sq) / (double)Bh;
+    const double ch = (double)(h == 0 ? c->c_lo : c->c_hi);
+    loss += ch * M * M;
+    alpha[h] = (float)(((4.0 * ch) * M) / (double)Bh);
+  }
+  /* hits per entry; the first sample of an entry applies its update */
+  for (int64_t s = 0; s < B; ++s) {
+    cnt[idx[s]] += 1;
+    if (first[idx[s]] == 0) first[idx[s]] = s + 1;
+  }
+  const float ln2 = (float)0.693147180559945309417232121458;
+  for (int64_t s = 0; s < B; ++s) {
+    const int64_t j = idx[s];
+    if (first[j] != s + 1) continue;
+    const int64_t h = c->split ? s / Bh : 0;
+    const float x = alpha[h] * r[s];
+    float g = x;
+    for (int32_t k = 1; k < cnt[j]; ++k) g = g + x;
+    const float wf = orc_bf16_decode(w[j]);
+    const float ua = -c->lr_add * g;
+    const float ge = (ln2 * wf) * g;
+    const float ut = -c->lr_mul * ge;
+    const float rho = fabsf(wf) > c->tau ? fabsf(wf) : c->tau;
+    float um = ut / rho;
+    if (um > c->rmax) um = c->rmax;
+    if (um < -c->rmax) um = -c->rmax;
+    float wn;
+    if (c->mode == 0) wn = wf + ua;
+    else if (c->mode == 1) wn = fmaf(wf, um, wf);
+    else wn = fmaf(wf, um, wf) + ua;
+    w[j] = orc_bf16_rne(wn);
+  }
+  free(idx); free(r); free(sq); free(cnt); free(first);
+  return loss;
 }
 
 /* ------------------------------------------------------------------------ */

@@ -146,6 +146,35 @@ int32_t orc_step_nvfp4(int64_t n, int64_t gidx0, int32_t gdt, int32_t mdt, uint8
 /* BF16 compute copy of NVFP4 weights: bf16(q_j * d_b) with d_b as above. */
 void orc_dequant_nvfp4_bf16(int64_t n, const uint8_t* q, const uint8_t* bscale, float G, uint16_t* out);
 
+/* BF16-stored matrix-fitting diagnostic (the toy diagnostic of Sec. 5.1 and
+ * its appendix).  One step: B entries of W are sampled uniformly with
+ * replacement (sample s takes the 32-bit random lane s of step t, as E4M3
+ * storage does, masked to the index range); the minibatch loss is
+ * c (mean of the sampled squared residuals)^2 -- per half when split (the
+ * mixed-scales regime: entries [0, n/2) and [n/2, n) are separate problems
+ * with B/2 samples each); the gradient of an entry hit k times is its
+ * contribution alpha r added k times, alpha = 4 c M / B_h; the update is
+ * the additive, multiplicative or combined step without moments, rounded to
+ * BF16 (nearest-even).  Means are perfect binary trees of binary64 sums
+ * over adjacent samples. */
+typedef struct {
+  int32_t mode;      /* 0 additive, 1 multiplicative, 2 combined (eta_a = lr_add, eta_m = lr_mul) */
+  int32_t split;     /* 1: the two halves are separate sub-problems */
+  int32_t batch;     /* B: a power of two, >= 64 */
+  int32_t pad;
+  float lr_add, lr_mul;
+  float rmax, tau;   /* clip of u_m and floor of rho */
+  float c_lo, c_hi;  /* loss constant of the first / second half (c_lo alone when split = 0) */
+  uint64_t seed;
+} orc_toy_config;
+
+/* Perfect binary tree of binary64 sums over adjacent pairs (n a power of two). */
+double orc_tree_sum(int64_t n, const double* x);
+
+/* One step on W (n BF16 entries, n a power of two), updated in place;
+ * returns the minibatch loss before the update, or NaN on bad arguments. */
+double orc_toy_step(const orc_toy_config* c, int64_t n, uint16_t* w, const float* wstar, int64_t t);
+
 /* Array forms of the scalar functions (plain loops), for the tests. */
 void orc_bf16_rne_n(int64_t n, const float* x, uint16_t* out);
 void orc_bf16_sr_n(int64_t n, const float* x, const uint32_t* r16, uint16_t* out);

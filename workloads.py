@@ -451,6 +451,49 @@ def materialize(wl: Workload, device="cpu", layout="separate", warm_state=False)
     return Materialized(wl, offsets, length, w, g, m, v, ve, fp8_exp, flat, formats, bscale, cc, gscale)
 
 
+# ---------------------------------------------------------------------------
+# The BF16-stored matrix-fitting diagnostic (the toy diagnostic of Sec. 5.1
+# and its appendix): W is n x n (stored flat), five regimes
+# ---------------------------------------------------------------------------
+TOY_N = 4096
+TOY_REGIMES = ("sign_flip", "zero_revival", "small", "large", "mixed")
+
+
+@dataclass
+class ToyProblem:
+    regime: str
+    w0: torch.Tensor       # BF16 initial weights (flat, n*n)
+    wstar: torch.Tensor    # binary32 targets (flat)
+    c_lo: float
+    c_hi: float
+    split: bool            # the two halves are separate sub-problems (mixed scales)
+
+
+def toy_problem(regime: str, n: int = TOY_N, seed: int = 0, device="cpu") -> ToyProblem:
+    """Targets and initial weights of one regime (the appendix's recipes):
+    sign flip (w* = +-1, w0 = -w*, c = 1); zero revival (w* = +-1, w0 = 0,
+    c = 1); small weights (w* = 1e-4 z, w0 = 0, c = 1e8); large weights
+    (w* = 900 max(|z|, 1/900), w0 = 100, c = 1e-7); mixed scales (the first
+    half small, the second half large, each with its own c)."""
+    N = n * n
+    g = _gen(device, seed, 0, 7000 + TOY_REGIMES.index(regime))
+    if regime in ("sign_flip", "zero_revival"):
+        ws = torch.randint(0, 2, (N,), generator=g, device=device).to(torch.float32) * 2 - 1
+        w0 = -ws if regime == "sign_flip" else torch.zeros(N, device=device)
+        return ToyProblem(regime, w0.to(torch.bfloat16), ws, 1.0, 1.0, False)
+    z = torch.randn(N, generator=g, dtype=torch.float32, device=device)
+    small = 1e-4 * z
+    large = 900.0 * torch.clamp(z.abs(), min=1.0 / 900.0)
+    if regime == "small":
+        return ToyProblem(regime, torch.zeros(N, dtype=torch.bfloat16, device=device), small, 1e8, 1e8, False)
+    if regime == "large":
+        return ToyProblem(regime, torch.full((N,), 100.0, device=device).to(torch.bfloat16), large, 1e-7, 1e-7, False)
+    half = N // 2
+    ws = torch.cat([small[:half], large[half:]])
+    w0 = torch.cat([torch.zeros(half, device=device), torch.full((N - half,), 100.0, device=device)])
+    return ToyProblem(regime, w0.to(torch.bfloat16), ws, 1e8, 1e-7, True)
+
+
 def to_numpy_bits(t: torch.Tensor):
     """Host numpy view: float32 stays float32, bfloat16 and float16 become
     uint16 bits, uint8 (E4M3 codes) stays uint8."""
