@@ -311,6 +311,42 @@ def host_link_ms(h_src, d_dst, h_dst, d_src, stream, reps: int = 3) -> float:
     return best
 
 
+def run_toy(steps: int):
+    """The BF16-stored matrix-fitting diagnostic: every regime with every
+    update rule for `steps` steps at n = 4096, B = 65536.  Reports the mean
+    device time per step (three launches) and, per run, the mean loss of the
+    last 64 steps over that of the first 4 (lower is better)."""
+    import torch
+    import workloads as W
+    from paper_2607_10611_gb300.toy import ToyDiagnostic
+    stream = torch.cuda.current_stream()
+    out, total_ms = {}, 0.0
+    for regime in W.TOY_REGIMES:
+        p = W.toy_problem(regime, device="cuda", seed=0)
+        out[regime] = {}
+        for mode in ("additive", "multiplicative", "combined"):
+            lr = W.TOY_LR[mode][regime]
+            w = p.w0.clone()
+            d = ToyDiagnostic(w, p.wstar, mode=mode, batch=65536, c_lo=p.c_lo, c_hi=p.c_hi, split=p.split, seed=1,
+                              lr_add=lr if mode != "multiplicative" else 0.0,
+                              lr_mul=lr if mode != "additive" else 0.0)
+            losses = torch.zeros(steps, dtype=torch.float64, device="cuda")
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            for t in range(1, steps + 1):
+                d.step(t, loss_out=losses[t - 1:t])
+            e1.record(stream)
+            torch.cuda.synchronize()
+            total_ms += e0.elapsed_time(e1)
+            L = losses.cpu().numpy()
+            out[regime][mode] = {"lr": lr, "loss_ratio": float(L[-64:].mean() / L[:4].mean()),
+                                 "final_loss": float(L[-64:].mean())}
+            d.close()
+            del w
+    return {"n": W.TOY_N, "batch": 65536, "steps_per_run": steps, "runs": 15,
+            "us_per_step": 1e3 * total_ms / (15 * steps), "launches_per_step": 3, "regimes": out}
+
+
 def max_over_ranks(ms: float, device: str) -> float:
     """The slowest rank's timed-region length (every rank gets it)."""
     import torch
@@ -364,6 +400,7 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--e2e-steps", type=int, default=5)
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    ap.add_argument("--toy-steps", type=int, default=2048, help="matrix-fitting diagnostic steps per run (0 skips)")
     ap.add_argument("--rounding", default=None, choices=["nearest", "stochastic"],
                     help="override the workload's weight rounding")
     ap.add_argument("--max-params", type=int, default=0,
@@ -431,6 +468,7 @@ def main():
             s2 = summarize(wl2, r2, 1, peak, peak_kind)
             s2["clocks"] = sampler.summary(*r2["wall"]) if sampler else None
             secondary.append(s2)
+    toy = run_toy(args.toy_steps) if (args.toy_steps and rank == 0 and world == 1) else None
     if sampler:
         sampler.stop()
     if rank != 0:
@@ -463,6 +501,7 @@ def main():
         "gpu_launches": args.steps * res["launches_per_step"],
         "clocks": clocks,
         "secondary": secondary,
+        "toy": toy,
     }
     print(json.dumps(line), flush=True)
     if world > 1:

@@ -313,6 +313,56 @@ int32_t mpadam_step_noalloc(const mpadam_tensor* tensors, int32_t n, const void*
                             const mpadam_config* cfg, int32_t* fp8_exp, uint32_t* fp8_amax,
                             int64_t step, struct CUstream_st* stream);
 
+/* ------------------------------------------------------------------------
+ * BF16-stored matrix-fitting diagnostic (the toy diagnostic of Sec. 5.1 and
+ * its appendix): minimise c ||W - W*||_F^4 over W stored in BF16, with the
+ * additive, multiplicative or combined step and no moments, to isolate how
+ * each update survives BF16 storage.  One step samples `batch` entries
+ * uniformly with replacement (sample s takes the 32-bit random lane s of
+ * step t: word s mod 4 of Philox4x32-10 block s div 4 with counter (block,
+ * t) and key `seed`, masked to the index range); the minibatch loss is
+ * c (mean of the sampled squared residuals)^2, the mean a perfect binary
+ * tree of binary64 sums over adjacent samples; the gradient of an entry hit
+ * k times is its contribution 4 c M r / B added k times (binary32); the
+ * entry then becomes bf16(w + w u_m + u_a) (nearest-even; u_a = -eta_a g,
+ * u_m = clip(-eta_m ((ln 2) w) g / max(|w|, tau), +-rmax), the additive
+ * step alone in mode 0, the multiplicative alone in mode 1).  With split,
+ * entries [0, n/2) and [n/2, n) are separate problems (c_lo, c_hi; batch/2
+ * samples each; the loss is the sum) -- the mixed-scales regime.
+ * ------------------------------------------------------------------------ */
+typedef enum { MPADAM_TOY_ADDITIVE = 0, MPADAM_TOY_MULTIPLICATIVE = 1, MPADAM_TOY_COMBINED = 2 } mpadam_toy_mode;
+
+typedef struct {
+  int32_t mode;      /* mpadam_toy_mode */
+  int32_t split;     /* 0 or 1 */
+  int32_t batch;     /* a power of two; batch (per half) >= 32 */
+  int32_t reserved;  /* must be 0 */
+  float lr_add;      /* eta_a (finite, >= 0) */
+  float lr_mul;      /* eta_m (finite, >= 0) */
+  float rmax;        /* clip of u_m (the paper: 0.75) */
+  float tau;         /* floor of rho (the paper: 1e-8), > 0 */
+  float c_lo, c_hi;  /* loss constants (c_lo alone when split = 0) */
+  uint64_t seed;
+} mpadam_toy_config;
+
+typedef struct mpadam_toy_state mpadam_toy_state;
+
+/* Set up the diagnostic for n entries (a power of two, 64 <= n <= 2^30):
+ * validates cfg and allocates (and zeroes) two int32[n] scratch arrays and
+ * the per-sample buffers, on the current device.  Errors: EINVAL, EALLOC,
+ * ECUDA.  On error *out is NULL. */
+int32_t mpadam_toy_create(int64_t n, const mpadam_toy_config* cfg, mpadam_toy_state** out);
+
+/* One step t (>= 1) on w (device, n BF16 bit patterns, updated in place)
+ * towards wstar (device, n binary32 targets), asynchronously on `stream`.
+ * loss_out: device double receiving the minibatch loss of this step (before
+ * the update), or NULL.  Three kernel launches.  Errors: EINVAL, ECUDA. */
+int32_t mpadam_toy_step(mpadam_toy_state* s, uint16_t* w, const float* wstar, int64_t step, double* loss_out,
+                        struct CUstream_st* stream);
+
+/* Frees the scratch (synchronises the device first).  NULL is a no-op. */
+int32_t mpadam_toy_destroy(mpadam_toy_state* s);
+
 #ifdef __cplusplus
 }
 #endif

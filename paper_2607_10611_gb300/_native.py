@@ -22,7 +22,8 @@ ROUNDING = {"nearest": MPADAM_ROUND_NEAREST, "stochastic": MPADAM_ROUND_STOCHAST
 
 EXPORTED = ["mpadam_create", "mpadam_create_ex", "mpadam_fp8_init", "mpadam_step", "mpadam_step_host",
             "mpadam_destroy", "mpadam_last_error", "mpadam_global_offset", "mpadam_global_length", "mpadam_set_grid",
-            "mpadam_launch_info", "mpadam_rng_lanes", "mpadam_step_noalloc", "mpadam_device_status"]
+            "mpadam_launch_info", "mpadam_rng_lanes", "mpadam_step_noalloc", "mpadam_device_status",
+            "mpadam_toy_create", "mpadam_toy_step", "mpadam_toy_destroy"]
 
 
 class MPAdamError(RuntimeError):
@@ -55,6 +56,16 @@ class mpadam_config(ctypes.Structure):
         ("weight_dtype", ctypes.c_int32), ("grad_dtype", ctypes.c_int32),
         ("moment_dtype", ctypes.c_int32), ("reserved", ctypes.c_int32),
     ]
+
+
+class mpadam_toy_config(ctypes.Structure):
+    _fields_ = [("mode", ctypes.c_int32), ("split", ctypes.c_int32), ("batch", ctypes.c_int32),
+                ("reserved", ctypes.c_int32), ("lr_add", ctypes.c_float), ("lr_mul", ctypes.c_float),
+                ("rmax", ctypes.c_float), ("tau", ctypes.c_float), ("c_lo", ctypes.c_float),
+                ("c_hi", ctypes.c_float), ("seed", ctypes.c_uint64)]
+
+
+TOY_MODES = {"additive": 0, "multiplicative": 1, "combined": 2}
 
 
 CONFIG_DEFAULTS = dict(lr_add=1e-3, lr_mul=1e-3, beta1=0.9, beta2=0.999, eps=1e-8, tau=1e-8,
@@ -102,6 +113,9 @@ def lib() -> ctypes.CDLL:
             "mpadam_rng_lanes": [u64, i64, i32, i64, i64, P, P],
             "mpadam_step_noalloc": [P, i32, P, P, P, P, i64, P],
             "mpadam_device_status": [P, P],
+            "mpadam_toy_create": [i64, P, P],
+            "mpadam_toy_step": [P, P, P, i64, P, P],
+            "mpadam_toy_destroy": [P],
         }
         for name, args in sig.items():
             f = getattr(L, name)
@@ -217,3 +231,17 @@ def mpadam_step_noalloc(tensors: Sequence[tuple], grads: Sequence[int], cfg: mpa
         arr[i] = mpadam_tensor(w, m, v, ve, n)
     _check(lib().mpadam_step_noalloc(arr, len(tensors), _ptr_array(grads), ctypes.byref(cfg),
                                      fp8_exp or None, fp8_amax or None, step, stream or None))
+
+
+def mpadam_toy_create(n: int, cfg: mpadam_toy_config) -> int:
+    out = ctypes.c_void_p()
+    _check(lib().mpadam_toy_create(n, ctypes.byref(cfg), ctypes.byref(out)))
+    return out.value
+
+
+def mpadam_toy_step(state: int, w: int, wstar: int, step: int, loss_out: int = 0, stream: int = 0) -> None:
+    _check(lib().mpadam_toy_step(state, w, wstar, step, loss_out or None, stream or None))
+
+
+def mpadam_toy_destroy(state: int) -> None:
+    _check(lib().mpadam_toy_destroy(state))

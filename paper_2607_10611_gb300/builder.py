@@ -18,8 +18,8 @@ INCLUDE = ROOT / "include"
 OUT_DIR = PKG / "_build"
 LIB = OUT_DIR / "libmpadam.so"
 
-SOURCES = ["mpadam_api.cu", "step_bf16.cu", "step_e4m3.cu", "step_e4m3b.cu", "step_nvfp4.cu"]
-HEADERS = ["step_args.h", "step_kernel.cuh"]
+SOURCES = ["mpadam_api.cu", "step_bf16.cu", "step_e4m3.cu", "step_e4m3b.cu", "step_nvfp4.cu", "toy.cu"]
+HEADERS = ["step_args.h", "step_kernel.cuh", "toy.h"]
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ARCH + [

@@ -17,6 +17,7 @@
 #include "mpadam.h"
 #include "step_args.h"
 #include "step_kernel.cuh"
+#include "toy.h"
 
 using mpadam::StepArgs;
 using mpadam::StepScalars;
@@ -1143,5 +1144,95 @@ extern "C" int32_t mpadam_step_noalloc(const mpadam_tensor* tensors, int32_t n, 
   void* params[] = {&a};
   e = cudaLaunchKernel(kernel, dim3(grid), dim3(mpadam::kThreads), params, (size_t)geo.dyn_smem, stream);
   if (e != cudaSuccess) return cuda_fail(e, "launch of the step kernel");
+  return MPADAM_OK;
+}
+
+// ---------------------------------------------------------------------------
+// Matrix-fitting diagnostic (kernels in toy.cu)
+// ---------------------------------------------------------------------------
+struct mpadam_toy_state {
+  mpadam::ToyArgs a{};
+  int device = 0;
+};
+
+extern "C" int32_t mpadam_toy_create(int64_t n, const mpadam_toy_config* cfg, mpadam_toy_state** out) {
+  if (!out) return fail(MPADAM_EINVAL, "out is NULL");
+  *out = nullptr;
+  if (!cfg) return fail(MPADAM_EINVAL, "config is NULL");
+  auto pow2 = [](int64_t x) { return x > 0 && (x & (x - 1)) == 0; };
+  if (!pow2(n) || n < 64 || n > (int64_t(1) << 30)) return fail(MPADAM_EINVAL, "n must be a power of two in [64, 2^30]");
+  if (cfg->mode < 0 || cfg->mode > 2) return fail(MPADAM_EINVAL, "mode must be 0, 1 or 2");
+  if (cfg->split != 0 && cfg->split != 1) return fail(MPADAM_EINVAL, "split must be 0 or 1");
+  if (cfg->reserved != 0) return fail(MPADAM_EINVAL, "reserved must be 0");
+  const int64_t halves = cfg->split ? 2 : 1;
+  if (!pow2(cfg->batch) || cfg->batch / halves < 32 || cfg->batch > (1 << 26))
+    return fail(MPADAM_EINVAL, "batch must be a power of two with at least 32 samples per problem (at most 2^26)");
+  auto fin_nonneg = [](float x) { return std::isfinite(x) && x >= 0.0f; };
+  if (!fin_nonneg(cfg->lr_add) || !fin_nonneg(cfg->lr_mul)) return fail(MPADAM_EINVAL, "learning rates must be finite, >= 0");
+  if (!fin_nonneg(cfg->rmax) || !(std::isfinite(cfg->tau) && cfg->tau > 0.0f))
+    return fail(MPADAM_EINVAL, "rmax must be finite >= 0 and tau finite > 0");
+  if (!std::isfinite(cfg->c_lo) || !std::isfinite(cfg->c_hi)) return fail(MPADAM_EINVAL, "c_lo, c_hi must be finite");
+  mpadam_toy_state* st = new (std::nothrow) mpadam_toy_state();
+  if (!st) return fail(MPADAM_EALLOC, "host allocation failed");
+  mpadam::ToyArgs& a = st->a;
+  cudaError_t e = cudaGetDevice(&st->device);
+  if (e != cudaSuccess) { delete st; return cuda_fail(e, "cudaGetDevice"); }
+  const size_t B = (size_t)cfg->batch;
+  if (cudaMalloc(&a.cnt, sizeof(int32_t) * n) != cudaSuccess || cudaMalloc(&a.first, sizeof(int32_t) * n) != cudaSuccess ||
+      cudaMalloc(&a.idx, sizeof(int32_t) * B) != cudaSuccess || cudaMalloc(&a.res, sizeof(float) * B) != cudaSuccess ||
+      cudaMalloc(&a.sq, sizeof(double) * B) != cudaSuccess || cudaMalloc(&a.alpha, sizeof(float) * 2) != cudaSuccess ||
+      cudaMalloc(&a.loss_h, sizeof(double) * 2) != cudaSuccess) {
+    mpadam_toy_destroy(st);
+    return fail(MPADAM_EALLOC, "allocation of the diagnostic's scratch failed");
+  }
+  if ((e = cudaMemset(a.cnt, 0, sizeof(int32_t) * n)) != cudaSuccess ||
+      (e = cudaMemset(a.first, 0, sizeof(int32_t) * n)) != cudaSuccess ||
+      (e = cudaDeviceSynchronize()) != cudaSuccess) {
+    mpadam_toy_destroy(st);
+    return cuda_fail(e, "clearing the diagnostic's scratch");
+  }
+  a.n = n;
+  a.batch = cfg->batch;
+  a.mode = cfg->mode;
+  a.split = cfg->split;
+  a.lr_add = cfg->lr_add;
+  a.lr_mul = cfg->lr_mul;
+  a.rmax = cfg->rmax;
+  a.tau = cfg->tau;
+  a.c_lo = cfg->c_lo;
+  a.c_hi = cfg->split ? cfg->c_hi : cfg->c_lo;
+  round_keys(cfg->seed, a.rk0, a.rk1);
+  *out = st;
+  return MPADAM_OK;
+}
+
+extern "C" int32_t mpadam_toy_step(mpadam_toy_state* s, uint16_t* w, const float* wstar, int64_t step,
+                                   double* loss_out, cudaStream_t stream) {
+  if (!s) return fail(MPADAM_EINVAL, "state is NULL");
+  if (!w || !wstar || !is_aligned(w, 2) || !is_aligned(wstar, 4)) return fail(MPADAM_EINVAL, "w / wstar NULL or misaligned");
+  if (loss_out && !is_aligned(loss_out, 8)) return fail(MPADAM_EINVAL, "loss_out misaligned");
+  if (step < 1) return fail(MPADAM_EINVAL, "step must be >= 1");
+  int dev = -1;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+  if (dev != s->device) return fail(MPADAM_EINVAL, "current device %d differs from the state's device %d", dev, s->device);
+  mpadam::ToyArgs a = s->a;
+  a.w = w;
+  a.wstar = wstar;
+  a.loss_out = loss_out;
+  a.t_lo = (uint32_t)(uint64_t)step;
+  a.t_hi = (uint32_t)((uint64_t)step >> 32);
+  e = mpadam::launch_toy_step(a, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "launch of the diagnostic's kernels");
+  return MPADAM_OK;
+}
+
+extern "C" int32_t mpadam_toy_destroy(mpadam_toy_state* s) {
+  if (!s) return MPADAM_OK;
+  cudaDeviceSynchronize();
+  mpadam::ToyArgs& a = s->a;
+  for (void* p : {(void*)a.cnt, (void*)a.first, (void*)a.idx, (void*)a.res, (void*)a.sq, (void*)a.alpha, (void*)a.loss_h})
+    if (p) cudaFree(p);
+  delete s;
   return MPADAM_OK;
 }

@@ -469,6 +469,20 @@ class ToyProblem:
     split: bool            # the two halves are separate sub-problems (mixed scales)
 
 
+# Learning rates at n = 4096, B = 65536 (eta_a, eta_m; the combined rule
+# shares one value across the five regimes, as in the paper's main figure).
+# Chosen by a sweep over {0.01, 0.03, ..., 30} on n = 128, B = 64 (the same
+# per-step hit rate B / n^2 = 1/256) for 2000 steps, scaled by the batch ratio
+# 1024 (the gradient of one sample scales as 1 / B).
+TOY_LR = {
+    "additive": {"sign_flip": 3072.0, "zero_revival": 30720.0, "small": 10240.0, "large": 30720.0,
+                 "mixed": 10240.0},
+    "multiplicative": {"sign_flip": 30720.0, "zero_revival": 1024.0, "small": 1024.0, "large": 3072.0,
+                       "mixed": 1024.0},
+    "combined": {r: 3072.0 for r in TOY_REGIMES},
+}
+
+
 def toy_problem(regime: str, n: int = TOY_N, seed: int = 0, device="cpu") -> ToyProblem:
     """Targets and initial weights of one regime (the appendix's recipes):
     sign flip (w* = +-1, w0 = -w*, c = 1); zero revival (w* = +-1, w0 = 0,
