@@ -258,9 +258,12 @@ def run_gpu(wl, steps: int, warmup: int, rank: int, e2e_steps: int):
 
     # end to end through the host-buffer entry point (one weight format: flat host buffers)
     if e2e_steps > 0 and "w" in mt.flat:
-        hg = torch.empty(mt.flat["g"].shape, dtype=mt.flat["g"].dtype, pin_memory=True)
+        # page-locked huge-page host buffers (mpadam_host_buffer_alloc)
+        from paper_2607_10611_gb300.optimizer import HostBuffer
+        hg_buf = HostBuffer(mt.flat["g"].numel(), mt.flat["g"].dtype)
+        hw_buf = HostBuffer(mt.flat["w"].numel(), mt.flat["w"].dtype)
+        hg, hw = hg_buf.tensor, hw_buf.tensor
         hg.copy_(mt.flat["g"])
-        hw = torch.empty(mt.flat["w"].shape, dtype=mt.flat["w"].dtype, pin_memory=True)
         hgs = [hg[o:o + x.numel()] for o, x in zip(mt.offsets, mt.g)]
         hws = [hw[o:o + x.numel()] for o, x in zip(mt.offsets, mt.w)]
         opt.step_host(hgs, hws, t)  # warm (allocates the staging buffer)
@@ -279,6 +282,8 @@ def run_gpu(wl, steps: int, warmup: int, rank: int, e2e_steps: int):
         res["d2h"] = sum(x.numel() for x in mt.w) * BYTES[wl.weight_dtype]
         res["link_ms"] = host_link_ms(hg, mt.flat["g"], hw, mt.flat["w"], stream)
         del hg, hw, hgs, hws
+        hg_buf.free()
+        hw_buf.free()
     opt.close()
     del mt, opt
     torch.cuda.synchronize()

@@ -256,6 +256,17 @@ int32_t mpadam_step(mpadam_state* s, const void* const* grads, int64_t step,
 int32_t mpadam_step_host(mpadam_state* s, const void* const* host_grads, void* const* host_w_out,
                          int64_t step, struct CUstream_st* stream);
 
+/* Page-locked host memory for mpadam_step_host's buffers (not from the
+ * paper: a deployment aid).  Allocates `bytes` of anonymous memory advised
+ * for transparent huge pages, touches it (so the pages are resident and
+ * large), and registers it with the CUDA driver (cudaHostRegister).  Copies
+ * from such a buffer keep the host link's full rate: on GB300 (Grace) hosts,
+ * copies from ordinary pinned memory of 64 KB pages measured 4x slower at
+ * times for buffers of several GB, huge-page buffers did not.  Release with
+ * mpadam_host_buffer_free (same size).  Errors: EINVAL, EALLOC, ECUDA. */
+int32_t mpadam_host_buffer_alloc(int64_t bytes, void** out);
+int32_t mpadam_host_buffer_free(void* ptr, int64_t bytes);
+
 /* Frees the library's metadata (synchronises the device first).  NULL is a
  * no-op.  Never touches caller-owned tensors. */
 int32_t mpadam_destroy(mpadam_state* s);

@@ -23,7 +23,8 @@ ROUNDING = {"nearest": MPADAM_ROUND_NEAREST, "stochastic": MPADAM_ROUND_STOCHAST
 EXPORTED = ["mpadam_create", "mpadam_create_ex", "mpadam_fp8_init", "mpadam_step", "mpadam_step_host",
             "mpadam_destroy", "mpadam_last_error", "mpadam_global_offset", "mpadam_global_length", "mpadam_set_grid",
             "mpadam_launch_info", "mpadam_rng_lanes", "mpadam_step_noalloc", "mpadam_device_status",
-            "mpadam_toy_create", "mpadam_toy_step", "mpadam_toy_destroy"]
+            "mpadam_toy_create", "mpadam_toy_step", "mpadam_toy_destroy", "mpadam_host_buffer_alloc",
+            "mpadam_host_buffer_free"]
 
 
 class MPAdamError(RuntimeError):
@@ -116,6 +117,8 @@ def lib() -> ctypes.CDLL:
             "mpadam_toy_create": [i64, P, P],
             "mpadam_toy_step": [P, P, P, i64, P, P],
             "mpadam_toy_destroy": [P],
+            "mpadam_host_buffer_alloc": [i64, P],
+            "mpadam_host_buffer_free": [P, i64],
         }
         for name, args in sig.items():
             f = getattr(L, name)
@@ -245,3 +248,13 @@ def mpadam_toy_step(state: int, w: int, wstar: int, step: int, loss_out: int = 0
 
 def mpadam_toy_destroy(state: int) -> None:
     _check(lib().mpadam_toy_destroy(state))
+
+
+def mpadam_host_buffer_alloc(nbytes: int) -> int:
+    out = ctypes.c_void_p()
+    _check(lib().mpadam_host_buffer_alloc(nbytes, ctypes.byref(out)))
+    return out.value
+
+
+def mpadam_host_buffer_free(ptr: int, nbytes: int) -> None:
+    _check(lib().mpadam_host_buffer_free(ptr, nbytes))

@@ -3,6 +3,7 @@
 // table fills of the allocation-free step).  The fused step kernel itself
 // lives in step_kernel.cuh.
 #include <cuda_runtime.h>
+#include <sys/mman.h>
 
 #include <algorithm>
 #include <cmath>
@@ -1234,5 +1235,36 @@ extern "C" int32_t mpadam_toy_destroy(mpadam_toy_state* s) {
   for (void* p : {(void*)a.cnt, (void*)a.first, (void*)a.idx, (void*)a.res, (void*)a.sq, (void*)a.alpha, (void*)a.loss_h})
     if (p) cudaFree(p);
   delete s;
+  return MPADAM_OK;
+}
+
+// ---------------------------------------------------------------------------
+// Huge-page, page-locked host buffers for mpadam_step_host
+// ---------------------------------------------------------------------------
+extern "C" int32_t mpadam_host_buffer_alloc(int64_t bytes, void** out) {
+  if (!out) return fail(MPADAM_EINVAL, "out is NULL");
+  *out = nullptr;
+  if (bytes <= 0) return fail(MPADAM_EINVAL, "bytes must be > 0");
+  void* p = mmap(nullptr, (size_t)bytes, PROT_READ | PROT_WRITE, MAP_PRIVATE | MAP_ANONYMOUS, -1, 0);
+  if (p == MAP_FAILED) return fail(MPADAM_EALLOC, "mmap of %lld bytes failed", (long long)bytes);
+#ifdef MADV_HUGEPAGE
+  madvise(p, (size_t)bytes, MADV_HUGEPAGE);  // advice only: a kernel without it still gives a valid buffer
+#endif
+  std::memset(p, 0, (size_t)bytes);  // resident before registration
+  cudaError_t e = cudaHostRegister(p, (size_t)bytes, cudaHostRegisterDefault);
+  if (e != cudaSuccess) {
+    munmap(p, (size_t)bytes);
+    return cuda_fail(e, "cudaHostRegister");
+  }
+  *out = p;
+  return MPADAM_OK;
+}
+
+extern "C" int32_t mpadam_host_buffer_free(void* ptr, int64_t bytes) {
+  if (!ptr) return MPADAM_OK;
+  if (bytes <= 0) return fail(MPADAM_EINVAL, "bytes must be > 0");
+  cudaError_t e = cudaHostUnregister(ptr);
+  munmap(ptr, (size_t)bytes);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaHostUnregister");
   return MPADAM_OK;
 }

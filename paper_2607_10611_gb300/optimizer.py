@@ -22,6 +22,32 @@ _STORAGE = {"bf16": torch.bfloat16, "e4m3": torch.uint8, "e4m3_b32": torch.uint8
 _SCALES = {"e4m3_b32": torch.float16, "nvfp4": torch.uint8}
 
 
+class HostBuffer:
+    """Page-locked, huge-page host memory from mpadam_host_buffer_alloc, as a
+    1-D CPU tensor of `dtype` (for mpadam_step_host's gradients and weights)."""
+
+    def __init__(self, numel: int, dtype: torch.dtype):
+        import ctypes
+        import numpy as np
+        itemsize = torch.empty(0, dtype=dtype).element_size()
+        self.nbytes = max(1, numel * itemsize)
+        self.ptr = N.mpadam_host_buffer_alloc(self.nbytes)
+        raw = (ctypes.c_uint8 * self.nbytes).from_address(self.ptr)
+        self.tensor = torch.from_numpy(np.frombuffer(raw, dtype=np.uint8)).view(dtype)[:numel]
+
+    def free(self):
+        if getattr(self, "ptr", None):
+            self.tensor = None
+            N.mpadam_host_buffer_free(self.ptr, self.nbytes)
+            self.ptr = None
+
+    def __del__(self):
+        try:
+            self.free()
+        except Exception:
+            pass
+
+
 class MPAdam:
     def __init__(self, w: Sequence[torch.Tensor], m: Sequence[torch.Tensor], v: Sequence[torch.Tensor],
                  ve: Sequence[torch.Tensor], *, weight_dtype="bf16", grad_dtype: str = "f32",

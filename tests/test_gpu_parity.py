@@ -273,3 +273,29 @@ def test_step_rejects_null_grads_on_gpu():
     with pytest.raises(N.MPAdamError):
         N.mpadam_step(s, [m.data_ptr()], 0)        # step 0
     N.mpadam_destroy(s)
+
+
+def test_step_host_with_huge_page_host_buffers():
+    """mpadam_host_buffer_alloc buffers as the host side of the pipelined
+    host-buffer step: same bits as the device step."""
+    from paper_2607_10611_gb300.optimizer import HostBuffer
+    p = P()
+    wl = W.SMALL["llama_7b"]
+    r1 = p.Run(wl, warm=True, layout="flat")
+    r2 = p.Run(wl, warm=True, layout="flat")
+    bg = HostBuffer(r2.mt.flat["g"].numel(), r2.mt.flat["g"].dtype)
+    bw = HostBuffer(r2.mt.flat["w"].numel(), r2.mt.flat["w"].dtype)
+    try:
+        bg.tensor.copy_(r2.mt.flat["g"])
+        hg = [bg.tensor[o:o + t.numel()] for o, t in zip(r2.mt.offsets, r2.mt.g)]
+        hw = [bw.tensor[o:o + t.numel()] for o, t in zip(r2.mt.offsets, r2.mt.w)]
+        for t in range(1, 4):
+            r1.opt.step(r1.dev["g"], t)
+            r2.opt.step_host(hg, hw, t)
+        torch.cuda.synchronize()
+        for k in range(len(hw)):
+            assert torch.equal(hw[k], r1.dev["w"][k].cpu())
+            assert torch.equal(r2.dev["w"][k], r1.dev["w"][k])
+    finally:
+        r1.close(); r2.close()
+        bg.free(); bw.free()
