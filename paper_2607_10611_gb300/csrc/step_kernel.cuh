@@ -972,14 +972,15 @@ __device__ __forceinline__ float e2m1_value(uint32_t c) {
 // binary32 -> E2M1 code: nearest-even, or stochastic (away from zero iff
 // r < floor(fraction * 2^32)); |x| >= 6 and infinities saturate; NaN -> +0.
 // Branch-free: with the grid spacing sp = 0.5, 1 or 2 of |x|'s binade
-// ([0, 2), [2, 4), [4, 6]), q = |x| / sp is exact, its integer part k and
-// fraction f give the code k + (0, 2 or 4) and the step up.
+// ([0, 2), [2, 4), [4, 6]), q = |x| / sp (a product with the power of two
+// 1 / sp: exact), its integer part k and fraction f give the code
+// k + (0, 2 or 4) and the step up.
 template <bool SR>
 __device__ __forceinline__ uint32_t e2m1_encode(float x, uint32_t r) {
   const float a = fminf(fabsf(x), 6.0f);
-  const float sp = a < 2.0f ? 0.5f : (a < 4.0f ? 1.0f : 2.0f);
+  const float rsp = a < 2.0f ? 2.0f : (a < 4.0f ? 1.0f : 0.5f);
   const uint32_t off = a < 2.0f ? 0u : (a < 4.0f ? 2u : 4u);
-  const float q = __fdiv_rn(a, sp);  // a power-of-two divisor: exact
+  const float q = __fmul_rn(a, rsp);
   const float kf = truncf(q);
   const float f = __fsub_rn(q, kf);  // exact
   const uint32_t k = __float2uint_rz(kf);
@@ -1025,9 +1026,9 @@ __device__ __forceinline__ uint32_t e2m1x8_rn(const float (&x)[8]) {
 // the same code (an end in another binade or sign reports false).
 __device__ __forceinline__ uint32_t e2m1_pair_sr(float xl, float xh, uint32_t r, bool& same) {
   const float al = fminf(fabsf(xl), 6.0f), ah = fminf(fabsf(xh), 6.0f);
-  const float sp = al < 2.0f ? 0.5f : (al < 4.0f ? 1.0f : 2.0f);
+  const float rsp = al < 2.0f ? 2.0f : (al < 4.0f ? 1.0f : 0.5f);
   const uint32_t off = al < 2.0f ? 0u : (al < 4.0f ? 2u : 4u);
-  const float ql = __fdiv_rn(al, sp), qh = __fdiv_rn(ah, sp);  // exact
+  const float ql = __fmul_rn(al, rsp), qh = __fmul_rn(ah, rsp);  // exact (powers of two)
   const float kl = truncf(ql), kh = truncf(qh);
   const uint32_t ul = r < __float2uint_rz(__fmul_rn(__fsub_rn(ql, kl), 4294967296.0f)) ? 1u : 0u;
   const uint32_t uh = r < __float2uint_rz(__fmul_rn(__fsub_rn(qh, kh), 4294967296.0f)) ? 1u : 0u;
@@ -1075,25 +1076,49 @@ __device__ __forceinline__ uint32_t pair_max(uint32_t x) {
   return max(x, __shfl_xor_sync(0xFFFFFFFFu, x, 1));
 }
 
-template <int GD, int MD, bool SR, bool OPT>
+// One element's canonical update recomputed from the stage's original
+// inputs (the stage is kept until the group is done when STAGED): the exact
+// weight of the element's group slot j.
+template <int GD, int MD>
+__device__ __forceinline__ float fp4_exact_from_stage(const StepArgs& a, uint32_t st, int c, int j, float d_old) {
+  constexpr int GS = esize_of(GD), MS = esize_of(MD);
+  const uint32_t word = lds_u32(st + 4 * c);
+  float q[8];
+  e2m1x8_to_f32(word, q);
+  const float w = __fmul_rn(q[j], d_old);
+  auto ld = [&](uint32_t base, int es) -> float {
+    const uint32_t addr = base + static_cast<uint32_t>(kGroup * es * c + es * j);
+    return es == 4 ? __uint_as_float(lds_u32(addr)) : __uint_as_float(lds_u16(addr) << 16);
+  };
+  const float g = ld(st + a.off_g, GS);
+  const float m = ld(st + a.off_m, MS), v = ld(st + a.off_v, MS), ve = ld(st + a.off_ve, MS);
+  return madam_update<false>(a.s, w, g, m, v, ve).wn;
+}
+
+// STAGED: every input of this group is in the stage at `st` (thread c) and
+// the stage is released only after this returns, so the rare exact branch
+// recomputes from there and the new moments are stored right after the
+// update -- fewer values live in registers through the encode.
+template <int GD, int MD, bool SR, bool OPT, bool STAGED>
 __device__ __forceinline__ void finish_fp4(const StepArgs& a, const TensorCtx& x, int64_t e0, int valid,
                                            uint32_t c_old, float (&w)[8], float (&g)[8], float (&m)[8],
-                                           float (&v)[8], float (&ve)[8]) {
+                                           float (&v)[8], float (&ve)[8], uint32_t st, int c) {
   const float G = x.gscale;
+  const float d_old = __fmul_rn(e4m3_value(c_old), G);
   const uint64_t gi = static_cast<uint64_t>(x.d.goff + e0) >> 3;  // global group index (random lanes)
-  uint32_t rnd[8];
-  if (SR) group_random_bits<kNVFP4>(a, gi << 3, rnd);
   const uint32_t vmask = valid >= kGroup ? 0xFFu : (valid > 0 ? (1u << valid) - 1u : 0u);
   uint32_t code[8];
   uint32_t c_new;
   float d;
+  auto exact_wn = [&](int j) -> float {
+    if constexpr (STAGED) return fp4_exact_from_stage<GD, MD>(a, st, c, j, d_old);
+    else return madam_wn_exact(a.s, w[j], g[j], m[j], v[j], ve[j]);
+  };
   if (!OPT && a.s.cert_ok) {
     // Certified path, as for block-scaled E4M3: fast weights and one error
     // bound et; the pair's maximum bounds decide the scale code (exact
     // maximum where they do not); then each element's interval, divided by
-    // d through an approximate reciprocal and widened by 2^-20 relative and
-    // 2^-126 absolute (beyond the approximation's error), is encoded at both
-    // ends.
+    // d through an approximate reciprocal, is encoded at both ends.
     float wf[8];
     float et = 0.0f, am = 0.0f;
     uint32_t bad = 0u;
@@ -1109,6 +1134,7 @@ __device__ __forceinline__ void finish_fp4(const StepArgs& a, const TensorCtx& x
         if ((vmask >> j) & 1u) am = fmaxf(am, fabsf(u.wn));
       }
     }
+    if constexpr (STAGED) put_moments<MD>(x, e0, valid, m, v, ve);
     bad &= vmask;
     const float lo_t = bad ? 0.0f : fmaxf(__fsub_rd(am, et), 0.0f);
     const float hi_t = bad ? INFINITY : __fadd_ru(am, et);
@@ -1125,7 +1151,7 @@ __device__ __forceinline__ void finish_fp4(const StepArgs& a, const TensorCtx& x
 #pragma unroll
         for (int j = 0; j < kGroup; ++j) {
           if ((vmask >> j) & 1u) {
-            const uint32_t bb = __float_as_uint(madam_wn_exact(a.s, w[j], g[j], m[j], v[j], ve[j])) & 0x7FFFFFFFu;
+            const uint32_t bb = __float_as_uint(exact_wn(j)) & 0x7FFFFFFFu;
             if (bb < 0x7F800000u) amx = max(amx, bb);
           }
         }
@@ -1136,30 +1162,30 @@ __device__ __forceinline__ void finish_fp4(const StepArgs& a, const TensorCtx& x
     d = __fmul_rn(e4m3_value(c_new), G);
     uint32_t redo = bad;
     if (d >= 1.1754943508222875e-38f /* 2^-126 */ && d <= 8.507059173023462e+37f /* 2^126 */) {
-      // w' / d bounded through one approximate reciprocal (1 ulp) and a
-      // product (half an ulp): within 2^-22 relative, widened to 2^-20
+      // w' / d for w' in [wf - et, wf + et]: q = wf * inv (inv = rcp.approx(d),
+      // 1 ulp; the product half an ulp) is within 2^-22 |q| of wf / d, and
+      // et / d <= et inv (1 + 2^-22); widened to 2^-20 and 2^-126 absolute.
       float inv;
       asm("rcp.approx.f32 %0, %1;" : "=f"(inv) : "f"(d));
+      const float ei = __fmaf_ru(et, __fmul_ru(inv, 1.0000009536743164f /* 1 + 2^-20 */), 1.1754943508222875e-38f);
+      float xl[8], xh[8];
+#pragma unroll
+      for (int j = 0; j < kGroup; ++j) {
+        const float q = __fmul_rn(wf[j], inv);
+        const float e2 = __fmaf_ru(fabsf(q), 9.5367431640625e-07f /* 2^-20 */, ei);
+        xl[j] = __fsub_rd(q, e2);
+        xh[j] = __fadd_ru(q, e2);
+      }
       if (SR) {
+        uint32_t rnd[8];
+        group_random_bits<kNVFP4>(a, gi << 3, rnd);
 #pragma unroll
         for (int j = 0; j < kGroup; ++j) {
-          const float ql = __fmul_rn(__fsub_rd(wf[j], et), inv);
-          const float qh = __fmul_rn(__fadd_ru(wf[j], et), inv);
-          const float xl = __fsub_rd(ql, __fmaf_ru(fabsf(ql), 9.5367431640625e-07f /* 2^-20 */, 1.1754943508222875e-38f));
-          const float xh = __fadd_ru(qh, __fmaf_ru(fabsf(qh), 9.5367431640625e-07f, 1.1754943508222875e-38f));
           bool same;
-          code[j] = e2m1_pair_sr(xl, xh, rnd[j], same);
+          code[j] = e2m1_pair_sr(xl[j], xh[j], rnd[j], same);
           if (!same) redo |= 1u << j;
         }
       } else {
-        float xl[8], xh[8];
-#pragma unroll
-        for (int j = 0; j < kGroup; ++j) {
-          const float ql = __fmul_rn(__fsub_rd(wf[j], et), inv);
-          const float qh = __fmul_rn(__fadd_ru(wf[j], et), inv);
-          xl[j] = __fsub_rd(ql, __fmaf_ru(fabsf(ql), 9.5367431640625e-07f /* 2^-20 */, 1.1754943508222875e-38f));
-          xh[j] = __fadd_ru(qh, __fmaf_ru(fabsf(qh), 9.5367431640625e-07f, 1.1754943508222875e-38f));
-        }
         const uint32_t pl = e2m1x8_rn(xl), diff = pl ^ e2m1x8_rn(xh);
 #pragma unroll
         for (int j = 0; j < kGroup; ++j) {
@@ -1172,14 +1198,17 @@ __device__ __forceinline__ void finish_fp4(const StepArgs& a, const TensorCtx& x
     }
     redo &= vmask;
     if (redo) {  // rare: the canonical weight of the undecided elements
+      uint32_t rnd[8];
+      if (SR) group_random_bits<kNVFP4>(a, gi << 3, rnd);
 #pragma unroll
       for (int j = 0; j < kGroup; ++j) {
         if ((redo >> j) & 1u) {
-          const float xe = __fdiv_rn(madam_wn_exact(a.s, w[j], g[j], m[j], v[j], ve[j]), d);
+          const float xe = __fdiv_rn(exact_wn(j), d);
           code[j] = e2m1_encode<SR>(xe, SR ? rnd[j] : 0u);
         }
       }
     }
+    if constexpr (!STAGED) put_moments<MD>(x, e0, valid, m, v, ve);
   } else {
     float wn[8];
     uint32_t amx = 0u;
@@ -1192,8 +1221,11 @@ __device__ __forceinline__ void finish_fp4(const StepArgs& a, const TensorCtx& x
     }
     c_new = nvfp4_scale_code(__uint_as_float(pair_max(amx)), G, c_old);
     d = __fmul_rn(e4m3_value(c_new), G);
+    uint32_t rnd[8];
+    if (SR) group_random_bits<kNVFP4>(a, gi << 3, rnd);
 #pragma unroll
     for (int j = 0; j < kGroup; ++j) code[j] = e2m1_encode<SR>(__fdiv_rn(wn[j], d), SR ? rnd[j] : 0u);
+    put_moments<MD>(x, e0, valid, m, v, ve);
   }
   uint32_t packed = 0u;
 #pragma unroll
@@ -1208,7 +1240,6 @@ __device__ __forceinline__ void finish_fp4(const StepArgs& a, const TensorCtx& x
     for (int i = 0; i < 4; ++i) o[i] = bf16x2_rn(__fmul_rn(q[2 * i], d), __fmul_rn(q[2 * i + 1], d));
     put_bf16(o, x.cc, e0, valid, x.vec);
   }
-  put_moments<MD>(x, e0, valid, m, v, ve);
 }
 
 // Eight NVFP4 weights decoded with d: from the stage or global memory as one
@@ -1267,7 +1298,7 @@ __device__ __noinline__ void general_fp4_group(const StepArgs& a, const TensorCt
     get_bf16<false>(v, v_st, st + a.off_v + kGroup * MS * c, x.d.v, e0, valid, x.vec);
     get_bf16<false>(ve, e_st, st + a.off_ve + kGroup * MS * c, x.d.ve, e0, valid, x.vec);
   }
-  finish_fp4<GD, MD, SR, OPT>(a, x, e0, valid, s_old, w, g, m, v, ve);
+  finish_fp4<GD, MD, SR, OPT, false>(a, x, e0, valid, s_old, w, g, m, v, ve, st, c);
 }
 
 // ---------------------------------------------------------------------------
@@ -1429,11 +1460,17 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
         get_bf16<false>(v, true, st + a.off_v + kGroup * MS * c, x.d.v, e0, kGroup, true);
         get_bf16<false>(ve, true, st + a.off_ve + kGroup * MS * c, x.d.ve, e0, kGroup, true);
       }
-      __syncwarp();
-      if (lane == 0) mbar_arrive(smem_addr(&empty_bar[s]));
-      if constexpr (WD == kE4M3B) finish_block<GD, MD, SR, OPT>(a, x, e0, kGroup, h_old, w, g, m, v, ve);
-      else if constexpr (WD == kNVFP4) finish_fp4<GD, MD, SR, OPT>(a, x, e0, kGroup, h_old, w, g, m, v, ve);
-      else finish_group<WD, GD, MD, SR, OPT>(a, x, e0, kGroup, w, g, m, v, ve, amax_bits);
+      if constexpr (WD == kNVFP4) {
+        // the stage stays until the group is done (its exact branch re-reads it)
+        finish_fp4<GD, MD, SR, OPT, true>(a, x, e0, kGroup, h_old, w, g, m, v, ve, st, c);
+        __syncwarp();
+        if (lane == 0) mbar_arrive(smem_addr(&empty_bar[s]));
+      } else {
+        __syncwarp();
+        if (lane == 0) mbar_arrive(smem_addr(&empty_bar[s]));
+        if constexpr (WD == kE4M3B) finish_block<GD, MD, SR, OPT>(a, x, e0, kGroup, h_old, w, g, m, v, ve);
+        else finish_group<WD, GD, MD, SR, OPT>(a, x, e0, kGroup, w, g, m, v, ve, amax_bits);
+      }
       if (++s == S) { s = 0; ++use; }
       continue;
     }
