@@ -346,7 +346,7 @@ typedef enum { MPADAM_TOY_ADDITIVE = 0, MPADAM_TOY_MULTIPLICATIVE = 1, MPADAM_TO
 typedef struct {
   int32_t mode;      /* mpadam_toy_mode */
   int32_t split;     /* 0 or 1 */
-  int32_t batch;     /* a power of two; batch (per half) >= 32 */
+  int32_t batch;     /* a power of two; 32 to 65536 samples per problem (per half when split) */
   int32_t reserved;  /* must be 0 */
   float lr_add;      /* eta_a (finite, >= 0) */
   float lr_mul;      /* eta_m (finite, >= 0) */
@@ -370,6 +370,16 @@ int32_t mpadam_toy_create(int64_t n, const mpadam_toy_config* cfg, mpadam_toy_st
  * the update), or NULL.  Three kernel launches.  Errors: EINVAL, ECUDA. */
 int32_t mpadam_toy_step(mpadam_toy_state* s, uint16_t* w, const float* wstar, int64_t step, double* loss_out,
                         struct CUstream_st* stream);
+
+/* `steps` consecutive steps first_step, first_step + 1, ... on `stream`, as
+ * many mpadam_toy_step calls would give, with the loss of step first_step + i
+ * written to losses[i] (device, double[steps]; or NULL).  The step number
+ * lives in device memory, advanced by the last kernel of each step, so the
+ * steps run as replays of a CUDA graph of 64 steps, captured on an internal
+ * stream at the first call with these w, wstar and losses pointers (the
+ * remainder runs as plain launches).  Errors: EINVAL, ECUDA. */
+int32_t mpadam_toy_run(mpadam_toy_state* s, uint16_t* w, const float* wstar, int64_t first_step, int64_t steps,
+                       double* losses, struct CUstream_st* stream);
 
 /* Frees the scratch (synchronises the device first).  NULL is a no-op. */
 int32_t mpadam_toy_destroy(mpadam_toy_state* s);

@@ -23,7 +23,7 @@ ROUNDING = {"nearest": MPADAM_ROUND_NEAREST, "stochastic": MPADAM_ROUND_STOCHAST
 EXPORTED = ["mpadam_create", "mpadam_create_ex", "mpadam_fp8_init", "mpadam_step", "mpadam_step_host",
             "mpadam_destroy", "mpadam_last_error", "mpadam_global_offset", "mpadam_global_length", "mpadam_set_grid",
             "mpadam_launch_info", "mpadam_rng_lanes", "mpadam_step_noalloc", "mpadam_device_status",
-            "mpadam_toy_create", "mpadam_toy_step", "mpadam_toy_destroy", "mpadam_host_buffer_alloc",
+            "mpadam_toy_create", "mpadam_toy_step", "mpadam_toy_run", "mpadam_toy_destroy", "mpadam_host_buffer_alloc",
             "mpadam_host_buffer_free"]
 
 
@@ -116,6 +116,7 @@ def lib() -> ctypes.CDLL:
             "mpadam_device_status": [P, P],
             "mpadam_toy_create": [i64, P, P],
             "mpadam_toy_step": [P, P, P, i64, P, P],
+            "mpadam_toy_run": [P, P, P, i64, i64, P, P],
             "mpadam_toy_destroy": [P],
             "mpadam_host_buffer_alloc": [i64, P],
             "mpadam_host_buffer_free": [P, i64],
@@ -244,6 +245,11 @@ def mpadam_toy_create(n: int, cfg: mpadam_toy_config) -> int:
 
 def mpadam_toy_step(state: int, w: int, wstar: int, step: int, loss_out: int = 0, stream: int = 0) -> None:
     _check(lib().mpadam_toy_step(state, w, wstar, step, loss_out or None, stream or None))
+
+
+def mpadam_toy_run(state: int, w: int, wstar: int, first_step: int, steps: int, losses: int = 0,
+                   stream: int = 0) -> None:
+    _check(lib().mpadam_toy_run(state, w, wstar, first_step, steps, losses or None, stream or None))
 
 
 def mpadam_toy_destroy(state: int) -> None:

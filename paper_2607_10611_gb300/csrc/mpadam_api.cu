@@ -1154,7 +1154,17 @@ extern "C" int32_t mpadam_step_noalloc(const mpadam_tensor* tensors, int32_t n, 
 struct mpadam_toy_state {
   mpadam::ToyArgs a{};
   int device = 0;
+  int64_t* t_dev = nullptr;           // run mode step counter {t, first t}
+  cudaStream_t cap = nullptr;         // capture stream of the run graph
+  cudaGraphExec_t exec = nullptr;     // kToyGraphSteps steps for the pointers below
+  const void* g_w = nullptr;
+  const void* g_ws = nullptr;
+  const void* g_loss = nullptr;
 };
+
+namespace {
+constexpr int64_t kToyGraphSteps = 64;  // steps per replay of the run graph
+}
 
 extern "C" int32_t mpadam_toy_create(int64_t n, const mpadam_toy_config* cfg, mpadam_toy_state** out) {
   if (!out) return fail(MPADAM_EINVAL, "out is NULL");
@@ -1166,8 +1176,8 @@ extern "C" int32_t mpadam_toy_create(int64_t n, const mpadam_toy_config* cfg, mp
   if (cfg->split != 0 && cfg->split != 1) return fail(MPADAM_EINVAL, "split must be 0 or 1");
   if (cfg->reserved != 0) return fail(MPADAM_EINVAL, "reserved must be 0");
   const int64_t halves = cfg->split ? 2 : 1;
-  if (!pow2(cfg->batch) || cfg->batch / halves < 32 || cfg->batch > (1 << 26))
-    return fail(MPADAM_EINVAL, "batch must be a power of two with at least 32 samples per problem (at most 2^26)");
+  if (!pow2(cfg->batch) || cfg->batch / halves < 32 || cfg->batch / halves > 32 * 2048)
+    return fail(MPADAM_EINVAL, "batch must be a power of two with 32 to 65536 samples per problem");
   auto fin_nonneg = [](float x) { return std::isfinite(x) && x >= 0.0f; };
   if (!fin_nonneg(cfg->lr_add) || !fin_nonneg(cfg->lr_mul)) return fail(MPADAM_EINVAL, "learning rates must be finite, >= 0");
   if (!fin_nonneg(cfg->rmax) || !(std::isfinite(cfg->tau) && cfg->tau > 0.0f))
@@ -1182,7 +1192,9 @@ extern "C" int32_t mpadam_toy_create(int64_t n, const mpadam_toy_config* cfg, mp
   if (cudaMalloc(&a.cnt, sizeof(int32_t) * n) != cudaSuccess || cudaMalloc(&a.first, sizeof(int32_t) * n) != cudaSuccess ||
       cudaMalloc(&a.idx, sizeof(int32_t) * B) != cudaSuccess || cudaMalloc(&a.res, sizeof(float) * B) != cudaSuccess ||
       cudaMalloc(&a.sq, sizeof(double) * B) != cudaSuccess || cudaMalloc(&a.alpha, sizeof(float) * 2) != cudaSuccess ||
-      cudaMalloc(&a.loss_h, sizeof(double) * 2) != cudaSuccess) {
+      cudaMalloc(&a.loss_h, sizeof(double) * 2) != cudaSuccess ||
+      cudaMalloc(&st->t_dev, sizeof(int64_t) * 2) != cudaSuccess ||
+      cudaMalloc(&a.partial, sizeof(double) * (B / 2048 + 2)) != cudaSuccess) {
     mpadam_toy_destroy(st);
     return fail(MPADAM_EALLOC, "allocation of the diagnostic's scratch failed");
   }
@@ -1228,11 +1240,64 @@ extern "C" int32_t mpadam_toy_step(mpadam_toy_state* s, uint16_t* w, const float
   return MPADAM_OK;
 }
 
+extern "C" int32_t mpadam_toy_run(mpadam_toy_state* s, uint16_t* w, const float* wstar, int64_t first_step,
+                                  int64_t steps, double* losses, cudaStream_t stream) {
+  if (!s) return fail(MPADAM_EINVAL, "state is NULL");
+  if (!w || !wstar || !is_aligned(w, 2) || !is_aligned(wstar, 4)) return fail(MPADAM_EINVAL, "w / wstar NULL or misaligned");
+  if (losses && !is_aligned(losses, 8)) return fail(MPADAM_EINVAL, "losses misaligned");
+  if (first_step < 1 || steps < 0) return fail(MPADAM_EINVAL, "first_step must be >= 1 and steps >= 0");
+  if (steps == 0) return MPADAM_OK;
+  int dev = -1;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+  if (dev != s->device) return fail(MPADAM_EINVAL, "current device %d differs from the state's device %d", dev, s->device);
+  mpadam::ToyArgs a = s->a;
+  a.w = w;
+  a.wstar = wstar;
+  a.loss_out = nullptr;
+  a.t_dev = s->t_dev;
+  a.loss_base = losses;
+  // the graph of kToyGraphSteps steps, captured once per set of pointers
+  if (steps >= kToyGraphSteps && (!s->exec || s->g_w != w || s->g_ws != wstar || s->g_loss != losses)) {
+    if (s->exec) { cudaGraphExecDestroy(s->exec); s->exec = nullptr; }
+    if (!s->cap && (e = cudaStreamCreateWithFlags(&s->cap, cudaStreamNonBlocking)) != cudaSuccess)
+      return cuda_fail(e, "cudaStreamCreate");
+    if ((e = cudaStreamBeginCapture(s->cap, cudaStreamCaptureModeThreadLocal)) != cudaSuccess)
+      return cuda_fail(e, "cudaStreamBeginCapture");
+    cudaError_t le = cudaSuccess;
+    for (int64_t i = 0; i < kToyGraphSteps && le == cudaSuccess; ++i) le = mpadam::launch_toy_step(a, s->cap);
+    cudaGraph_t graph = nullptr;
+    e = cudaStreamEndCapture(s->cap, &graph);
+    if (le != cudaSuccess || e != cudaSuccess) {
+      if (graph) cudaGraphDestroy(graph);
+      return cuda_fail(le != cudaSuccess ? le : e, "capture of the diagnostic's run graph");
+    }
+    e = cudaGraphInstantiate(&s->exec, graph, 0);
+    cudaGraphDestroy(graph);
+    if (e != cudaSuccess) { s->exec = nullptr; return cuda_fail(e, "cudaGraphInstantiate"); }
+    s->g_w = w;
+    s->g_ws = wstar;
+    s->g_loss = losses;
+  }
+  if ((e = mpadam::launch_toy_set_step(s->t_dev, first_step, stream)) != cudaSuccess)
+    return cuda_fail(e, "launch of the step-counter kernel");
+  int64_t done = 0;
+  for (; s->exec && done + kToyGraphSteps <= steps; done += kToyGraphSteps)
+    if ((e = cudaGraphLaunch(s->exec, stream)) != cudaSuccess) return cuda_fail(e, "cudaGraphLaunch");
+  for (; done < steps; ++done)
+    if ((e = mpadam::launch_toy_step(a, stream)) != cudaSuccess) return cuda_fail(e, "launch of the diagnostic's kernels");
+  return MPADAM_OK;
+}
+
 extern "C" int32_t mpadam_toy_destroy(mpadam_toy_state* s) {
   if (!s) return MPADAM_OK;
   cudaDeviceSynchronize();
+  if (s->exec) cudaGraphExecDestroy(s->exec);
+  if (s->cap) cudaStreamDestroy(s->cap);
+  if (s->t_dev) cudaFree(s->t_dev);
   mpadam::ToyArgs& a = s->a;
-  for (void* p : {(void*)a.cnt, (void*)a.first, (void*)a.idx, (void*)a.res, (void*)a.sq, (void*)a.alpha, (void*)a.loss_h})
+  for (void* p : {(void*)a.cnt, (void*)a.first, (void*)a.idx, (void*)a.res, (void*)a.sq, (void*)a.alpha, (void*)a.loss_h,
+                  (void*)a.partial})
     if (p) cudaFree(p);
   delete s;
   return MPADAM_OK;

@@ -6,11 +6,13 @@
 // entry, rounding it to BF16.  Three launches per step:
 //   1. sample (Philox lanes), residuals, hit counts and each entry's first
 //      sample (atomics on two n-entry scratch arrays, zero between steps);
-//   2. one CTA per half: the mean of the squared residuals as a perfect
-//      binary tree of binary64 sums over adjacent samples, the gradient
-//      scale alpha = 4 c M / B_h and the loss;
-//   3. the first sample of each entry applies the entry's update (its
-//      contribution alpha r added once per hit) and clears the scratch.
+//   2. partial sums of the squared residuals over aligned chunks of 2048
+//      samples (subtrees of the perfect binary tree of binary64 sums over
+//      adjacent samples);
+//   3. every CTA completes the tree from the partials (at most 32 per
+//      problem), forms M, the loss and alpha = 4 c M / B_h; the first sample
+//      of each entry applies the entry's update (its contribution alpha r
+//      added once per hit) and clears the scratch.
 // Every result is deterministic and equals the oracle's bit for bit.
 #include <cuda_runtime.h>
 
@@ -23,15 +25,34 @@
 namespace mpadam {
 namespace {
 
+// This step's number: from the device counter in run mode, else the argument.
+__device__ __forceinline__ void toy_step_number(const ToyArgs& a, uint32_t& lo, uint32_t& hi) {
+  if (a.t_dev) {
+    const uint64_t t = static_cast<uint64_t>(*a.t_dev);
+    lo = static_cast<uint32_t>(t);
+    hi = static_cast<uint32_t>(t >> 32);
+  } else {
+    lo = a.t_lo;
+    hi = a.t_hi;
+  }
+}
+
+__global__ void toy_set_step_kernel(int64_t* t_dev, int64_t first) {
+  t_dev[0] = first;
+  t_dev[1] = first;
+}
+
 __global__ void toy_sample_kernel(const __grid_constant__ ToyArgs a) {
   const int64_t s = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x;
   if (s >= a.batch) return;
+  uint32_t t_lo, t_hi;
+  toy_step_number(a, t_lo, t_hi);
   const int64_t Bh = a.batch / (a.split ? 2 : 1);
   const int64_t range = a.n / (a.split ? 2 : 1);
   const int64_t h = a.split ? s / Bh : 0;
   // 32-bit random lane s of step t: word s mod 4 of Philox block s / 4
   const uint64_t blk = static_cast<uint64_t>(s) >> 2;
-  const uint4 r4 = philox4x32_10(static_cast<uint32_t>(blk), static_cast<uint32_t>(blk >> 32), a.t_lo, a.t_hi, a.rk0,
+  const uint4 r4 = philox4x32_10(static_cast<uint32_t>(blk), static_cast<uint32_t>(blk >> 32), t_lo, t_hi, a.rk0,
                                  a.rk1);
   const uint32_t lanes[4] = {r4.x, r4.y, r4.z, r4.w};
   const uint32_t lane = lanes[s & 3];
@@ -45,59 +66,89 @@ __global__ void toy_sample_kernel(const __grid_constant__ ToyArgs a) {
   atomicMax(&a.first[idx], INT_MAX - static_cast<int32_t>(s));  // the smallest sample wins
 }
 
-// Tree sum of one half's squared residuals: thread t takes the contiguous
-// chunk of L = B_h / T samples (a binary-counter stack keeps the pairing of
-// a perfect tree), then adjacent lanes, then adjacent warps.
-__global__ void __launch_bounds__(1024) toy_reduce_kernel(const __grid_constant__ ToyArgs a) {
+// Tree sum of the squared residuals, stage 1: CTA b of a problem sums the
+// aligned chunk of C = min(2048, B_h) samples [bC, bC + C) as a perfect
+// binary tree (adjacent pairs per thread, then adjacent lanes, then adjacent
+// warps) into partial[problem][b].
+constexpr int kToyChunk = 2048;
+
+__global__ void __launch_bounds__(kToyChunk / 2) toy_partial_kernel(const __grid_constant__ ToyArgs a) {
   __shared__ double warp_sum[32];
-  const int h = blockIdx.x;
   const int64_t Bh = a.batch / (a.split ? 2 : 1);
-  const int T = blockDim.x;
-  const int64_t L = Bh / T;
-  const double* v = a.sq + h * Bh + threadIdx.x * L;
-  double stk[40];
-  int top = 0;
-  for (int64_t i = 0; i < L; ++i) {
-    double x = v[i];
-    int lvl = 0;
-    for (uint64_t j = static_cast<uint64_t>(i); j & 1u; j >>= 1) x = stk[lvl++] + x;
-    stk[lvl] = x;
-    top = lvl;
-  }
-  double x = stk[top];
-#pragma unroll
-  for (int off = 1; off < 32; off <<= 1) {
+  const int64_t C = Bh < kToyChunk ? Bh : kToyChunk;
+  const int64_t per = Bh / C;  // chunks per problem
+  const int h = static_cast<int>(blockIdx.x / per), b = static_cast<int>(blockIdx.x % per);
+  const double* v = a.sq + h * Bh + b * C;
+  const int pairs = static_cast<int>(C / 2);
+  const int t = threadIdx.x;
+  double x = t < pairs ? v[2 * t] + v[2 * t + 1] : 0.0;
+  const int span = pairs < 32 ? pairs : 32;  // lanes holding pair sums
+  for (int off = 1; off < span; off <<= 1) {
     const double y = __shfl_xor_sync(0xFFFFFFFFu, x, off);
-    x = (threadIdx.x & off) ? y + x : x + y;
+    x = (t & off) ? y + x : x + y;
   }
-  if ((threadIdx.x & 31) == 0) warp_sum[threadIdx.x >> 5] = x;
+  const int nw = (pairs + 31) / 32;
+  if ((t & 31) == 0 && t < pairs) warp_sum[t >> 5] = x;
   __syncthreads();
-  if (threadIdx.x < 32) {
-    const int nw = T >> 5;
-    double w = threadIdx.x < nw ? warp_sum[threadIdx.x] : 0.0;
+  if (t < 32) {
+    double w = t < nw ? warp_sum[t] : 0.0;
     for (int off = 1; off < nw; off <<= 1) {
       const double y = __shfl_xor_sync(0xFFFFFFFFu, w, off);
-      w = (threadIdx.x & off) ? y + w : w + y;
+      w = (t & off) ? y + w : w + y;
     }
-    if (threadIdx.x == 0) {
-      const double M = w / static_cast<double>(Bh);
-      const double ch = static_cast<double>(h == 0 ? a.c_lo : a.c_hi);
-      a.loss_h[h] = ch * M * M;
-      a.alpha[h] = static_cast<float>(((4.0 * ch) * M) / static_cast<double>(Bh));
-    }
+    if (t == 0) a.partial[h * per + b] = w;
   }
 }
 
+// Stage 2 (every update CTA): the problem's partial sums, a perfect tree
+// over at most 32 adjacent chunks, then M, the loss and alpha.
+__device__ __forceinline__ void toy_finish_mean(const ToyArgs& a, int h, double& loss_h, float& alpha_h) {
+  const int64_t Bh = a.batch / (a.split ? 2 : 1);
+  const int64_t C = Bh < kToyChunk ? Bh : kToyChunk;
+  const int per = static_cast<int>(Bh / C);
+  const int lane = threadIdx.x & 31;
+  double w = lane < per ? a.partial[h * per + lane] : 0.0;
+  for (int off = 1; off < per; off <<= 1) {
+    const double y = __shfl_xor_sync(0xFFFFFFFFu, w, off);
+    w = (lane & off) ? y + w : w + y;
+  }
+  const double M = w / static_cast<double>(Bh);
+  const double ch = static_cast<double>(h == 0 ? a.c_lo : a.c_hi);
+  loss_h = ch * M * M;
+  alpha_h = static_cast<float>(((4.0 * ch) * M) / static_cast<double>(Bh));
+}
+
 __global__ void toy_update_kernel(const __grid_constant__ ToyArgs a) {
+  __shared__ double s_loss[2];
+  __shared__ float s_alpha[2];
+  if (threadIdx.x < 64) {  // warp 0: the first problem, warp 1: the second
+    const int h = threadIdx.x >> 5;
+    if (h < (a.split ? 2 : 1)) {
+      double l;
+      float al;
+      toy_finish_mean(a, h, l, al);
+      if ((threadIdx.x & 31) == 0) { s_loss[h] = l; s_alpha[h] = al; }
+    }
+  }
+  __syncthreads();
   const int64_t s = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x;
-  if (s == 0 && a.loss_out) *a.loss_out = a.split ? (0.0 + a.loss_h[0]) + a.loss_h[1] : 0.0 + a.loss_h[0];
+  if (s == 0) {
+    const double loss = a.split ? (0.0 + s_loss[0]) + s_loss[1] : 0.0 + s_loss[0];
+    if (a.t_dev) {  // run mode: record the loss by step, then advance the step counter
+      const int64_t t = *a.t_dev;
+      if (a.loss_base) a.loss_base[t - a.t_dev[1]] = loss;
+      *a.t_dev = t + 1;  // read again only by the next step's kernels
+    } else if (a.loss_out) {
+      *a.loss_out = loss;
+    }
+  }
   if (s >= a.batch) return;
   const int32_t idx = a.idx[s];
   if (a.first[idx] != INT_MAX - static_cast<int32_t>(s)) return;  // the entry's first sample applies its update
   const int64_t Bh = a.batch / (a.split ? 2 : 1);
   const int h = a.split ? static_cast<int>(s / Bh) : 0;
   const int32_t k = a.cnt[idx];
-  const float x = __fmul_rn(a.alpha[h], a.res[s]);
+  const float x = __fmul_rn(s_alpha[h], a.res[s]);
   float g = x;
   for (int32_t i = 1; i < k; ++i) g = __fadd_rn(g, x);
   const float wf = __uint_as_float(static_cast<uint32_t>(a.w[idx]) << 16);
@@ -127,10 +178,16 @@ cudaError_t launch_toy_step(const ToyArgs& a, cudaStream_t stream) {
   toy_sample_kernel<<<blocks, 256, 0, stream>>>(a);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  toy_reduce_kernel<<<halves, static_cast<unsigned>(Bh < 1024 ? Bh : 1024), 0, stream>>>(a);
+  const int64_t C = Bh < kToyChunk ? Bh : kToyChunk;
+  toy_partial_kernel<<<static_cast<unsigned>(halves * (Bh / C)), kToyChunk / 2, 0, stream>>>(a);
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   toy_update_kernel<<<blocks, 256, 0, stream>>>(a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_toy_set_step(int64_t* t_dev, int64_t first, cudaStream_t stream) {
+  toy_set_step_kernel<<<1, 1, 0, stream>>>(t_dev, first);
   return cudaGetLastError();
 }
 

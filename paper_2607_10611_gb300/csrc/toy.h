@@ -17,10 +17,14 @@ struct ToyArgs {
   int32_t* idx;         // [batch]
   float* res;           // [batch]
   double* sq;           // [batch]
-  float* alpha;         // [2]
-  double* loss_h;       // [2]
-  double* loss_out;     // caller's device double, or nullptr
-  int64_t n, batch;     // powers of two; batch / halves >= 32, <= 2^16 * 1024
+  float* alpha;         // [2] (unused)
+  double* loss_h;       // [2] (unused)
+  double* partial;      // [batch / 2048 + 2] chunk sums of the squared residuals
+  double* loss_out;     // caller's device double, or nullptr (step-by-step mode)
+  int64_t* t_dev;       // run mode: [0] = this step's t (advanced by the update kernel), [1] = the run's first t;
+                        // nullptr in step-by-step mode (t from t_lo / t_hi)
+  double* loss_base;    // run mode: the loss of step t goes to loss_base[t - t_dev[1]] (or nowhere if nullptr)
+  int64_t n, batch;     // powers of two; 32 <= batch / halves <= 32 * 2048
   int32_t mode, split;
   float lr_add, lr_mul, rmax, tau, c_lo, c_hi;
   uint32_t rk0[kPhiloxRounds], rk1[kPhiloxRounds];
@@ -28,5 +32,7 @@ struct ToyArgs {
 };
 
 cudaError_t launch_toy_step(const ToyArgs& a, cudaStream_t stream);
+// Run mode: sets t_dev = {first, first} on `stream` (before the steps).
+cudaError_t launch_toy_set_step(int64_t* t_dev, int64_t first, cudaStream_t stream);
 
 }  // namespace mpadam

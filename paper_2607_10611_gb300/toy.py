@@ -40,6 +40,14 @@ class ToyDiagnostic:
         out = self.loss if loss_out is None else loss_out
         N.mpadam_toy_step(self.state, self.w.data_ptr(), self.wstar.data_ptr(), t, out.data_ptr(), s)
 
+    def run(self, first_step: int, steps: int, losses: Optional[torch.Tensor] = None,
+            stream: Optional[torch.cuda.Stream] = None):
+        """Steps first_step .. first_step + steps - 1 (CUDA-graph replays);
+        losses: a CUDA float64 tensor of `steps` elements, or None."""
+        s = (stream or torch.cuda.current_stream(self.w.device)).cuda_stream
+        N.mpadam_toy_run(self.state, self.w.data_ptr(), self.wstar.data_ptr(), first_step, steps,
+                         losses.data_ptr() if losses is not None else 0, s)
+
     def close(self):
         if getattr(self, "state", None):
             N.mpadam_toy_destroy(self.state)

@@ -70,3 +70,28 @@ def test_toy_rejects_bad_arguments():
         cfg = N.mpadam_toy_config(**{**ok, **over})
         with pytest.raises(N.MPAdamError):
             N.mpadam_toy_create(n, cfg)
+
+
+@pytest.mark.parametrize("regime", ["sign_flip", "mixed"])
+def test_toy_run_graph_replays_equal_single_steps(regime):
+    """mpadam_toy_run (CUDA-graph replays of 64 steps, a plain remainder,
+    the step number in device memory) gives the bits of step-by-step calls,
+    also when called again and with new pointers (a new capture)."""
+    from paper_2607_10611_gb300.toy import ToyDiagnostic
+    p = W.toy_problem(regime, n=256, seed=3)
+    kw = dict(mode="combined", batch=1024, c_lo=p.c_lo, c_hi=p.c_hi, split=p.split, seed=2,
+              lr_add=48.0, lr_mul=48.0)
+    ws = p.wstar.to("cuda")
+    w1, w2 = p.w0.to("cuda"), p.w0.to("cuda")
+    d1, d2 = ToyDiagnostic(w1, ws, **kw), ToyDiagnostic(w2, ws, **kw)
+    steps = 2 * 64 + 5
+    l1 = torch.zeros(steps, dtype=torch.float64, device="cuda")
+    for t in range(1, steps + 1):
+        d1.step(t, loss_out=l1[t - 1:t])
+    l2 = torch.zeros(steps, dtype=torch.float64, device="cuda")
+    d2.run(1, 70, l2[:70])
+    d2.run(71, steps - 70, l2[70:])       # new losses pointer: a new capture
+    torch.cuda.synchronize()
+    assert torch.equal(w1, w2)
+    assert torch.equal(l1, l2)
+    d1.close(); d2.close()
