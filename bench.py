@@ -71,8 +71,11 @@ def measured_peaks():
 
 
 def kernel_source_hash() -> str:
+    """Hash of the step kernel's sources (the files its DRAM traffic depends
+    on: the kernel template, its argument layout and its instantiations)."""
     h = hashlib.sha256()
-    for f in sorted((ROOT / "paper_2607_10611_gb300" / "csrc").glob("*")):
+    csrc = ROOT / "paper_2607_10611_gb300" / "csrc"
+    for f in sorted([csrc / "step_kernel.cuh", csrc / "step_args.h", *csrc.glob("step_*.cu")]):
         h.update(f.read_bytes())
     return h.hexdigest()[:16]
 
