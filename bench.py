@@ -261,11 +261,19 @@ def run_gpu(wl, steps: int, warmup: int, rank: int, e2e_steps: int):
 
     # end to end through the host-buffer entry point (one weight format: flat host buffers)
     if e2e_steps > 0 and "w" in mt.flat:
-        # page-locked huge-page host buffers (mpadam_host_buffer_alloc)
+        # page-locked host buffers: huge-page ones from mpadam_host_buffer_alloc,
+        # or the driver's (torch pin_memory), whichever copies faster here
         from paper_2607_10611_gb300.optimizer import HostBuffer
-        hg_buf = HostBuffer(mt.flat["g"].numel(), mt.flat["g"].dtype)
-        hw_buf = HostBuffer(mt.flat["w"].numel(), mt.flat["w"].dtype)
-        hg, hw = hg_buf.tensor, hw_buf.tensor
+        kind = pinned_kind_for_this_host(stream)
+        if kind == "huge_pages":
+            hg_buf = HostBuffer(mt.flat["g"].numel(), mt.flat["g"].dtype)
+            hw_buf = HostBuffer(mt.flat["w"].numel(), mt.flat["w"].dtype)
+            hg, hw = hg_buf.tensor, hw_buf.tensor
+        else:
+            hg_buf = hw_buf = None
+            hg = torch.empty(mt.flat["g"].shape, dtype=mt.flat["g"].dtype, pin_memory=True)
+            hw = torch.empty(mt.flat["w"].shape, dtype=mt.flat["w"].dtype, pin_memory=True)
+        res["host_buffers"] = kind
         hg.copy_(mt.flat["g"])
         hgs = [hg[o:o + x.numel()] for o, x in zip(mt.offsets, mt.g)]
         hws = [hw[o:o + x.numel()] for o, x in zip(mt.offsets, mt.w)]
@@ -285,13 +293,41 @@ def run_gpu(wl, steps: int, warmup: int, rank: int, e2e_steps: int):
         res["d2h"] = sum(x.numel() for x in mt.w) * BYTES[wl.weight_dtype]
         res["link_ms"] = host_link_ms(hg, mt.flat["g"], hw, mt.flat["w"], stream)
         del hg, hw, hgs, hws
-        hg_buf.free()
-        hw_buf.free()
+        if hg_buf is not None:
+            hg_buf.free()
+            hw_buf.free()
     opt.close()
     del mt, opt
     torch.cuda.synchronize()
     torch.cuda.empty_cache()
     return res
+
+
+def pinned_kind_for_this_host(stream) -> str:
+    """'huge_pages' (mpadam_host_buffer_alloc) or 'driver' (torch pin_memory):
+    the faster of a 1 GiB host-to-device copy from each, best of three."""
+    import torch
+    from paper_2607_10611_gb300.optimizer import HostBuffer
+    n = 1 << 29
+    dev = torch.empty(n, dtype=torch.bfloat16, device=stream.device)
+    def best(h):
+        t = float("inf")
+        for _ in range(3):
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            torch.cuda.synchronize()
+            a.record(stream)
+            dev.copy_(h, non_blocking=True)
+            b.record(stream)
+            torch.cuda.synchronize()
+            t = min(t, a.elapsed_time(b))
+        return t
+    hb = HostBuffer(n, torch.bfloat16)
+    t_huge = best(hb.tensor)
+    hb.free()
+    hp = torch.empty(n, dtype=torch.bfloat16, pin_memory=True)
+    t_drv = best(hp)
+    del hp, dev
+    return "huge_pages" if t_huge <= t_drv else "driver"
 
 
 def host_link_ms(h_src, d_dst, h_dst, d_src, stream, reps: int = 3) -> float:
@@ -396,7 +432,8 @@ def summarize(wl, res, n_gpus, peak, peak_kind):
                       "ms_per_step": res["e2e_ms"],
                       "host_link_ms": res["link_ms"],
                       "host_link_gbs": (res["h2d"] + res["d2h"]) / (res["link_ms"] * 1e-3) / 1e9,
-                      "frac_of_host_link_bound": res["link_ms"] / res["e2e_ms"]}
+                      "frac_of_host_link_bound": res["link_ms"] / res["e2e_ms"],
+                      "host_buffers": res.get("host_buffers")}
     return out
 
 

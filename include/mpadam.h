@@ -258,8 +258,9 @@ int32_t mpadam_step_host(mpadam_state* s, const void* const* host_grads, void* c
 
 /* Page-locked host memory for mpadam_step_host's buffers (not from the
  * paper: a deployment aid).  Allocates `bytes` of anonymous memory advised
- * for transparent huge pages, touches it (so the pages are resident and
- * large), and registers it with the CUDA driver (cudaHostRegister).  Copies
+ * for transparent huge pages and preferring the host NUMA node nearest the
+ * current device, touches it (so the pages are resident and large), and
+ * registers it with the CUDA driver (cudaHostRegister).  Copies
  * from such a buffer keep the host link's full rate: on GB300 (Grace) hosts,
  * copies from ordinary pinned memory of 64 KB pages measured 4x slower at
  * times for buffers of several GB, huge-page buffers did not.  Release with

@@ -4,6 +4,8 @@
 // lives in step_kernel.cuh.
 #include <cuda_runtime.h>
 #include <sys/mman.h>
+#include <sys/syscall.h>
+#include <unistd.h>
 
 #include <algorithm>
 #include <cmath>
@@ -1315,6 +1317,17 @@ extern "C" int32_t mpadam_host_buffer_alloc(int64_t bytes, void** out) {
 #ifdef MADV_HUGEPAGE
   madvise(p, (size_t)bytes, MADV_HUGEPAGE);  // advice only: a kernel without it still gives a valid buffer
 #endif
+  // Place the pages on the host NUMA node nearest the current GPU (as the
+  // driver's own pinned allocations are): on multi-socket hosts, first touch
+  // by a thread on the far socket put them across the socket link.
+  int dev = 0, node = -1;
+  if (cudaGetDevice(&dev) == cudaSuccess && cudaDeviceGetAttribute(&node, cudaDevAttrHostNumaId, dev) == cudaSuccess &&
+      node >= 0 && node < 1024) {
+    unsigned long mask[1024 / (8 * sizeof(unsigned long))] = {};
+    mask[node / (8 * sizeof(unsigned long))] |= 1UL << (node % (8 * sizeof(unsigned long)));
+    const long kMpolPreferred = 1;
+    syscall(SYS_mbind, p, (unsigned long)bytes, kMpolPreferred, mask, 1024UL + 1UL, 0UL);  // advice: failure is harmless
+  }
   std::memset(p, 0, (size_t)bytes);  // resident before registration
   cudaError_t e = cudaHostRegister(p, (size_t)bytes, cudaHostRegisterDefault);
   if (e != cudaSuccess) {
