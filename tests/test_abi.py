@@ -86,3 +86,48 @@ def test_null_state_and_bad_step(N):
     assert lib.mpadam_destroy(None) == N.MPADAM_OK
     assert lib.mpadam_rng_lanes(0, 1, 7, 0, 4, None, None) == N.MPADAM_EINVAL
     assert lib.mpadam_rng_lanes(0, 1, N.MPADAM_BF16, -1, 4, None, None) == N.MPADAM_EINVAL
+
+
+def test_create_ex_rejects_bad_lists_on_the_host(N):
+    """Per-tensor formats, block scales, compute copies and tensor scales are
+    validated before any CUDA call."""
+    cfg = N.make_config()
+    W, M, S, C = 0x10000, 0x20000, 0x30000, 0x40000
+    bad = [
+        (W, M, M, M, 64, 9, 0, 0),                    # unknown format
+        (W, M, M, M, 64, "e4m3_b32", 0, 0),           # block scales missing
+        (W, M, M, M, 64, "e4m3_b32", S + 1, 0),       # misaligned FP16 scales
+        (W, M, M, M, 64, "nvfp4", 0, 0, 1e-3),        # NVFP4 scales missing
+        (W, M, M, M, 64, "nvfp4", S, 0, 0.0),         # no tensor scale
+        (W, M, M, M, 64, "nvfp4", S, 0, float("nan")),
+        (W, M, M, M, 64, "bf16", 0, C),               # compute copy of BF16 weights
+        (W, M, M, M, 64, "bf16", S, 0),               # block scales on BF16 weights
+        (W, M, M, M, 64, "e4m3_b32", S, 0, 1e-3),     # tensor scale on another format
+        (W, M, M, M, 64, "e4m3", 0, 0),               # E4M3 without the fp8 rings
+        (W, M, M + 2, M, 64, "bf16", 0, 0),           # misaligned fp32 moment
+    ]
+    for t in bad:
+        with pytest.raises(N.MPAdamError) as ei:
+            N.mpadam_create_ex([t], cfg)
+        assert ei.value.status == N.MPADAM_EINVAL, t
+    for fmt in ("e4m3_b32", "nvfp4"):  # the uniform entry point cannot carry block scales
+        with pytest.raises(N.MPAdamError):
+            N.mpadam_create(_tensor_tuple(), N.make_config(weight_dtype=fmt))
+
+
+def test_toy_create_rejects_bad_config_on_the_host(N):
+    ok = dict(mode=2, split=0, batch=64, reserved=0, lr_add=1.0, lr_mul=1.0, rmax=0.75, tau=1e-8, c_lo=1.0,
+              c_hi=1.0, seed=0)
+    for n, over in [(100, {}), (32, {}), (1 << 31, {}), (64, {"batch": 48}), (64, {"batch": 32, "split": 1}),
+                    (64, {"batch": 1 << 17}), (64, {"mode": 3}), (64, {"split": 2}), (64, {"tau": 0.0}),
+                    (64, {"lr_add": -1.0}), (64, {"lr_mul": float("inf")}), (64, {"reserved": 1}),
+                    (64, {"c_lo": float("nan")})]:
+        with pytest.raises(N.MPAdamError) as ei:
+            N.mpadam_toy_create(n, N.mpadam_toy_config(**{**ok, **over}))
+        assert ei.value.status == N.MPADAM_EINVAL, (n, over)
+    lib = N.lib()
+    assert lib.mpadam_toy_step(None, None, None, 1, None, None) == N.MPADAM_EINVAL
+    assert lib.mpadam_toy_run(None, None, None, 1, 1, None, None) == N.MPADAM_EINVAL
+    assert lib.mpadam_toy_destroy(None) == N.MPADAM_OK
+    assert lib.mpadam_host_buffer_alloc(0, None) == N.MPADAM_EINVAL
+    assert lib.mpadam_host_buffer_free(None, 16) == N.MPADAM_OK
