@@ -268,6 +268,13 @@ int32_t mpadam_step_host(mpadam_state* s, const void* const* host_grads, void* c
 int32_t mpadam_host_buffer_alloc(int64_t bytes, void** out);
 int32_t mpadam_host_buffer_free(void* ptr, int64_t bytes);
 
+/* Fault injection for tests (the paper has no counterpart): the library's
+ * device or pinned allocation after `after` more successful ones fails once,
+ * as if the driver had refused it (every entry point then returns
+ * MPADAM_EALLOC and releases what it had allocated); -1 disarms.  Process-
+ * wide.  Errors: EINVAL. */
+int32_t mpadam_debug_fail_allocation(int32_t after);
+
 /* Frees the library's metadata (synchronises the device first).  NULL is a
  * no-op.  Never touches caller-owned tensors. */
 int32_t mpadam_destroy(mpadam_state* s);

@@ -24,7 +24,7 @@ EXPORTED = ["mpadam_create", "mpadam_create_ex", "mpadam_fp8_init", "mpadam_step
             "mpadam_destroy", "mpadam_last_error", "mpadam_global_offset", "mpadam_global_length", "mpadam_set_grid",
             "mpadam_launch_info", "mpadam_rng_lanes", "mpadam_step_noalloc", "mpadam_device_status",
             "mpadam_toy_create", "mpadam_toy_step", "mpadam_toy_run", "mpadam_toy_destroy", "mpadam_host_buffer_alloc",
-            "mpadam_host_buffer_free"]
+            "mpadam_host_buffer_free", "mpadam_debug_fail_allocation"]
 
 
 class MPAdamError(RuntimeError):
@@ -120,6 +120,7 @@ def lib() -> ctypes.CDLL:
             "mpadam_toy_destroy": [P],
             "mpadam_host_buffer_alloc": [i64, P],
             "mpadam_host_buffer_free": [P, i64],
+            "mpadam_debug_fail_allocation": [i32],
         }
         for name, args in sig.items():
             f = getattr(L, name)
@@ -264,3 +265,9 @@ def mpadam_host_buffer_alloc(nbytes: int) -> int:
 
 def mpadam_host_buffer_free(ptr: int, nbytes: int) -> None:
     _check(lib().mpadam_host_buffer_free(ptr, nbytes))
+
+
+def mpadam_debug_fail_allocation(after: int) -> None:
+    """Test hook: the library's allocation after `after` more successful ones
+    fails once (-1 disarms)."""
+    _check(lib().mpadam_debug_fail_allocation(after))

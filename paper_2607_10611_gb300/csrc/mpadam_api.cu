@@ -8,6 +8,7 @@
 #include <unistd.h>
 
 #include <algorithm>
+#include <atomic>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
@@ -30,6 +31,32 @@ using mpadam::TensorDesc;
 namespace {
 
 thread_local std::string g_last_error;
+
+// Allocation-failure injection for the tests (mpadam_debug_fail_allocation):
+// the allocation after `countdown` more successful ones fails, once.
+std::atomic<int32_t> g_fail_countdown{-1};
+
+bool injected_failure() {
+  int32_t c = g_fail_countdown.load();
+  while (c >= 0) {
+    if (g_fail_countdown.compare_exchange_weak(c, c - 1)) return c == 0;
+  }
+  return false;
+}
+
+// Every device and pinned allocation of the library goes through these.
+cudaError_t dev_malloc(void** p, size_t bytes) {
+  if (injected_failure()) { *p = nullptr; return cudaErrorMemoryAllocation; }
+  return cudaMalloc(p, bytes);
+}
+template <typename T>
+cudaError_t dev_malloc(T** p, size_t bytes) {
+  return dev_malloc(reinterpret_cast<void**>(p), bytes);
+}
+cudaError_t host_malloc(void** p, size_t bytes) {
+  if (injected_failure()) { *p = nullptr; return cudaErrorMemoryAllocation; }
+  return cudaMallocHost(p, bytes);
+}
 
 int32_t fail(int32_t code, const char* fmt, ...) {
   char buf[512];
@@ -352,7 +379,7 @@ int32_t upload_cta_table(Group& g, int32_t grid) {
     if (g.d_cta_first) cudaFree(g.d_cta_first);
     g.d_cta_first = nullptr;
     g.cta_cap = 0;
-    if (cudaMalloc(&g.d_cta_first, sizeof(int32_t) * grid) != cudaSuccess)
+    if (dev_malloc(&g.d_cta_first, sizeof(int32_t) * grid) != cudaSuccess)
       return fail(MPADAM_EALLOC, "cudaMalloc of %d CTA entries failed", grid);
     g.cta_cap = grid;
   }
@@ -549,11 +576,11 @@ int32_t create_state(const std::vector<TensorIn>& t, const mpadam_config* cfg, i
     }
 
     const size_t nn = n > 0 ? (size_t)n : 1;
-    if (cudaMalloc(&s->d_desc, sizeof(TensorDesc) * nn) != cudaSuccess ||
-        cudaMalloc(reinterpret_cast<void**>(&s->d_grads), sizeof(void*) * nn) != cudaSuccess ||
-        (any_aux && cudaMalloc(&s->d_aux, sizeof(TensorAux) * nn) != cudaSuccess) ||
-        cudaMalloc(&s->d_err, sizeof(int32_t)) != cudaSuccess ||
-        cudaMallocHost(reinterpret_cast<void**>(&s->h_grads), sizeof(void*) * nn) != cudaSuccess) {
+    if (dev_malloc(&s->d_desc, sizeof(TensorDesc) * nn) != cudaSuccess ||
+        dev_malloc(reinterpret_cast<void**>(&s->d_grads), sizeof(void*) * nn) != cudaSuccess ||
+        (any_aux && dev_malloc(&s->d_aux, sizeof(TensorAux) * nn) != cudaSuccess) ||
+        dev_malloc(&s->d_err, sizeof(int32_t)) != cudaSuccess ||
+        host_malloc(reinterpret_cast<void**>(&s->h_grads), sizeof(void*) * nn) != cudaSuccess) {
       release(s);
       return fail(MPADAM_EALLOC, "allocation of the tensor tables failed");
     }
@@ -646,7 +673,7 @@ int32_t prepare_pipeline(mpadam_state* s) {
   std::vector<int32_t> first((size_t)chunks * g.grid);
   for (int32_t c = 0; c < chunks; ++c)
     cta_first_table(s->numel.data(), s->n, ct[c + 1] - ct[c], g.grid, first.data() + (size_t)c * g.grid, ct[c]);
-  if (cudaMalloc(&s->d_chunk_first, sizeof(int32_t) * first.size()) != cudaSuccess)
+  if (dev_malloc(&s->d_chunk_first, sizeof(int32_t) * first.size()) != cudaSuccess)
     return fail(MPADAM_EALLOC, "cudaMalloc of the chunk tables failed");
   cudaError_t e = cudaMemcpy(s->d_chunk_first, first.data(), sizeof(int32_t) * first.size(), cudaMemcpyHostToDevice);
   if (e != cudaSuccess) return cuda_fail(e, "upload of the chunk tables");
@@ -867,7 +894,7 @@ int32_t mpadam_step_host(mpadam_state* s, const void* const* host_grads, void* c
   const size_t gsz = elem_size(s->cfg.grad_dtype);
   cudaError_t e;
   if (!s->d_gstage) {
-    if (cudaMalloc(&s->d_gstage, (size_t)s->length * gsz) != cudaSuccess)
+    if (dev_malloc(&s->d_gstage, (size_t)s->length * gsz) != cudaSuccess)
       return fail(MPADAM_EALLOC, "cudaMalloc of %lld bytes of gradient staging failed",
                   (long long)((size_t)s->length * gsz));
     s->stage_ptrs.resize(s->n);
@@ -1191,12 +1218,12 @@ extern "C" int32_t mpadam_toy_create(int64_t n, const mpadam_toy_config* cfg, mp
   cudaError_t e = cudaGetDevice(&st->device);
   if (e != cudaSuccess) { delete st; return cuda_fail(e, "cudaGetDevice"); }
   const size_t B = (size_t)cfg->batch;
-  if (cudaMalloc(&a.cnt, sizeof(int32_t) * n) != cudaSuccess || cudaMalloc(&a.first, sizeof(int32_t) * n) != cudaSuccess ||
-      cudaMalloc(&a.idx, sizeof(int32_t) * B) != cudaSuccess || cudaMalloc(&a.res, sizeof(float) * B) != cudaSuccess ||
-      cudaMalloc(&a.sq, sizeof(double) * B) != cudaSuccess || cudaMalloc(&a.alpha, sizeof(float) * 2) != cudaSuccess ||
-      cudaMalloc(&a.loss_h, sizeof(double) * 2) != cudaSuccess ||
-      cudaMalloc(&st->t_dev, sizeof(int64_t) * 2) != cudaSuccess ||
-      cudaMalloc(&a.partial, sizeof(double) * (B / 2048 + 2)) != cudaSuccess) {
+  if (dev_malloc(&a.cnt, sizeof(int32_t) * n) != cudaSuccess || dev_malloc(&a.first, sizeof(int32_t) * n) != cudaSuccess ||
+      dev_malloc(&a.idx, sizeof(int32_t) * B) != cudaSuccess || dev_malloc(&a.res, sizeof(float) * B) != cudaSuccess ||
+      dev_malloc(&a.sq, sizeof(double) * B) != cudaSuccess || dev_malloc(&a.alpha, sizeof(float) * 2) != cudaSuccess ||
+      dev_malloc(&a.loss_h, sizeof(double) * 2) != cudaSuccess ||
+      dev_malloc(&st->t_dev, sizeof(int64_t) * 2) != cudaSuccess ||
+      dev_malloc(&a.partial, sizeof(double) * (B / 2048 + 2)) != cudaSuccess) {
     mpadam_toy_destroy(st);
     return fail(MPADAM_EALLOC, "allocation of the diagnostic's scratch failed");
   }
@@ -1344,5 +1371,11 @@ extern "C" int32_t mpadam_host_buffer_free(void* ptr, int64_t bytes) {
   cudaError_t e = cudaHostUnregister(ptr);
   munmap(ptr, (size_t)bytes);
   if (e != cudaSuccess) return cuda_fail(e, "cudaHostUnregister");
+  return MPADAM_OK;
+}
+
+extern "C" int32_t mpadam_debug_fail_allocation(int32_t after) {
+  if (after < -1) return fail(MPADAM_EINVAL, "after must be >= -1");
+  g_fail_countdown.store(after);
   return MPADAM_OK;
 }

@@ -46,36 +46,60 @@ def host_tensors(mt: W.Materialized) -> List[dict]:
     return out
 
 
+GUARD_BYTES = 64      # canary bytes before and after every separately allocated array
+CANARY = 0xA5
+
+
+def _guarded(t: torch.Tensor, misalign: int = 0):
+    """A CUDA copy of t inside a larger buffer whose bytes before and after
+    it hold a canary pattern (and, with misalign, shifted by that many
+    elements); returns (view, guard record)."""
+    es = t.element_size()
+    g = GUARD_BYTES // es
+    buf = torch.empty(t.numel() + 2 * g + misalign, dtype=t.dtype, device="cuda")
+    buf.view(torch.uint8).fill_(CANARY)
+    v = buf[g + misalign:g + misalign + t.numel()]
+    v.copy_(t)
+    return v, (buf, (g + misalign) * es, t.numel() * es)
+
+
+def canary_damage(guards) -> int:
+    """Bytes outside the arrays' own ranges that no longer hold the canary."""
+    bad = 0
+    for buf, start, nbytes in guards:
+        b = buf.view(torch.uint8)
+        bad += int((b[:start] != CANARY).sum()) + int((b[start + nbytes:] != CANARY).sum())
+    return bad
+
+
 def device_copy(mt: W.Materialized, layout: str = "separate", misalign: int = 0) -> Dict[str, list]:
-    """Copy a CPU-materialised workload to cuda:0.  misalign > 0 shifts every
-    tensor by that many elements inside a larger allocation (vector path off)."""
-    out = {}
+    """Copy a CPU-materialised workload to cuda:0.  Separately allocated
+    arrays sit between canary bytes (checked by canary_damage(out["_guards"]));
+    misalign > 0 also shifts every tensor by that many elements (vector path
+    off)."""
+    out = {"_guards": []}
     for key in ("w", "g", "m", "v", "ve"):
         src = getattr(mt, key)
         if layout == "flat" and key in mt.flat:
-            base = mt.flat[key].to("cuda")
+            base, guard = _guarded(mt.flat[key])
+            out["_guards"].append(guard)
             out[key] = [base[o:o + t.numel()] for o, t in zip(mt.offsets, src)]
-        elif misalign:
+        else:
             views = []
             for t in src:
-                buf = torch.zeros(t.numel() + misalign, dtype=t.dtype, device="cuda")
-                v = buf[misalign:]
-                v.copy_(t)
+                v, guard = _guarded(t, misalign)
+                out["_guards"].append(guard)
                 views.append(v)
             out[key] = views
-        else:
-            out[key] = [t.to("cuda") for t in src]
     for key, src in (("bscale", mt.bscale), ("cc", mt.cc)):
         views = []
         for t in (src or [None] * len(mt.w)):
             if t is None:
                 views.append(None)
-            elif misalign:
-                buf = torch.zeros(t.numel() + misalign, dtype=t.dtype, device="cuda")
-                views.append(buf[misalign:])
-                views[-1].copy_(t)
             else:
-                views.append(t.to("cuda"))
+                v, guard = _guarded(t, misalign)
+                out["_guards"].append(guard)
+                views.append(v)
         out[key] = views
     return out
 
@@ -163,7 +187,8 @@ class Run:
         """Mismatch counts per array (and the E4M3 scale state read for step
         t_next); compute copies are checked when compute_copy, once a step has
         written them."""
-        res = {"w": 0, "m": 0, "v": 0, "ve": 0, "bscale": 0, "cc": 0, "elements": 0, "contract_ok": True}
+        res = {"w": 0, "m": 0, "v": 0, "ve": 0, "bscale": 0, "cc": 0, "elements": 0, "contract_ok": True,
+               "canary": canary_damage(self.dev["_guards"])}
         for k in range(len(self.host)):
             h = self.host[k]
             res["elements"] += h["g"].size
