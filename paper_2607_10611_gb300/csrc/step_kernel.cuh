@@ -770,12 +770,14 @@ __device__ __forceinline__ void finish_group(const StepArgs& a, const TensorCtx&
 
 // One group of a partial tile, or of a tensor whose arrays are not all staged
 // or aligned: loads each array from the stage when its bytes were staged, else
-// from global memory; kept out of line so the whole-tile path stays lean.
+// from global memory; kept out of line so the whole-tile path stays lean.  The
+// running E4M3 maximum goes in and comes back by value: a reference would pin
+// the caller's copy to local memory for the whole loop.
 template <int WD, int GD, int MD, bool SR, bool OPT>
-__device__ __noinline__ void general_group(const StepArgs& a, const TensorCtx& x, int64_t tile_e0, int count,
-                                           int c, uint32_t st, uint32_t& amax_bits) {
+__device__ __noinline__ uint32_t general_group(const StepArgs& a, const TensorCtx& x, int64_t tile_e0, int count,
+                                               int c, uint32_t st, uint32_t amax_bits) {
   constexpr int WS = esize_of(WD), GS = esize_of(GD), MS = esize_of(MD);
-  if (kGroup * c >= count) return;
+  if (kGroup * c >= count) return amax_bits;
   const int valid = count - kGroup * c < kGroup ? count - kGroup * c : kGroup;
   const int64_t e0 = tile_e0 + kGroup * c;
   const uint32_t end = static_cast<uint32_t>(kGroup * (c + 1));  // elements through this group
@@ -801,6 +803,7 @@ __device__ __noinline__ void general_group(const StepArgs& a, const TensorCtx& x
     get_bf16<false>(ve, e_st, st + a.off_ve + kGroup * MS * c, x.d.ve, e0, valid, x.vec);
   }
   finish_group<WD, GD, MD, SR, OPT>(a, x, e0, valid, w, g, m, v, ve, amax_bits);
+  return amax_bits;
 }
 
 // ---------------------------------------------------------------------------
@@ -1010,14 +1013,13 @@ __device__ __forceinline__ void e2m1x8_to_f32(uint32_t packed, float (&x)[8]) {
 
 // Eight binary32 -> packed E2M1 codes, nearest-even with saturation at +-6
 // (the hardware conversion; used only on finite values).
-__device__ __forceinline__ uint32_t e2m1x8_rn(const float (&x)[8]) {
+// Two binary32 -> two E2M1 codes, nearest-even (hardware conversion; x0 in
+// the low nibble).
+__device__ __forceinline__ uint32_t e2m1x2_rn(float x0, float x1) {
   uint32_t p;
-  asm("{\n .reg .b8 b0, b1, b2, b3;\n"
-      " cvt.rn.satfinite.e2m1x2.f32 b0, %2, %1;\n cvt.rn.satfinite.e2m1x2.f32 b1, %4, %3;\n"
-      " cvt.rn.satfinite.e2m1x2.f32 b2, %6, %5;\n cvt.rn.satfinite.e2m1x2.f32 b3, %8, %7;\n"
-      " mov.b32 %0, {b0, b1, b2, b3};\n}"
+  asm("{\n .reg .b8 b;\n cvt.rn.satfinite.e2m1x2.f32 b, %2, %1;\n cvt.u32.u8 %0, b;\n}"
       : "=r"(p)
-      : "f"(x[0]), "f"(x[1]), "f"(x[2]), "f"(x[3]), "f"(x[4]), "f"(x[5]), "f"(x[6]), "f"(x[7]));
+      : "f"(x0), "f"(x1));
   return p;
 }
 
@@ -1036,23 +1038,59 @@ __device__ __forceinline__ uint32_t e2m1_pair_sr(float xl, float xh, uint32_t r,
   return ((__float_as_uint(xl) >> 28) & 8u) | (__float2uint_rz(kl) + off + ul);
 }
 
-// Does E4M3 scale code c cover A (6 * (s * G) >= A, products rounded)?
-__device__ __forceinline__ bool fp4_covers(uint32_t c, float G, float A) {
-  return __fmul_rn(6.0f, __fmul_rn(e4m3_value(c), G)) >= A;
+// A block scale code with the two products its covering test and the encode
+// use: d = fl(v(c) G) (the block's step) and p = fl(6 d) (the largest
+// magnitude the code covers: c covers A iff p >= A).
+struct Fp4Code {
+  uint32_t c;
+  float d, p;
+};
+
+// Value of a positive finite E4M3 code (1..126) through the hardware widening
+// conversion (exact: every E4M3 value is an FP16 value).
+__device__ __forceinline__ float e4m3_value_cvt(uint32_t c) {
+  uint32_t h;
+  asm("{\n .reg .b16 lo;\n cvt.u16.u32 lo, %1;\n cvt.rn.f16x2.e4m3x2 %0, lo;\n}" : "=r"(h) : "r"(c & 0xFFu));
+  return __half2float(__ushort_as_half(static_cast<unsigned short>(h & 0xFFFFu)));
+}
+
+// c in [1, 126]
+__device__ __forceinline__ Fp4Code fp4_code(uint32_t c, float G) {
+  Fp4Code r;
+  r.c = c;
+  r.d = __fmul_rn(e4m3_value_cvt(c), G);
+  r.p = __fmul_rn(6.0f, r.d);
+  return r;
 }
 
 // Block scale code of the next encode: the smallest code in [1, 126] that
-// covers A (finite, >= 0), 126 when none does, c_old when A = 0.  Starts at
-// the E4M3 code of an estimate of A / (6 G) and steps to the smallest
-// covering code (covering is monotone in the code).
-__device__ __forceinline__ uint32_t nvfp4_scale_code(float A, float G, uint32_t c_old) {
-  if (!(A > 0.0f)) return c_old;
+// covers A (finite, >= 0), 126 when none does, c_old when A = 0.  Covering is
+// monotone in the code, so c is that code iff c covers A and c - 1 does not
+// (or c = 1).  The candidate is A / (6 G) rounded up onto the E4M3 grid;
+// both tests run side by side, and only a candidate that fails them (an
+// estimate within rounding of a grid point, or a step d out of the normal
+// range) walks to the answer one code at a time.
+static __device__ __noinline__ Fp4Code nvfp4_scale_code_walk(float A, float G, int32_t c) {
+  for (int i = 0; i < 126 && c > 1 && fp4_code(static_cast<uint32_t>(c - 1), G).p >= A; ++i) --c;
+  for (int i = 0; i < 126 && c < 126 && !(fp4_code(static_cast<uint32_t>(c), G).p >= A); ++i) ++c;
+  return fp4_code(static_cast<uint32_t>(c), G);
+}
+
+__device__ __forceinline__ Fp4Code nvfp4_scale_code(float A, float G, uint32_t c_old) {
+  if (!(A > 0.0f)) {  // the old code, whatever it holds (zero, NaN, a sign)
+    Fp4Code r;
+    r.c = c_old;
+    r.d = __fmul_rn(e4m3_value(c_old), G);
+    r.p = __fmul_rn(6.0f, r.d);
+    return r;
+  }
   const float est = div_approx<false>(A, __fmul_rn(6.0f, G));
-  int32_t c = static_cast<int32_t>(e4m3_encode<false>(est, 0u) & 0x7Fu);
+  int32_t c = static_cast<int32_t>(e4m3_encode<true>(est, 0u) & 0x7Fu);  // random bits 0: rounds up
   c = c < 1 ? 1 : (c > 126 ? 126 : c);
-  for (int i = 0; i < 126 && c > 1 && fp4_covers(static_cast<uint32_t>(c - 1), G, A); ++i) --c;
-  for (int i = 0; i < 126 && c < 126 && !fp4_covers(static_cast<uint32_t>(c), G, A); ++i) ++c;
-  return static_cast<uint32_t>(c);
+  const Fp4Code hi = fp4_code(static_cast<uint32_t>(c), G);
+  const float p_lo = c > 1 ? fp4_code(static_cast<uint32_t>(c - 1), G).p : 0.0f;
+  if (hi.p >= A && (c == 1 || !(p_lo >= A))) return hi;
+  return nvfp4_scale_code_walk(A, G, c);
 }
 
 // Eight packed codes (element j in bits [4j, 4j + 4)) -> the group's bytes.
@@ -1077,8 +1115,8 @@ __device__ __forceinline__ uint32_t pair_max(uint32_t x) {
 }
 
 // One element's canonical update recomputed from the stage's original
-// inputs (the stage is kept until the group is done when STAGED): the exact
-// weight of the element's group slot j.
+// inputs (kept until the group is done): the exact weight of the element's
+// group slot j.
 template <int GD, int MD>
 __device__ __forceinline__ float fp4_exact_from_stage(const StepArgs& a, uint32_t st, int c, int j, float d_old) {
   constexpr int GS = esize_of(GD), MS = esize_of(MD);
@@ -1095,11 +1133,42 @@ __device__ __forceinline__ float fp4_exact_from_stage(const StepArgs& a, uint32_
   return madam_update<false>(a.s, w, g, m, v, ve).wn;
 }
 
-// STAGED: every input of this group is in the stage at `st` (thread c) and
-// the stage is released only after this returns, so the rare exact branch
-// recomputes from there and the new moments are stored right after the
-// update -- fewer values live in registers through the encode.
-template <int GD, int MD, bool SR, bool OPT, bool STAGED>
+// One element's canonical weight recomputed from global memory after the
+// stage has been released: its code (this thread overwrites it only once the
+// group is done), its gradient, and the binary32 moments this thread stored
+// right after the update.  Those are the values the canonical sequence feeds
+// into the weight update, so this serves binary32 moments only (BF16 moments
+// are stored rounded).  L2-only loads: the moments were written by this
+// thread.  Out of line: the call is rare and its pointers would otherwise stay
+// live through the encode.
+template <int GD>
+__device__ __noinline__ float fp4_exact_from_global(const StepArgs& a, const TensorCtx& x, int64_t e,
+                                                    float d_old) {
+  const uint8_t* pw = static_cast<const uint8_t*>(x.d.w) + (e >> 1);
+  uint32_t byte, bg, bm, bv, be;
+  asm volatile("ld.global.cg.u8 %0, [%1];" : "=r"(byte) : "l"(pw) : "memory");
+  const float w = __fmul_rn(e2m1_value((e & 1) ? (byte >> 4) : (byte & 0xFu)), d_old);
+  if (GD == kF32) {
+    asm volatile("ld.global.cg.u32 %0, [%1];" : "=r"(bg) : "l"(static_cast<const float*>(x.g) + e) : "memory");
+  } else {
+    asm volatile("ld.global.cg.u16 %0, [%1];" : "=r"(bg) : "l"(static_cast<const uint16_t*>(x.g) + e) : "memory");
+    bg <<= 16;
+  }
+  asm volatile("ld.global.cg.u32 %0, [%1];" : "=r"(bm) : "l"(static_cast<const float*>(x.d.m) + e) : "memory");
+  asm volatile("ld.global.cg.u32 %0, [%1];" : "=r"(bv) : "l"(static_cast<const float*>(x.d.v) + e) : "memory");
+  asm volatile("ld.global.cg.u32 %0, [%1];" : "=r"(be) : "l"(static_cast<const float*>(x.d.ve) + e) : "memory");
+  return madam_wn_exact(a.s, w, __uint_as_float(bg), __uint_as_float(bm), __uint_as_float(bv), __uint_as_float(be));
+}
+
+// Where the rare exact branch of finish_fp4 finds an element's inputs:
+// kExactRegs -- still in registers (the moments are stored at the end);
+// kExactStage -- in the stage at `st` (thread c), kept until the group is done;
+// kExactGlobal -- in global memory (binary32 moments only; the stage has
+// already been released).  The last two store the new moments right after
+// the update, so fewer values live in registers through the encode.
+constexpr int kExactRegs = 0, kExactStage = 1, kExactGlobal = 2;
+
+template <int GD, int MD, bool SR, bool OPT, int SRC>
 __device__ __forceinline__ void finish_fp4(const StepArgs& a, const TensorCtx& x, int64_t e0, int valid,
                                            uint32_t c_old, float (&w)[8], float (&g)[8], float (&m)[8],
                                            float (&v)[8], float (&ve)[8], uint32_t st, int c) {
@@ -1107,11 +1176,13 @@ __device__ __forceinline__ void finish_fp4(const StepArgs& a, const TensorCtx& x
   const float d_old = __fmul_rn(e4m3_value(c_old), G);
   const uint64_t gi = static_cast<uint64_t>(x.d.goff + e0) >> 3;  // global group index (random lanes)
   const uint32_t vmask = valid >= kGroup ? 0xFFu : (valid > 0 ? (1u << valid) - 1u : 0u);
-  uint32_t code[8];
+  uint32_t packed = 0u;  // element j's code in bits [4j, 4j + 4)
   uint32_t c_new;
   float d;
+  static_assert(SRC != kExactGlobal || MD == kF32, "exact recompute from global needs binary32 moments");
   auto exact_wn = [&](int j) -> float {
-    if constexpr (STAGED) return fp4_exact_from_stage<GD, MD>(a, st, c, j, d_old);
+    if constexpr (SRC == kExactStage) return fp4_exact_from_stage<GD, MD>(a, st, c, j, d_old);
+    else if constexpr (SRC == kExactGlobal) return fp4_exact_from_global<GD>(a, x, e0 + j, d_old);
     else return madam_wn_exact(a.s, w[j], g[j], m[j], v[j], ve[j]);
   };
   if (!OPT && a.s.cert_ok) {
@@ -1134,17 +1205,17 @@ __device__ __forceinline__ void finish_fp4(const StepArgs& a, const TensorCtx& x
         if ((vmask >> j) & 1u) am = fmaxf(am, fabsf(u.wn));
       }
     }
-    if constexpr (STAGED) put_moments<MD>(x, e0, valid, m, v, ve);
+    if constexpr (SRC != kExactRegs) put_moments<MD>(x, e0, valid, m, v, ve);
     bad &= vmask;
     const float lo_t = bad ? 0.0f : fmaxf(__fsub_rd(am, et), 0.0f);
     const float hi_t = bad ? INFINITY : __fadd_ru(am, et);
     const uint32_t plo = pair_max(__float_as_uint(lo_t));
     const uint32_t phi = pair_max(__float_as_uint(hi_t));
-    const uint32_t cl = nvfp4_scale_code(__uint_as_float(plo), G, c_old);
+    const Fp4Code cl = nvfp4_scale_code(__uint_as_float(plo), G, c_old);
     // the upper bound has the same code iff that code still covers it (or is the top one)
     const bool certain = plo != 0u && phi < 0x7E800000u /* 2^126 */ &&
-                         (cl == 126u || fp4_covers(cl, G, __uint_as_float(phi)));
-    c_new = cl;
+                         (cl.c == 126u || cl.p >= __uint_as_float(phi));
+    Fp4Code cn = cl;
     if (__any_sync(0xFFFFFFFFu, !certain)) {  // exact block maximum for the undecided pairs
       uint32_t amx = 0u;
       if (!certain) {
@@ -1157,9 +1228,10 @@ __device__ __forceinline__ void finish_fp4(const StepArgs& a, const TensorCtx& x
         }
       }
       amx = pair_max(amx);
-      if (!certain) c_new = nvfp4_scale_code(__uint_as_float(amx), G, c_old);
+      if (!certain) cn = nvfp4_scale_code(__uint_as_float(amx), G, c_old);
     }
-    d = __fmul_rn(e4m3_value(c_new), G);
+    c_new = cn.c;
+    d = __fmul_rn(e4m3_value(c_new), G);  // = cn.d, recomputed: fewer values live across the branch
     uint32_t redo = bad;
     if (d >= 1.1754943508222875e-38f /* 2^-126 */ && d <= 8.507059173023462e+37f /* 2^126 */) {
       // w' / d for w' in [wf - et, wf + et]: q = wf * inv (inv = rcp.approx(d),
@@ -1168,30 +1240,37 @@ __device__ __forceinline__ void finish_fp4(const StepArgs& a, const TensorCtx& x
       float inv;
       asm("rcp.approx.f32 %0, %1;" : "=f"(inv) : "f"(d));
       const float ei = __fmaf_ru(et, __fmul_ru(inv, 1.0000009536743164f /* 1 + 2^-20 */), 1.1754943508222875e-38f);
-      float xl[8], xh[8];
-#pragma unroll
-      for (int j = 0; j < kGroup; ++j) {
+      auto ends = [&](int j, float& xl, float& xh) {
         const float q = __fmul_rn(wf[j], inv);
         const float e2 = __fmaf_ru(fabsf(q), 9.5367431640625e-07f /* 2^-20 */, ei);
-        xl[j] = __fsub_rd(q, e2);
-        xh[j] = __fadd_ru(q, e2);
-      }
+        xl = __fsub_rd(q, e2);
+        xh = __fadd_ru(q, e2);
+      };
       if (SR) {
         uint32_t rnd[8];
         group_random_bits<kNVFP4>(a, gi << 3, rnd);
 #pragma unroll
         for (int j = 0; j < kGroup; ++j) {
+          float xl, xh;
+          ends(j, xl, xh);
           bool same;
-          code[j] = e2m1_pair_sr(xl[j], xh[j], rnd[j], same);
+          packed |= (e2m1_pair_sr(xl, xh, rnd[j], same) & 0xFu) << (4 * j);
           if (!same) redo |= 1u << j;
         }
-      } else {
-        const uint32_t pl = e2m1x8_rn(xl), diff = pl ^ e2m1x8_rn(xh);
+      } else {  // two elements at a time, both ends
+        uint32_t diff = 0u;
 #pragma unroll
-        for (int j = 0; j < kGroup; ++j) {
-          code[j] = (pl >> (4 * j)) & 0xFu;
-          if ((diff >> (4 * j)) & 0xFu) redo |= 1u << j;
+        for (int i = 0; i < kGroup / 2; ++i) {
+          float l0, h0, l1, h1;
+          ends(2 * i, l0, h0);
+          ends(2 * i + 1, l1, h1);
+          const uint32_t bl = e2m1x2_rn(l0, l1);
+          packed |= bl << (8 * i);
+          diff |= (bl ^ e2m1x2_rn(h0, h1)) << (8 * i);
         }
+#pragma unroll
+        for (int j = 0; j < kGroup; ++j)
+          if ((diff >> (4 * j)) & 0xFu) redo |= 1u << j;
       }
     } else {
       redo = 0xFFu;
@@ -1204,11 +1283,11 @@ __device__ __forceinline__ void finish_fp4(const StepArgs& a, const TensorCtx& x
       for (int j = 0; j < kGroup; ++j) {
         if ((redo >> j) & 1u) {
           const float xe = __fdiv_rn(exact_wn(j), d);
-          code[j] = e2m1_encode<SR>(xe, SR ? rnd[j] : 0u);
+          packed = (packed & ~(0xFu << (4 * j))) | ((e2m1_encode<SR>(xe, SR ? rnd[j] : 0u) & 0xFu) << (4 * j));
         }
       }
     }
-    if constexpr (!STAGED) put_moments<MD>(x, e0, valid, m, v, ve);
+    if constexpr (SRC == kExactRegs) put_moments<MD>(x, e0, valid, m, v, ve);
   } else {
     float wn[8];
     uint32_t amx = 0u;
@@ -1219,17 +1298,16 @@ __device__ __forceinline__ void finish_fp4(const StepArgs& a, const TensorCtx& x
       const uint32_t bb = __float_as_uint(u.wn) & 0x7FFFFFFFu;
       if (((vmask >> j) & 1u) && bb < 0x7F800000u) amx = max(amx, bb);
     }
-    c_new = nvfp4_scale_code(__uint_as_float(pair_max(amx)), G, c_old);
-    d = __fmul_rn(e4m3_value(c_new), G);
+    const Fp4Code cn = nvfp4_scale_code(__uint_as_float(pair_max(amx)), G, c_old);
+    c_new = cn.c;
+    d = cn.d;
     uint32_t rnd[8];
     if (SR) group_random_bits<kNVFP4>(a, gi << 3, rnd);
 #pragma unroll
-    for (int j = 0; j < kGroup; ++j) code[j] = e2m1_encode<SR>(__fdiv_rn(wn[j], d), SR ? rnd[j] : 0u);
+    for (int j = 0; j < kGroup; ++j)
+      packed |= (e2m1_encode<SR>(__fdiv_rn(wn[j], d), SR ? rnd[j] : 0u) & 0xFu) << (4 * j);
     put_moments<MD>(x, e0, valid, m, v, ve);
   }
-  uint32_t packed = 0u;
-#pragma unroll
-  for (int j = 0; j < kGroup; ++j) packed |= (code[j] & 0xFu) << (4 * j);
   put_fp4(packed, x.d.w, e0, valid, x.vec);
   if ((threadIdx.x & 1) == 0 && valid > 0) static_cast<uint8_t*>(x.scale)[e0 / kFp4Block] = static_cast<uint8_t>(c_new);
   if (x.cc) {
@@ -1298,7 +1376,7 @@ __device__ __noinline__ void general_fp4_group(const StepArgs& a, const TensorCt
     get_bf16<false>(v, v_st, st + a.off_v + kGroup * MS * c, x.d.v, e0, valid, x.vec);
     get_bf16<false>(ve, e_st, st + a.off_ve + kGroup * MS * c, x.d.ve, e0, valid, x.vec);
   }
-  finish_fp4<GD, MD, SR, OPT, false>(a, x, e0, valid, s_old, w, g, m, v, ve, st, c);
+  finish_fp4<GD, MD, SR, OPT, kExactRegs>(a, x, e0, valid, s_old, w, g, m, v, ve, st, c);
 }
 
 // ---------------------------------------------------------------------------
@@ -1460,9 +1538,15 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
         get_bf16<false>(v, true, st + a.off_v + kGroup * MS * c, x.d.v, e0, kGroup, true);
         get_bf16<false>(ve, true, st + a.off_ve + kGroup * MS * c, x.d.ve, e0, kGroup, true);
       }
-      if constexpr (WD == kNVFP4) {
-        // the stage stays until the group is done (its exact branch re-reads it)
-        finish_fp4<GD, MD, SR, OPT, true>(a, x, e0, kGroup, h_old, w, g, m, v, ve, st, c);
+      if constexpr (WD == kNVFP4 && MD == kF32) {
+        // released at once: the rare exact branch re-reads global memory
+        __syncwarp();
+        if (lane == 0) mbar_arrive(smem_addr(&empty_bar[s]));
+        finish_fp4<GD, MD, SR, OPT, kExactGlobal>(a, x, e0, kGroup, h_old, w, g, m, v, ve, st, c);
+      } else if constexpr (WD == kNVFP4) {
+        // BF16 moments: the stage stays until the group is done (its exact
+        // branch re-reads the binary32 originals there)
+        finish_fp4<GD, MD, SR, OPT, kExactStage>(a, x, e0, kGroup, h_old, w, g, m, v, ve, st, c);
         __syncwarp();
         if (lane == 0) mbar_arrive(smem_addr(&empty_bar[s]));
       } else {
@@ -1480,8 +1564,8 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
     else if constexpr (WD == kNVFP4)
       general_fp4_group<GD, MD, SR, OPT>(a, x, tile_e0, count, c, smem0 + static_cast<uint32_t>(s * a.stage_bytes));
     else
-      general_group<WD, GD, MD, SR, OPT>(a, x, tile_e0, count, c, smem0 + static_cast<uint32_t>(s * a.stage_bytes),
-                                         amax_bits);
+      amax_bits = general_group<WD, GD, MD, SR, OPT>(a, x, tile_e0, count, c,
+                                                     smem0 + static_cast<uint32_t>(s * a.stage_bytes), amax_bits);
     __syncwarp();
     if (lane == 0) mbar_arrive(smem_addr(&empty_bar[s]));
     if (++s == S) { s = 0; ++use; }

@@ -128,9 +128,13 @@ def test_nvfp4_block_maxima_at_the_top_code(lr):
         r.close()
 
 
-def test_nvfp4_nan_inf_and_odd_scales():
+@pytest.mark.parametrize("md", ["bf16", "f32"])
+def test_nvfp4_nan_inf_and_odd_scales(md):
+    """Non-finite inputs and odd block scales send elements to the exact
+    branch: re-read from the stage (BF16 moments) or from global memory
+    (binary32 moments, the stage already released)."""
     p = P()
-    wl = _fp4(md="bf16")
+    wl = _fp4(md=md)
     mt = W.materialize(wl, "cpu", warm_state=True)
     big = max(range(len(mt.g)), key=lambda k: mt.g[k].numel())
     g = mt.g[big]
