@@ -239,8 +239,11 @@ def run_gpu(wl, steps: int, warmup: int, rank: int, e2e_steps: int, flush_l2: bo
     starts = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
     ends = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
     region0, region1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    # lists that fit in L2 (129 MB): a 256 MB write between launches, outside each launch's events
+    # lists that fit in L2 (129 MB): between launches, outside each launch's events, a 256 MB
+    # write and then a 256 MB read of another buffer, so that L2 holds none of the inputs and
+    # no dirty lines whose write-back the next launch would pay for
     flush = torch.empty(64 << 20, dtype=torch.float32, device=dev) if flush_l2 else None
+    flush_rd = torch.ones(64 << 20, dtype=torch.float32, device=dev) if flush_l2 else None
     if torch.distributed.is_initialized():
         torch.distributed.barrier()
     torch.cuda.synchronize()
@@ -249,6 +252,7 @@ def run_gpu(wl, steps: int, warmup: int, rank: int, e2e_steps: int, flush_l2: bo
     for i in range(steps):
         if flush is not None:
             flush.fill_(float(i))
+            flush_rd.amax()
         starts[i].record(stream)
         opt.step_ptrs(gptrs, t, stream.cuda_stream)
         ends[i].record(stream)
@@ -260,9 +264,11 @@ def run_gpu(wl, steps: int, warmup: int, rank: int, e2e_steps: int, flush_l2: bo
         torch.distributed.barrier()
     total_ms = region0.elapsed_time(region1)
     launch_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
+    copy_ms = same_size_copy_ms(algorithmic_bytes(wl), flush, flush_rd, stream) if flush is not None else None
     res = {"total_ms": total_ms, "launch_ms": launch_ms, "wall": (wall0, wall1),
-           "grid": opt.launch_info(), "launches_per_step": launches_per_step, "l2_flushed": flush is not None}
-    del flush
+           "grid": opt.launch_info(), "launches_per_step": launches_per_step, "l2_flushed": flush is not None,
+           "copy_ms": copy_ms}
+    del flush, flush_rd
 
     # end to end through the host-buffer entry point (one weight format: flat host buffers)
     if e2e_steps > 0 and "w" in mt.flat:
@@ -306,6 +312,28 @@ def run_gpu(wl, steps: int, warmup: int, rank: int, e2e_steps: int, flush_l2: bo
     torch.cuda.synchronize()
     torch.cuda.empty_cache()
     return res
+
+
+def same_size_copy_ms(nbytes: float, flush, flush_rd, stream, reps: int = 20) -> float:
+    """Median event-timed device-to-device copy moving the same bytes (half
+    read, half written) under the same flush: what a plain copy reaches at
+    this size, where launch and DRAM latency, not bandwidth, set the time."""
+    import torch
+    n = max(1, int(nbytes // 2) // 4)
+    a = torch.ones(n, dtype=torch.float32, device=stream.device)
+    b = torch.empty_like(a)
+    ts = []
+    for i in range(reps):
+        flush.fill_(float(i))
+        flush_rd.amax()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        b.copy_(a)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ts.append(e0.elapsed_time(e1))
+    del a, b
+    return sorted(ts)[len(ts) // 2]
 
 
 def pinned_kind_for_this_host(stream) -> str:
@@ -416,14 +444,15 @@ def summarize(wl, res, n_gpus, peak, peak_kind):
     n = wl.n_params
     ms = res["total_ms"] / len(res["launch_ms"])
     if res.get("l2_flushed"):   # the region also holds the flushes: time the launches alone
-        ms = sum(res["launch_ms"]) / len(res["launch_ms"])
+        ms = res.get("launch_total_ms", sum(res["launch_ms"])) / len(res["launch_ms"])
     bpp = algorithmic_bytes_per_param(wl)
     launch = sorted(res["launch_ms"])
     avg_launch = sum(launch) / len(launch)
     achieved = algorithmic_bytes(wl) / (avg_launch * 1e-3) / 1e9
     out = {
         "workload": wl.name, "params": n, "tensors": len(wl.specs),
-        "l2": "flushed between launches (256 MB write)" if res.get("l2_flushed") else "inputs larger than L2",
+        "l2": "flushed between launches (256 MB write, then 256 MB read)" if res.get("l2_flushed")
+              else "inputs larger than L2",
         "ms_per_step": ms, "gparams_per_s": whole_job_rate(n, n_gpus, ms),
         "hbm_gbs": algorithmic_bytes(wl) / (ms * 1e-3) / 1e9,
         "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
@@ -434,6 +463,10 @@ def summarize(wl, res, n_gpus, peak, peak_kind):
                      "launch_ms_min": round(launch[0], 4), "launch_ms_max": round(launch[-1], 4),
                      "launch_ms_first_last": [round(res["launch_ms"][0], 4), round(res["launch_ms"][-1], 4)]},
     }
+    if res.get("copy_ms"):
+        # context for lists that fit in L2: a plain copy of the same bytes, same flush
+        out["roofline"]["copy_same_bytes_ms"] = round(res["copy_ms"], 4)
+        out["roofline"]["frac_of_copy_same_bytes"] = round(res["copy_ms"] / avg_launch, 4)
     if "e2e_ms" in res:
         out["e2e"] = {"value": n_gpus * n / (res["e2e_ms"] * 1e-3) / 1e9, "unit": UNIT,
                       "h2d_bytes_per_step": res["h2d"], "d2h_bytes_per_step": res["d2h"],
@@ -510,9 +543,12 @@ def main():
     sampler = ClockSampler(gpu_index, out_dir / f"clocks_rank{rank}.csv") if rank == 0 else None
     time.sleep(0.3 if sampler else 0)
 
-    res = run_gpu(wl, args.steps, warmup, rank, args.e2e_steps if rank == 0 else 0)
+    res = run_gpu(wl, args.steps, warmup, rank, args.e2e_steps if rank == 0 else 0,
+                  flush_l2=algorithmic_bytes(wl) < 512e6)
     if world > 1:
         res["total_ms"] = max_over_ranks(res["total_ms"], "cuda")
+        if res.get("l2_flushed"):  # timed per launch: the slowest rank's launch total
+            res["launch_total_ms"] = max_over_ranks(sum(res["launch_ms"]), "cuda")
     clocks = sampler.summary(*res["wall"]) if sampler else None
     main_sum = summarize(wl, res, world, peak, peak_kind)
 
@@ -546,7 +582,8 @@ def main():
         "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
         "config": {"workload": wl.name, "params": wl.n_params, "tensors": len(wl.specs),
                    "weights": wl.weight_dtype, "grads": wl.grad_dtype, "moments": wl.moment_dtype,
-                   "rounding": wl.rounding, "l2": "inputs larger than L2 (no flush needed)",
+                   "rounding": wl.rounding,
+                   "l2": main_sum["l2"] if res.get("l2_flushed") else "inputs larger than L2 (no flush needed)",
                    "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
                    "grid": res["grid"][0], "threads": res["grid"][1]},
         "hbm_gbs": round(main_sum["hbm_gbs"], 1),
