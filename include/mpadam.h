@@ -294,6 +294,21 @@ int32_t mpadam_global_length(const mpadam_state* s, int64_t* length);
 int32_t mpadam_set_grid(mpadam_state* s, int32_t ctas);
 int32_t mpadam_launch_info(const mpadam_state* s, int32_t* ctas, int32_t* threads);
 
+/* Work balance of mpadam_step's launches.  Each CTA owns an equal run of
+ * tiles (3840 elements each).  It keeps the first static_q / 1024 of that
+ * run; the rest of every run goes to a pool of chunks of at most
+ * chunk_tiles tiles, which the CTAs that finish first claim one at a time.
+ * SMs do not all stream memory at the same rate, so without the pool a
+ * launch waits on the slowest.  static_q = 1024 turns the pool off.
+ * Default: static_q = 768, chunk_tiles = 4, except that lists' per-tensor
+ * scaled E4M3 tensors keep static runs until this is called (they measured
+ * slower with the pool).  Results do not depend on either value.
+ * Synchronises the device.  The host-buffer and allocation-free entry
+ * points always use static runs.
+ * Errors: EINVAL (static_q outside [0, 1024], chunk_tiles outside
+ * [1, 2^20]), EALLOC, ECUDA. */
+int32_t mpadam_set_tail_pool(mpadam_state* s, int32_t static_q, int32_t chunk_tiles);
+
 /* Device-side status of the steps issued so far: synchronises the device,
  * returns in *code the error bits the step kernel recorded (0 = none; a
  * non-zero value means a bounded wait inside the kernel gave up and that

@@ -22,7 +22,7 @@ ROUNDING = {"nearest": MPADAM_ROUND_NEAREST, "stochastic": MPADAM_ROUND_STOCHAST
 
 EXPORTED = ["mpadam_create", "mpadam_create_ex", "mpadam_fp8_init", "mpadam_step", "mpadam_step_host",
             "mpadam_destroy", "mpadam_last_error", "mpadam_global_offset", "mpadam_global_length", "mpadam_set_grid",
-            "mpadam_launch_info", "mpadam_rng_lanes", "mpadam_step_noalloc", "mpadam_device_status",
+            "mpadam_set_tail_pool", "mpadam_launch_info", "mpadam_rng_lanes", "mpadam_step_noalloc", "mpadam_device_status",
             "mpadam_toy_create", "mpadam_toy_step", "mpadam_toy_run", "mpadam_toy_destroy", "mpadam_host_buffer_alloc",
             "mpadam_host_buffer_free", "mpadam_debug_fail_allocation"]
 
@@ -110,6 +110,7 @@ def lib() -> ctypes.CDLL:
             "mpadam_global_offset": [P, i32, P],
             "mpadam_global_length": [P, P],
             "mpadam_set_grid": [P, i32],
+            "mpadam_set_tail_pool": [P, i32, i32],
             "mpadam_launch_info": [P, P, P],
             "mpadam_rng_lanes": [u64, i64, i32, i64, i64, P, P],
             "mpadam_step_noalloc": [P, i32, P, P, P, P, i64, P],
@@ -208,6 +209,10 @@ def mpadam_global_length(state: int) -> int:
 
 def mpadam_set_grid(state: int, ctas: int) -> None:
     _check(lib().mpadam_set_grid(state, ctas))
+
+
+def mpadam_set_tail_pool(state: int, static_q: int, chunk_tiles: int) -> None:
+    _check(lib().mpadam_set_tail_pool(state, static_q, chunk_tiles))
 
 
 def mpadam_launch_info(state: int) -> tuple:

@@ -293,6 +293,8 @@ struct Group {
   int32_t default_grid = 0, grid = 0;
   int32_t* d_cta_first = nullptr;
   int32_t cta_cap = 0;
+  mpadam::PoolChunk* d_pool = nullptr;  // tail pool of the current grid (none when static_q is 1024)
+  int32_t pool_chunks = 0, pool_cap = 0;
 };
 
 struct mpadam_state {
@@ -325,6 +327,12 @@ struct mpadam_state {
   std::vector<int64_t> chunk_tile;            // chunk c covers tiles [chunk_tile[c], chunk_tile[c+1])
   std::vector<int64_t> chunk_elem;            // and global elements [chunk_elem[2c], chunk_elem[2c+1])
   int32_t* d_chunk_first = nullptr;           // [chunks][grid] CTA start tensors
+  // tail pool of mpadam_step's launches: static prefix of each CTA's range (1/1024) and chunk length.
+  // Until set_tail_pool is called, per-tensor-scaled E4M3 groups keep static ranges: measured
+  // slower with the pool (the other formats gain 3-12 %).
+  int32_t pool_q = 768, pool_chunk = 4;
+  bool pool_set = false;
+  uint32_t* d_pool_next = nullptr;            // [groups] claim counters, zeroed before each step
 };
 
 namespace {
@@ -346,8 +354,11 @@ void release(mpadam_state* s) {
   if (s->d_desc) cudaFree(s->d_desc);
   if (s->d_aux) cudaFree(s->d_aux);
   if (s->d_grads) cudaFree(const_cast<void**>(s->d_grads));
-  for (auto& g : s->groups)
+  for (auto& g : s->groups) {
     if (g.d_cta_first) cudaFree(g.d_cta_first);
+    if (g.d_pool) cudaFree(g.d_pool);
+  }
+  if (s->d_pool_next) cudaFree(s->d_pool_next);
   if (s->d_err) cudaFree(s->d_err);
   if (s->d_gstage) cudaFree(s->d_gstage);
   release_pipeline(s);
@@ -391,6 +402,55 @@ int32_t upload_cta_table(Group& g, int32_t grid) {
   return MPADAM_OK;
 }
 
+// The tail pool of a group for `grid` CTAs: CTA b keeps the first
+// (te - tb) * q / 1024 tiles of its range [tb, te) (the kernel computes the
+// same split) and the rest of every range becomes chunks of at most `chunk`
+// tiles, in tile order.
+int32_t upload_pool(Group& g, int32_t grid, int32_t q, int32_t chunk) {
+  g.pool_chunks = 0;
+  if (q >= 1024 || g.tiles == 0) return MPADAM_OK;
+  std::vector<mpadam::PoolChunk> pool;
+  int32_t k = 0;
+  int64_t tile_off = 0;
+  auto tensor_of = [&](int64_t t) {  // t never decreases across calls
+    while (k < g.count && tile_off + tiles_of(g.numel[k]) <= t) {
+      tile_off += tiles_of(g.numel[k]);
+      ++k;
+    }
+    return k;
+  };
+  for (int32_t b = 0; b < grid; ++b) {
+    const int64_t tb = (int64_t)b * g.tiles / grid, te = ((int64_t)b + 1) * g.tiles / grid;
+    for (int64_t t = tb + (te - tb) * q / 1024; t < te; t += chunk) {
+      mpadam::PoolChunk pc;
+      pc.start = t;
+      pc.count = (int32_t)std::min<int64_t>(chunk, te - t);
+      pc.first = tensor_of(t);
+      pool.push_back(pc);
+    }
+  }
+  if (pool.size() > (size_t)INT32_MAX) return fail(MPADAM_EINVAL, "tail pool too large");
+  if ((int32_t)pool.size() > g.pool_cap) {
+    if (g.d_pool) cudaFree(g.d_pool);
+    g.d_pool = nullptr;
+    g.pool_cap = 0;
+    if (dev_malloc(&g.d_pool, sizeof(mpadam::PoolChunk) * pool.size()) != cudaSuccess)
+      return fail(MPADAM_EALLOC, "cudaMalloc of %zu tail-pool chunks failed", pool.size());
+    g.pool_cap = (int32_t)pool.size();
+  }
+  if (!pool.empty()) {
+    cudaError_t e = cudaMemcpy(g.d_pool, pool.data(), sizeof(mpadam::PoolChunk) * pool.size(), cudaMemcpyHostToDevice);
+    if (e != cudaSuccess) return cuda_fail(e, "upload of the tail pool");
+  }
+  g.pool_chunks = (int32_t)pool.size();
+  return MPADAM_OK;
+}
+
+// The static share a group's launches use.
+int32_t pool_q_of(const mpadam_state* s, const Group& g) {
+  return g.wd == MPADAM_E4M3 && !s->pool_set ? 1024 : s->pool_q;
+}
+
 void fill_common(StepArgs& a, const mpadam_config& cfg, const Geometry& geo, int64_t total_tiles, int32_t n,
                  int32_t* fp8_exp, uint32_t* fp8_amax) {
   std::memset(&a, 0, sizeof a);
@@ -406,6 +466,7 @@ void fill_common(StepArgs& a, const mpadam_config& cfg, const Geometry& geo, int
   round_keys(cfg.seed, a.rk0, a.rk1);
   a.fp8_exp = fp8_exp;
   a.fp8_amax = fp8_amax;
+  a.static_q = 1024;  // static ranges only unless a launch brings a tail pool
 }
 
 void fill_step(StepArgs& a, const mpadam_config& cfg, int64_t step) {
@@ -580,6 +641,7 @@ int32_t create_state(const std::vector<TensorIn>& t, const mpadam_config* cfg, i
         dev_malloc(reinterpret_cast<void**>(&s->d_grads), sizeof(void*) * nn) != cudaSuccess ||
         (any_aux && dev_malloc(&s->d_aux, sizeof(TensorAux) * nn) != cudaSuccess) ||
         dev_malloc(&s->d_err, sizeof(int32_t)) != cudaSuccess ||
+        dev_malloc(&s->d_pool_next, sizeof(uint32_t) * std::max<size_t>(1, s->groups.size())) != cudaSuccess ||
         host_malloc(reinterpret_cast<void**>(&s->h_grads), sizeof(void*) * nn) != cudaSuccess) {
       release(s);
       return fail(MPADAM_EALLOC, "allocation of the tensor tables failed");
@@ -598,6 +660,7 @@ int32_t create_state(const std::vector<TensorIn>& t, const mpadam_config* cfg, i
     }
     for (auto& g : s->groups) {
       rc = upload_cta_table(g, g.default_grid);
+      if (!rc) rc = upload_pool(g, g.grid, pool_q_of(s, g), s->pool_chunk);
       if (rc) { release(s); return rc; }
     }
   } catch (const std::bad_alloc&) {
@@ -630,11 +693,17 @@ int32_t upload_grad_table(mpadam_state* s, const void* const* grads, cudaStream_
 
 // One launch of a group's step kernel over its tiles [tile_base, tile_base + count).
 int32_t launch_step(mpadam_state* s, const Group& g, int64_t step, cudaStream_t stream, int64_t tile_base,
-                    int64_t count, const int32_t* cta_first, int32_t grid) {
+                    int64_t count, const int32_t* cta_first, int32_t grid, uint32_t* pool_next = nullptr) {
   StepArgs a = base_args(s, g);
   a.cta_first = cta_first;
   a.tile_base = tile_base;
   a.total_tiles = count;
+  if (pool_next && g.pool_chunks > 0) {  // whole-group launches only: the pool covers all of its tiles
+    a.pool = g.d_pool;
+    a.pool_next = pool_next;
+    a.pool_chunks = g.pool_chunks;
+    a.static_q = pool_q_of(s, g);
+  }
   fill_step(a, s->cfg, step);
   void* params[] = {&a};
   cudaError_t e = cudaLaunchKernel(g.kernel, dim3(grid), dim3(mpadam::kThreads), params, (size_t)g.geo.dyn_smem,
@@ -770,6 +839,25 @@ int32_t mpadam_set_grid(mpadam_state* s, int32_t ctas) {
   release_pipeline(s);  // the host-buffer pipeline's per-chunk tables follow the grid: rebuilt on next use
   for (auto& g : s->groups) {
     rc = upload_cta_table(g, ctas == 0 ? g.default_grid : ctas);
+    if (!rc) rc = upload_pool(g, g.grid, pool_q_of(s, g), s->pool_chunk);
+    if (rc) return rc;
+  }
+  return MPADAM_OK;
+}
+
+int32_t mpadam_set_tail_pool(mpadam_state* s, int32_t static_q, int32_t chunk_tiles) {
+  if (!s) return fail(MPADAM_EINVAL, "state is NULL");
+  if (static_q < 0 || static_q > 1024) return fail(MPADAM_EINVAL, "static_q must be in [0, 1024]");
+  if (chunk_tiles < 1 || chunk_tiles > (1 << 20)) return fail(MPADAM_EINVAL, "chunk_tiles must be in [1, 2^20]");
+  int32_t rc = check_device(s);
+  if (rc) return rc;
+  cudaError_t e = cudaDeviceSynchronize();  // the old pool may be in use
+  if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceSynchronize");
+  s->pool_q = static_q;
+  s->pool_chunk = chunk_tiles;
+  s->pool_set = true;
+  for (auto& g : s->groups) {
+    rc = upload_pool(g, g.grid, pool_q_of(s, g), s->pool_chunk);
     if (rc) return rc;
   }
   return MPADAM_OK;
@@ -812,9 +900,16 @@ int32_t mpadam_step(mpadam_state* s, const void* const* grads, int64_t step, cud
   if (rc) return rc;
   rc = upload_grad_table(s, grads, stream);
   if (rc) return rc;
-  for (const auto& g : s->groups) {
+  bool pooled = false;
+  for (const auto& g : s->groups) pooled = pooled || g.pool_chunks > 0;
+  if (pooled) {  // the pools' claim counters start at zero
+    cudaError_t e = cudaMemsetAsync(s->d_pool_next, 0, sizeof(uint32_t) * s->groups.size(), stream);
+    if (e != cudaSuccess) return cuda_fail(e, "clearing the tail-pool counters");
+  }
+  for (size_t i = 0; i < s->groups.size(); ++i) {
+    const Group& g = s->groups[i];
     if (g.tiles == 0) continue;
-    rc = launch_step(s, g, step, stream, 0, g.tiles, g.d_cta_first, g.grid);
+    rc = launch_step(s, g, step, stream, 0, g.tiles, g.d_cta_first, g.grid, s->d_pool_next + i);
     if (rc) return rc;
   }
   return MPADAM_OK;

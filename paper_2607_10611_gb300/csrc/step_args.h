@@ -11,6 +11,14 @@
 // order starting at tensor cta_first[b].  Inside a tile, consumer thread c
 // owns the 8 elements [8c, 8c + 8).
 //
+// Tail pool.  A launch may keep only a prefix of each CTA's range static:
+// CTA b then walks [tb, tb + (te - tb) * static_q / 1024) and the rest of
+// every range is cut into PoolChunks, handed out in order by an atomic
+// counter to whichever CTA runs out of work first.  SMs do not all stream
+// at the same rate, so a fixed split leaves the kernel waiting on the
+// slowest; the pool evens out the end.  The producer warp decides each
+// tile and posts its index and tensor beside the stage.
+//
 // Element indices for stochastic rounding are independent of this
 // decomposition: element j of tensor k has global index goff[k] + j, where
 // goff[0] = 0 and goff[k+1] = goff[k] + numel[k] rounded up to a multiple of 8.
@@ -91,6 +99,14 @@ struct StepScalars {
   int32_t cert_ok;   // eps >= 2^-28, tau >= 2^-125, c2 <= 2^14, eta_m <= 4: certified fast path allowed
 };
 
+// A run of consecutive tiles of the tail pool.
+struct PoolChunk {
+  int64_t start;  // first tile (this launch's numbering)
+  int32_t count;  // tiles
+  int32_t first;  // tensor holding tile `start`
+};
+static_assert(sizeof(PoolChunk) == 16, "PoolChunk must stay 16 bytes");
+
 struct StepArgs {
   const TensorDesc* desc;    // [n_tensors]
   const void* const* grads;  // [n_tensors] device pointers
@@ -111,8 +127,12 @@ struct StepArgs {
   uint32_t* fp8_amax;        // [3][n_tensors] binary32 bits
   int32_t e_cur_slot, e_next_slot;
   int32_t a_cur_slot, a_next_slot, a_zero_slot;
-  int32_t pad1;
+  int32_t static_q;          // static prefix of each CTA's range, in 1/1024 (1024 when pool is nullptr)
   int32_t* err;              // DeviceError bits, or nullptr
+  const PoolChunk* pool;     // [pool_chunks] tail pool, or nullptr (static ranges only)
+  uint32_t* pool_next;       // next unclaimed pool chunk; zero when the launch starts
+  int32_t pool_chunks;
+  int32_t pad2;
 };
 
 // Kernel entry for the given formats (grad f32/bf16, moments f32/bf16,

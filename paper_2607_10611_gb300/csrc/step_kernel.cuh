@@ -1388,6 +1388,8 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
   extern __shared__ __align__(128) uint8_t smem[];
   __shared__ __align__(8) uint64_t full_bar[kMaxStages];
   __shared__ __align__(8) uint64_t empty_bar[kMaxStages];
+  __shared__ int64_t stage_tile[kMaxStages];  // tile the producer put in each stage (-1: no more work)
+  __shared__ int32_t stage_k[kMaxStages];     // and its tensor
 
   const int tid = threadIdx.x;
   const int warp = tid >> 5, lane = tid & 31;
@@ -1404,30 +1406,44 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
   const int64_t T = a.total_tiles;
   const int64_t tb = a.tile_base + static_cast<int64_t>(blockIdx.x) * T / gridDim.x;
   const int64_t te = a.tile_base + (static_cast<int64_t>(blockIdx.x) + 1) * T / gridDim.x;
-  if (tb >= te) return;
+  if (tb >= te && !a.pool) return;
+  // static part of the range; the rest went to the tail pool
+  const int64_t ts = a.pool ? tb + (te - tb) * a.static_q / 1024 : te;
   const uint32_t smem0 = smem_addr(smem);
 
   // ------------------------------------------------------------ producer --
   if (warp == kConsumerWarps) {
     if (lane != 0) return;
     const uint64_t pol = evict_first_policy();
-    int k = a.cta_first[blockIdx.x];
-    TensorDesc d = a.desc[k];
-    const void* gp = a.grads[k];
-    const uint8_t* sp = (WD == kE4M3B || WD == kNVFP4) ? static_cast<const uint8_t*>(a.aux[k].scale) : nullptr;
-    int64_t tiles = (d.numel + kTile - 1) / kTile;
+    int k = -1;
+    TensorDesc d{};
+    const void* gp = nullptr;
+    const uint8_t* sp = nullptr;
+    int64_t tiles = 0;
+    auto load = [&](int kk) {
+      k = kk;
+      d = a.desc[k];
+      gp = a.grads[k];
+      if (WD == kE4M3B || WD == kNVFP4) sp = static_cast<const uint8_t*>(a.aux[k].scale);
+      tiles = (d.numel + kTile - 1) / kTile;
+    };
+    int64_t t = tb, t_end = ts;  // the current run of consecutive tiles
+    if (t < t_end) load(a.cta_first[blockIdx.x]);
     int s = 0;
     uint32_t use = 0;
     int64_t issued = 0;
     bool failed = false;
-    for (int64_t t = tb; t < te; ++t) {
-      while (t >= d.tile_off + tiles) {
-        ++k;
-        d = a.desc[k];
-        gp = a.grads[k];
-        if (WD == kE4M3B || WD == kNVFP4) sp = static_cast<const uint8_t*>(a.aux[k].scale);
-        tiles = (d.numel + kTile - 1) / kTile;
+    for (;;) {
+      if (t >= t_end) {  // static part done: next chunk of the tail pool, if any
+        if (!a.pool) break;
+        const uint32_t j = atomicAdd(a.pool_next, 1u);
+        if (j >= static_cast<uint32_t>(a.pool_chunks)) break;
+        const PoolChunk pc = a.pool[j];
+        t = pc.start;
+        t_end = pc.start + pc.count;
+        if (pc.first != k) load(pc.first);
       }
+      while (t >= d.tile_off + tiles) load(k + 1);
       if (use > 0 && !mbar_wait(smem_addr(&empty_bar[s]), (use - 1) & 1u)) {
         if (a.err) atomicOr(a.err, kErrEmptyWait);
         failed = true;
@@ -1446,6 +1462,8 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
                                          : 0u;
       const uint32_t bar = smem_addr(&full_bar[s]);
       const uint32_t st = smem0 + static_cast<uint32_t>(s * a.stage_bytes);
+      stage_tile[s] = t;  // published by the arrive below (release)
+      stage_k[s] = k;
       mbar_arrive_expect_tx(bar, nw + ng + nm + nv + nve + ns);
       if (nw) tma_load(st, static_cast<const uint8_t*>(d.w) + (WD == kNVFP4 ? e0 / 2 : e0 * WS), nw, bar, pol);
       if (ng) tma_load(st + a.off_g, static_cast<const uint8_t*>(gp) + e0 * GS, ng, bar, pol);
@@ -1454,6 +1472,7 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
       if (nve) tma_load(st + a.off_ve, static_cast<const uint8_t*>(d.ve) + e0 * MS, nve, bar, pol);
       if (ns) tma_load(st + a.off_s, sp + s0, ns, bar, pol);
       ++issued;
+      ++t;
       if (++s == S) { s = 0; ++use; }
     }
     if (failed) {  // wait (bounded) for this CTA's copies still in flight, then leave
@@ -1463,36 +1482,44 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
         if (!mbar_wait(smem_addr(&full_bar[it % S]), static_cast<uint32_t>((it / S) & 1)) && a.err)
           atomicOr(a.err, kErrDrainWait);
       }
+      return;
     }
+    // no more work: once the next stage is free, post the end marker there
+    if (use > 0 && !mbar_wait(smem_addr(&empty_bar[s]), (use - 1) & 1u)) {
+      if (a.err) atomicOr(a.err, kErrEmptyWait);
+      return;
+    }
+    stage_tile[s] = -1;
+    mbar_arrive(smem_addr(&full_bar[s]));
     return;
   }
 
   // ----------------------------------------------------------- consumers --
   const int c = tid;  // consumer index, owns elements [8c, 8c + 8) of every tile
   const int n = a.n_tensors;
-  int k = a.cta_first[blockIdx.x];
+  int k = -1;
   TensorCtx x;
-  load_tensor<WD, GD, MD>(a, k, x);
   int32_t e_next = 0;
-  if (WD == kE4M3) {
-    const int32_t e_cur = a.fp8_exp[static_cast<int64_t>(a.e_cur_slot) * n + x.d.ring];
-    e_next = fp8_next_exponent(a.fp8_amax[static_cast<int64_t>(a.a_cur_slot) * n + x.d.ring], e_cur);
-    x.dec_scale = pow2f(e_cur);
-    x.enc_scale = pow2f(-e_next);
-    x.cc_scale = pow2f(e_next);
-  }
   uint32_t amax_bits = 0u;
   int s = 0;
   uint32_t use = 0;
-  for (int64_t t = tb; t < te; ++t) {
-    if (t >= x.d.tile_off + x.tiles) {  // next tensor: flush this one's E4M3 amax
-      if (WD == kE4M3) {
+  for (;;) {
+    if (!__all_sync(0xFFFFFFFFu, mbar_wait(smem_addr(&full_bar[s]), use & 1u))) {  // warp-uniform give-up
+      if (a.err && lane == 0) atomicOr(a.err, kErrFullWait);
+      return;
+    }
+    const int64_t t = stage_tile[s];
+    if (t < 0) break;  // the producer's end marker
+    const int kt = stage_k[s];
+    if (kt != k) {  // another tensor: flush this one's E4M3 amax
+      if (WD == kE4M3 && k >= 0) {
         const uint32_t wmax = __reduce_max_sync(0xFFFFFFFFu, amax_bits);
         if (lane == 0 && wmax != 0u)
           atomicMax(&a.fp8_amax[static_cast<int64_t>(a.a_next_slot) * n + x.d.ring], wmax);
         amax_bits = 0u;
       }
-      do { ++k; load_tensor<WD, GD, MD>(a, k, x); } while (t >= x.d.tile_off + x.tiles);
+      k = kt;
+      load_tensor<WD, GD, MD>(a, k, x);
       if (WD == kE4M3) {
         const int32_t e_cur = a.fp8_exp[static_cast<int64_t>(a.e_cur_slot) * n + x.d.ring];
         e_next = fp8_next_exponent(a.fp8_amax[static_cast<int64_t>(a.a_cur_slot) * n + x.d.ring], e_cur);
@@ -1505,10 +1532,6 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
     if (WD == kE4M3 && tile_e0 == 0 && c == 0) {  // the CTA holding the tensor's first tile
       a.fp8_exp[static_cast<int64_t>(a.e_next_slot) * n + x.d.ring] = e_next;
       a.fp8_amax[static_cast<int64_t>(a.a_zero_slot) * n + x.d.ring] = 0u;
-    }
-    if (!__all_sync(0xFFFFFFFFu, mbar_wait(smem_addr(&full_bar[s]), use & 1u))) {  // warp-uniform give-up
-      if (a.err && lane == 0) atomicOr(a.err, kErrFullWait);
-      return;
     }
     const int count = static_cast<int>(x.d.numel - tile_e0 < kTile ? x.d.numel - tile_e0 : kTile);
     if (count == kTile && x.fast) {  // whole tile, every array staged: straight-line group
@@ -1570,7 +1593,7 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
     if (lane == 0) mbar_arrive(smem_addr(&empty_bar[s]));
     if (++s == S) { s = 0; ++use; }
   }
-  if (WD == kE4M3) {
+  if (WD == kE4M3 && k >= 0) {
     const uint32_t wmax = __reduce_max_sync(0xFFFFFFFFu, amax_bits);
     if (lane == 0 && wmax != 0u) atomicMax(&a.fp8_amax[static_cast<int64_t>(a.a_next_slot) * n + x.d.ring], wmax);
   }

@@ -140,6 +140,10 @@ class MPAdam:
     def set_grid(self, ctas: int):
         N.mpadam_set_grid(self.state, ctas)
 
+    def set_tail_pool(self, static_q: int, chunk_tiles: int):
+        """Static share (in 1/1024) of each CTA's tile run and the pool's chunk length."""
+        N.mpadam_set_tail_pool(self.state, static_q, chunk_tiles)
+
     def launch_info(self):
         return N.mpadam_launch_info(self.state)
 
