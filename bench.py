@@ -214,6 +214,9 @@ def time_oracle(wl, target_s: float, t_step: int = 1):
 # ---------------------------------------------------------------------------
 # GPU arm
 # ---------------------------------------------------------------------------
+TAIL_POOL = None  # (static share in 1/1024, chunk tiles) for mpadam_set_tail_pool, or the library's default
+
+
 def run_gpu(wl, steps: int, warmup: int, rank: int, e2e_steps: int, flush_l2: bool = False):
     import torch
     import workloads as W
@@ -228,6 +231,8 @@ def run_gpu(wl, steps: int, warmup: int, rank: int, e2e_steps: int, flush_l2: bo
                  grad_dtype=wl.grad_dtype, moment_dtype=wl.moment_dtype, rounding=wl.rounding,
                  seed=wl.seed + rank, fp8_exp=mt.fp8_exp, block_scales=mt.bscale if extended else None,
                  compute=mt.cc if extended else None, global_scales=mt.gscale if extended else None)
+    if TAIL_POOL:
+        opt.set_tail_pool(*TAIL_POOL)
     launches_per_step = len(set(mt.formats))
     stream = torch.cuda.current_stream(dev)
     gptrs = [g.data_ptr() for g in mt.g]
@@ -492,6 +497,8 @@ def main():
     ap.add_argument("--toy-steps", type=int, default=2048, help="matrix-fitting diagnostic steps per run (0 skips)")
     ap.add_argument("--rounding", default=None, choices=["nearest", "stochastic"],
                     help="override the workload's weight rounding")
+    ap.add_argument("--tail-pool", default=None, metavar="Q,CHUNK",
+                    help="static share (1/1024) and chunk tiles of the step's tail pool (default: the library's)")
     ap.add_argument("--max-params", type=int, default=0,
                     help="truncate the list to its first N params (small profiling cases)")
     args = ap.parse_args()
@@ -501,6 +508,9 @@ def main():
     wl = W.CONFIGS[args.config]
     if args.rounding:
         wl = W.replace(wl, rounding=args.rounding)
+    if args.tail_pool:
+        global TAIL_POOL
+        TAIL_POOL = tuple(int(x) for x in args.tail_pool.split(","))
     if args.max_params:
         wl, got = oracle_sample(wl, args.max_params)
         wl = W.replace(wl, name=f"{wl.name}[:{got}]")
