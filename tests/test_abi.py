@@ -86,6 +86,8 @@ def test_null_state_and_bad_step(N):
     assert lib.mpadam_destroy(None) == N.MPADAM_OK
     assert lib.mpadam_rng_lanes(0, 1, 7, 0, 4, None, None) == N.MPADAM_EINVAL
     assert lib.mpadam_rng_lanes(0, 1, N.MPADAM_BF16, -1, 4, None, None) == N.MPADAM_EINVAL
+    assert lib.mpadam_set_tail_pool(None, 768, 4) == N.MPADAM_EINVAL
+    assert lib.mpadam_set_grid(None, 0) == N.MPADAM_EINVAL
 
 
 def test_create_ex_rejects_bad_lists_on_the_host(N):
