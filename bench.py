@@ -72,11 +72,16 @@ def measured_peaks():
 
 def kernel_source_hash() -> str:
     """Hash of the step kernel's sources (the files its DRAM traffic depends
-    on: the kernel template, its argument layout and its instantiations)."""
+    on: the kernel template, its argument layout and its instantiations),
+    with comments and blank lines left out, so that editing a comment does
+    not retire the recorded counters."""
+    import re
     h = hashlib.sha256()
     csrc = ROOT / "paper_2607_10611_gb300" / "csrc"
     for f in sorted([csrc / "step_kernel.cuh", csrc / "step_args.h", *csrc.glob("step_*.cu")]):
-        h.update(f.read_bytes())
+        text = re.sub(r"/\*.*?\*/", "", f.read_text(), flags=re.S)
+        lines = (re.sub(r"//.*$", "", ln).rstrip() for ln in text.splitlines())
+        h.update("\n".join(ln for ln in lines if ln).encode())
     return h.hexdigest()[:16]
 
 

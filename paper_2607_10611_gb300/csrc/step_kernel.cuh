@@ -1,12 +1,15 @@
 // step_kernel.cuh -- the fused M+Adam step kernel for sm_103a (GB300).
 //
 // One launch = one pass over every element of the tensor list.  Each CTA
-// (one per SM) is a producer/consumer pipeline over its range of tiles:
-//   - one producer warp (one elected lane) streams each tile's slice of every
-//     array -- weights w, gradients g and the moments mu, nu, nu_e, each one
-//     contiguous run of bytes -- into a multi-stage shared-memory ring with
+// (one per SM) is a producer/consumer pipeline over its tiles:
+//   - one producer warp (one elected lane) picks each tile -- the next of its
+//     own range, then chunks claimed from the launch's tail pool -- posts the
+//     tile and its tensor beside the stage, and streams the tile's slice of
+//     every array (weights w, gradients g and the moments mu, nu, nu_e, each
+//     one contiguous run of bytes) into a multi-stage shared-memory ring with
 //     1-D TMA bulk copies (cp.async.bulk ... mbarrier::complete_tx), evict-
-//     first in L2 since every byte is used once;
+//     first in L2 since every byte is used once; an end marker in the next
+//     stage tells the consumers that the work is done;
 //   - fifteen consumer warps wait on the stage's mbarrier, read their 8
 //     elements from shared memory, run the canonical binary32 update
 //     (Algorithm 1 with the Algorithm 2 options, arxiv 2607.10611), round the
@@ -19,9 +22,12 @@
 // aligned, are read by the consumers directly from global memory with the
 // same arithmetic.  No tensor cores: nothing here is a contraction.
 //
-// Numerics: every floating-point operation is an explicit round-to-nearest
-// intrinsic (__fmul_rn, __fadd_rn, __fmaf_rn, __fdiv_rn, __fsqrt_rn), so build
-// flags cannot contract or approximate anything.
+// Numerics: every floating-point operation of the canonical sequence is an
+// explicit round-to-nearest intrinsic (__fmul_rn, __fadd_rn, __fmaf_rn,
+// __fdiv_rn, __fsqrt_rn), so build flags cannot contract or approximate
+// anything.  The certified fast path below uses approximate square roots and
+// divisions only where a rounding test proves the stored result equal to the
+// canonical one; everything else is recomputed canonically.
 //
 // Every wait on an mbarrier is bounded; a wait that gives up sets a bit in
 // *err, the producer waits (again bounded) for its own copies in flight, and
