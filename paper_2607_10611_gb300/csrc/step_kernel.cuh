@@ -1506,6 +1506,20 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
   int k = -1;
   TensorCtx x;
   int32_t e_next = 0;
+  auto enter = [&](int kk) {  // take up tensor kk
+    k = kk;
+    load_tensor<WD, GD, MD>(a, k, x);
+    if (WD == kE4M3) {
+      const int32_t e_cur = a.fp8_exp[static_cast<int64_t>(a.e_cur_slot) * n + x.d.ring];
+      e_next = fp8_next_exponent(a.fp8_amax[static_cast<int64_t>(a.a_cur_slot) * n + x.d.ring], e_cur);
+      x.dec_scale = pow2f(e_cur);
+      x.enc_scale = pow2f(-e_next);
+      x.cc_scale = pow2f(e_next);
+    }
+  };
+  // The first tile posted is the first of this CTA's own range when it has
+  // one: take up its tensor while the copies are in flight.
+  if (tb < ts) enter(a.cta_first[blockIdx.x]);
   uint32_t amax_bits = 0u;
   int s = 0;
   uint32_t use = 0;
@@ -1524,15 +1538,7 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
           atomicMax(&a.fp8_amax[static_cast<int64_t>(a.a_next_slot) * n + x.d.ring], wmax);
         amax_bits = 0u;
       }
-      k = kt;
-      load_tensor<WD, GD, MD>(a, k, x);
-      if (WD == kE4M3) {
-        const int32_t e_cur = a.fp8_exp[static_cast<int64_t>(a.e_cur_slot) * n + x.d.ring];
-        e_next = fp8_next_exponent(a.fp8_amax[static_cast<int64_t>(a.a_cur_slot) * n + x.d.ring], e_cur);
-        x.dec_scale = pow2f(e_cur);
-        x.enc_scale = pow2f(-e_next);
-        x.cc_scale = pow2f(e_next);
-      }
+      enter(kt);
     }
     const int64_t tile_e0 = (t - x.d.tile_off) * kTile;
     if (WD == kE4M3 && tile_e0 == 0 && c == 0) {  // the CTA holding the tensor's first tile
