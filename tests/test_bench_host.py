@@ -2,7 +2,8 @@
 - the max-over-ranks timing and whole-job rate of the replicated (N > 1)
   run, with two gloo ranks;
 - the reference arm (the oracle timed on the host) prints one valid line;
-- the product path refuses to run without its CUDA library (no fallback)."""
+- the product path refuses to run without its CUDA library (no fallback);
+- the hash that keys recorded DRAM traffic follows code, not comments."""
 import json
 import os
 import subprocess
@@ -64,3 +65,22 @@ def test_product_path_fails_loudly_without_its_library(monkeypatch, tmp_path):
     monkeypatch.setattr(_native, "_LIB", None)
     with pytest.raises(RuntimeError, match="build the CUDA library"):
         _native.lib()
+
+
+def test_kernel_source_hash_ignores_comments_but_not_code(tmp_path, monkeypatch):
+    """The hash that keys the recorded DRAM traffic changes with the kernel's
+    code, not with its comments or blank lines."""
+    import shutil
+    sys.path.insert(0, str(ROOT))
+    import bench
+    csrc = tmp_path / "paper_2607_10611_gb300" / "csrc"
+    shutil.copytree(ROOT / "paper_2607_10611_gb300" / "csrc", csrc)
+    monkeypatch.setattr(bench, "ROOT", tmp_path)
+    h0 = bench.kernel_source_hash()
+    k = csrc / "step_kernel.cuh"
+    text = k.read_text()
+    k.write_text("// a new comment\n\n/* and a block\n   comment */\n" + text.replace("\n", "  // note\n", 1))
+    assert bench.kernel_source_hash() == h0
+    k.write_text(text.replace("constexpr uint32_t kSpinLimit = 1u << 22;", "constexpr uint32_t kSpinLimit = 1u << 21;"))
+    assert bench.kernel_source_hash() != h0
+
