@@ -28,6 +28,7 @@ import math
 import os
 import subprocess
 import sys
+import tempfile
 import time
 from datetime import datetime
 from pathlib import Path
@@ -502,6 +503,8 @@ def main():
     ap.add_argument("--toy-steps", type=int, default=2048, help="matrix-fitting diagnostic steps per run (0 skips)")
     ap.add_argument("--rounding", default=None, choices=["nearest", "stochastic"],
                     help="override the workload's weight rounding")
+    ap.add_argument("--clocks-dir", default=None,
+                    help="directory for the raw nvidia-smi clock samples (clocks_rank0.csv); default: the temp dir")
     ap.add_argument("--tail-pool", default=None, metavar="Q,CHUNK",
                     help="static share (1/1024) and chunk tiles of the step's tail pool (default: the library's)")
     ap.add_argument("--max-params", type=int, default=0,
@@ -552,8 +555,8 @@ def main():
         torch.distributed.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
         torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", "0")))
     peak, peak_kind = measured_peaks()
-    out_dir = ROOT / "gpurun_out"
-    out_dir.mkdir(exist_ok=True)
+    out_dir = Path(args.clocks_dir) if args.clocks_dir else Path(tempfile.gettempdir())
+    out_dir.mkdir(parents=True, exist_ok=True)
     gpu_index = int(os.environ.get("LOCAL_RANK", "0"))
     sampler = ClockSampler(gpu_index, out_dir / f"clocks_rank{rank}.csv") if rank == 0 else None
     time.sleep(0.3 if sampler else 0)
