@@ -229,9 +229,12 @@ int32_t mpadam_fp8_init(mpadam_state* s, const int32_t* init_exp, int64_t first_
 /* One M+Adam step t (>= 1) over every tensor, asynchronously on `stream`.
  * grads: host array of n device pointers, grads[k] holding numel[k]
  * gradients of grad_dtype (read only).  The pointer table is re-uploaded
- * only when it differs from the previous call's.  The same (inputs, t, seed)
- * reproduce the same bits, so a resumed run calls with the step it stopped
- * at.  Errors: EINVAL (t < 1, NULL/misaligned grads), ECUDA (launch). */
+ * only when it differs from the previous call's.  On `stream` the call puts
+ * one kernel launch per weight format and, while a tail pool is on (see
+ * mpadam_set_tail_pool), one cudaMemsetAsync of the pool's counters before
+ * them.  Steps of one state must not overlap on the GPU.  The same (inputs, t, seed) reproduce the
+ * same bits, so a resumed run calls with the step it stopped at.
+ * Errors: EINVAL (t < 1, NULL/misaligned grads), ECUDA (launch). */
 int32_t mpadam_step(mpadam_state* s, const void* const* grads, int64_t step,
                     struct CUstream_st* stream);
 
