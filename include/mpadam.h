@@ -278,6 +278,20 @@ int32_t mpadam_host_buffer_free(void* ptr, int64_t bytes);
  * wide.  Errors: EINVAL. */
 int32_t mpadam_debug_fail_allocation(int32_t after);
 
+/* Host only, no GPU: the tile schedule mpadam_step's launches walk for a list
+ * of n tensors (numel, in launch order) on `ctas` CTAs with the tail pool
+ * (static_q, chunk_tiles) of mpadam_set_tail_pool.  Tiles are 3840 elements,
+ * numbered tensor by tensor.  cta_runs[3b..3b+2] = (tb, ts, te): CTA b walks
+ * [tb, ts) itself and its tiles [ts, te) go to the pool; cta_first[b] is the
+ * tensor holding tile tb.  pool[3i..3i+2] = (first tile, tile count, tensor
+ * of the first tile) of chunk i, in the order CTAs claim them;
+ * *pool_count = number of chunks.  Outputs: cta_runs [3 * ctas],
+ * cta_first [ctas], pool [3 * pool_cap].  Errors: EINVAL (arguments, or
+ * pool_cap below the chunk count, which is still reported), EALLOC. */
+int32_t mpadam_debug_tile_schedule(const int64_t* numel, int32_t n, int32_t ctas, int32_t static_q,
+                                   int32_t chunk_tiles, int64_t* cta_runs, int32_t* cta_first,
+                                   int64_t* pool, int32_t pool_cap, int32_t* pool_count);
+
 /* Frees the library's metadata (synchronises the device first).  NULL is a
  * no-op.  Never touches caller-owned tensors. */
 int32_t mpadam_destroy(mpadam_state* s);

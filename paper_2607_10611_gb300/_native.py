@@ -24,7 +24,7 @@ EXPORTED = ["mpadam_create", "mpadam_create_ex", "mpadam_fp8_init", "mpadam_step
             "mpadam_destroy", "mpadam_last_error", "mpadam_global_offset", "mpadam_global_length", "mpadam_set_grid",
             "mpadam_set_tail_pool", "mpadam_launch_info", "mpadam_rng_lanes", "mpadam_step_noalloc", "mpadam_device_status",
             "mpadam_toy_create", "mpadam_toy_step", "mpadam_toy_run", "mpadam_toy_destroy", "mpadam_host_buffer_alloc",
-            "mpadam_host_buffer_free", "mpadam_debug_fail_allocation"]
+            "mpadam_host_buffer_free", "mpadam_debug_fail_allocation", "mpadam_debug_tile_schedule"]
 
 
 class MPAdamError(RuntimeError):
@@ -122,6 +122,7 @@ def lib() -> ctypes.CDLL:
             "mpadam_host_buffer_alloc": [i64, P],
             "mpadam_host_buffer_free": [P, i64],
             "mpadam_debug_fail_allocation": [i32],
+            "mpadam_debug_tile_schedule": [P, i32, i32, i32, i32, P, P, P, i32, P],
         }
         for name, args in sig.items():
             f = getattr(L, name)
@@ -276,3 +277,24 @@ def mpadam_debug_fail_allocation(after: int) -> None:
     """Test hook: the library's allocation after `after` more successful ones
     fails once (-1 disarms)."""
     _check(lib().mpadam_debug_fail_allocation(after))
+
+
+def mpadam_debug_tile_schedule(numel, ctas: int, static_q: int, chunk_tiles: int):
+    """The step's tile schedule, computed on the host: per CTA (tb, ts, te)
+    and its first tensor, and the tail pool's chunks (start, count, tensor)."""
+    import numpy as np
+    nm = np.ascontiguousarray(numel, dtype=np.int64)
+    runs = np.zeros((ctas, 3), dtype=np.int64)
+    first = np.zeros(ctas, dtype=np.int32)
+    count = ctypes.c_int32(0)
+    cap = 0
+    while True:
+        pool = np.zeros((max(cap, 1), 3), dtype=np.int64)
+        rc = lib().mpadam_debug_tile_schedule(nm.ctypes.data, len(nm), ctas, static_q, chunk_tiles,
+                                               runs.ctypes.data, first.ctypes.data, pool.ctypes.data, cap,
+                                               ctypes.byref(count))
+        if rc == MPADAM_EINVAL and count.value > cap:
+            cap = count.value
+            continue
+        _check(rc)
+        return runs, first, pool[:count.value]

@@ -402,25 +402,26 @@ int32_t upload_cta_table(Group& g, int32_t grid) {
   return MPADAM_OK;
 }
 
-// The tail pool of a group for `grid` CTAs: CTA b keeps the first
-// (te - tb) * q / 1024 tiles of its range [tb, te) (the kernel computes the
-// same split) and the rest of every range becomes chunks of at most `chunk`
-// tiles, in tile order.
-int32_t upload_pool(Group& g, int32_t grid, int32_t q, int32_t chunk) {
-  g.pool_chunks = 0;
-  if (q >= 1024 || g.tiles == 0) return MPADAM_OK;
-  std::vector<mpadam::PoolChunk> pool;
+// The tail pool of `grid` CTAs over a list of `count` tensors (numel) with
+// `tiles` tiles in all: CTA b keeps the first (te - tb) * q / 1024 tiles of
+// its range [tb, te) (the kernel computes the same split) and the rest of
+// every range becomes chunks of at most `chunk` tiles, in tile order, each
+// with the tensor holding its first tile.  Host only.
+void pool_host(const int64_t* numel, int32_t count, int64_t tiles, int32_t grid, int32_t q, int32_t chunk,
+               std::vector<mpadam::PoolChunk>& pool) {
+  pool.clear();
+  if (q >= 1024 || tiles == 0) return;
   int32_t k = 0;
   int64_t tile_off = 0;
   auto tensor_of = [&](int64_t t) {  // t never decreases across calls
-    while (k < g.count && tile_off + tiles_of(g.numel[k]) <= t) {
-      tile_off += tiles_of(g.numel[k]);
+    while (k < count && tile_off + tiles_of(numel[k]) <= t) {
+      tile_off += tiles_of(numel[k]);
       ++k;
     }
     return k;
   };
   for (int32_t b = 0; b < grid; ++b) {
-    const int64_t tb = (int64_t)b * g.tiles / grid, te = ((int64_t)b + 1) * g.tiles / grid;
+    const int64_t tb = (int64_t)b * tiles / grid, te = ((int64_t)b + 1) * tiles / grid;
     for (int64_t t = tb + (te - tb) * q / 1024; t < te; t += chunk) {
       mpadam::PoolChunk pc;
       pc.start = t;
@@ -429,6 +430,14 @@ int32_t upload_pool(Group& g, int32_t grid, int32_t q, int32_t chunk) {
       pool.push_back(pc);
     }
   }
+}
+
+// The group's tail pool for `grid` CTAs, uploaded (none when q is 1024).
+int32_t upload_pool(Group& g, int32_t grid, int32_t q, int32_t chunk) {
+  g.pool_chunks = 0;
+  std::vector<mpadam::PoolChunk> pool;
+  pool_host(g.numel.data(), g.count, g.tiles, grid, q, chunk, pool);
+  if (pool.empty()) return MPADAM_OK;
   if (pool.size() > (size_t)INT32_MAX) return fail(MPADAM_EINVAL, "tail pool too large");
   if ((int32_t)pool.size() > g.pool_cap) {
     if (g.d_pool) cudaFree(g.d_pool);
@@ -438,10 +447,8 @@ int32_t upload_pool(Group& g, int32_t grid, int32_t q, int32_t chunk) {
       return fail(MPADAM_EALLOC, "cudaMalloc of %zu tail-pool chunks failed", pool.size());
     g.pool_cap = (int32_t)pool.size();
   }
-  if (!pool.empty()) {
-    cudaError_t e = cudaMemcpy(g.d_pool, pool.data(), sizeof(mpadam::PoolChunk) * pool.size(), cudaMemcpyHostToDevice);
-    if (e != cudaSuccess) return cuda_fail(e, "upload of the tail pool");
-  }
+  cudaError_t e = cudaMemcpy(g.d_pool, pool.data(), sizeof(mpadam::PoolChunk) * pool.size(), cudaMemcpyHostToDevice);
+  if (e != cudaSuccess) return cuda_fail(e, "upload of the tail pool");
   g.pool_chunks = (int32_t)pool.size();
   return MPADAM_OK;
 }
@@ -1472,5 +1479,45 @@ extern "C" int32_t mpadam_host_buffer_free(void* ptr, int64_t bytes) {
 extern "C" int32_t mpadam_debug_fail_allocation(int32_t after) {
   if (after < -1) return fail(MPADAM_EINVAL, "after must be >= -1");
   g_fail_countdown.store(after);
+  return MPADAM_OK;
+}
+
+extern "C" int32_t mpadam_debug_tile_schedule(const int64_t* numel, int32_t n, int32_t ctas, int32_t static_q,
+                                              int32_t chunk_tiles, int64_t* cta_runs, int32_t* cta_first,
+                                              int64_t* pool, int32_t pool_cap, int32_t* pool_count) {
+  if (n < 0 || (n > 0 && !numel)) return fail(MPADAM_EINVAL, "numel is NULL or n < 0");
+  if (ctas < 1 || ctas > (1 << 20)) return fail(MPADAM_EINVAL, "ctas must be in [1, 2^20]");
+  if (static_q < 0 || static_q > 1024) return fail(MPADAM_EINVAL, "static_q must be in [0, 1024]");
+  if (chunk_tiles < 1 || chunk_tiles > (1 << 20)) return fail(MPADAM_EINVAL, "chunk_tiles must be in [1, 2^20]");
+  if (!cta_runs || !cta_first || !pool_count || (pool_cap > 0 && !pool) || pool_cap < 0)
+    return fail(MPADAM_EINVAL, "NULL output or negative pool_cap");
+  int64_t tiles = 0;
+  for (int32_t k = 0; k < n; ++k) {
+    if (numel[k] < 0) return fail(MPADAM_EINVAL, "numel[%d] < 0", k);
+    tiles += tiles_of(numel[k]);
+  }
+  try {
+    std::vector<mpadam::PoolChunk> chunks;
+    pool_host(numel, n, tiles, ctas, static_q, chunk_tiles, chunks);
+    *pool_count = (int32_t)std::min<size_t>(chunks.size(), (size_t)INT32_MAX);
+    if (chunks.size() > (size_t)pool_cap) return fail(MPADAM_EINVAL, "pool_cap %d < %zu chunks", pool_cap, chunks.size());
+    for (size_t i = 0; i < chunks.size(); ++i) {
+      pool[3 * i] = chunks[i].start;
+      pool[3 * i + 1] = chunks[i].count;
+      pool[3 * i + 2] = chunks[i].first;
+    }
+    std::vector<int32_t> first(ctas);
+    cta_first_table(numel, n, tiles, ctas, first.data());
+    for (int32_t b = 0; b < ctas; ++b) {
+      const int64_t tb = (int64_t)b * tiles / ctas, te = ((int64_t)b + 1) * tiles / ctas;
+      // the kernel's split: a launch brings a pool only when it has chunks
+      cta_runs[3 * b] = tb;
+      cta_runs[3 * b + 1] = chunks.empty() ? te : tb + (te - tb) * static_q / 1024;
+      cta_runs[3 * b + 2] = te;
+      cta_first[b] = first[b];
+    }
+  } catch (const std::bad_alloc&) {
+    return fail(MPADAM_EALLOC, "host allocation failed");
+  }
   return MPADAM_OK;
 }
