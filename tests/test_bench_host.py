@@ -3,7 +3,8 @@
   run, with two gloo ranks;
 - the reference arm (the oracle timed on the host) prints one valid line;
 - the product path refuses to run without its CUDA library (no fallback);
-- the hash that keys recorded DRAM traffic follows code, not comments."""
+- the hash that keys recorded DRAM traffic follows code, not comments;
+- the algorithmic bytes behind the roofline, per tensor role."""
 import json
 import os
 import subprocess
@@ -84,3 +85,23 @@ def test_kernel_source_hash_ignores_comments_but_not_code(tmp_path, monkeypatch)
     k.write_text(text.replace("constexpr uint32_t kSpinLimit = 1u << 22;", "constexpr uint32_t kSpinLimit = 1u << 21;"))
     assert bench.kernel_source_hash() != h0
 
+
+
+@pytest.mark.parametrize("name,per_matrix,per_other", [
+    ("llama_7b", 18.0, 18.0),          # bf16 w read+written, bf16 g, three bf16 moments read+written
+    ("llama_1p5b", 28.0, 28.0),        # E4M3 w (1+1), bf16 g, three fp32 moments (24)
+    ("gpt2_124m", 30.0, 30.0),         # bf16 w (2+2), bf16 g, fp32 moments
+    ("flat_1m", 32.0, 32.0),           # bf16 w, fp32 g, fp32 moments
+    ("llama_1p5b_mixed", 30.125, 30.0),  # + 2-byte block scale per 32 (r+w) + 2-byte compute copy
+    ("llama_1p5b_nvfp4", 29.125, 30.0),  # half-byte codes (r+w), 1-byte scale per 16 (r+w), copy
+])
+def test_roofline_bytes_per_element(name, per_matrix, per_other):
+    """The denominator of the roofline: algorithmic bytes of one step, from
+    first principles per tensor role (linears in the low-precision format,
+    the rest BF16 in the mixed lists)."""
+    sys.path.insert(0, str(ROOT))
+    import bench
+    import workloads as W
+    wl = W.CONFIGS[name]
+    want = sum(s.numel * (per_matrix if s.role == "matrix" else per_other) for s in wl.specs)
+    assert bench.algorithmic_bytes(wl) == pytest.approx(want, rel=1e-9)
