@@ -347,9 +347,9 @@ int32_t mpadam_rng_lanes(uint64_t seed, int64_t step, int32_t weight_dtype, int6
  * config of mpadam_create plus the arguments of mpadam_step, keeps no state
  * object, and calls no cudaMalloc, cudaFree or other allocating routine:
  * the metadata the step kernel reads (tensor descriptors, gradient pointers,
- * per-CTA start tensors, 606,208 bytes at most) lives in one file-scope
- * device array that every GPU loading the library holds until the process
- * exits.  Limits: at most 8192 tensors (larger lists: MPADAM_EINVAL; use
+ * per-CTA start tensors) and the kernel's error word live in one file-scope
+ * device array of 606,464 bytes that every GPU loading the library holds
+ * until the process exits.  Limits: at most 8192 tensors (larger lists: MPADAM_EINVAL; use
  * mpadam_create).  The first call on a device looks up that array's device
  * address (set-up, once per device, with that device current); make that
  * first call before any stream capture.  Every call rewrites the array's
@@ -359,10 +359,23 @@ int32_t mpadam_rng_lanes(uint64_t seed, int64_t step, int32_t weight_dtype, int6
  * the shared array.  Results are bit-identical to mpadam_step on the same
  * inputs.  E4M3 weights use the caller's fp8_exp / fp8_amax rings exactly as
  * mpadam_step does (seed them with mpadam_fp8_init or equivalent values).
+ * A bounded wait inside the step kernel that gives up (the launch's results
+ * are then incomplete) sets a bit in the array's error word, which is not
+ * reported by this call's return value: read it with mpadam_noalloc_status.
  * Errors: EINVAL, EUNSUPPORTED, ECUDA. */
 int32_t mpadam_step_noalloc(const mpadam_tensor* tensors, int32_t n, const void* const* grads,
                             const mpadam_config* cfg, int32_t* fp8_exp, uint32_t* fp8_amax,
                             int64_t step, struct CUstream_st* stream);
+
+/* Device-side status of the allocation-free steps on the current device
+ * (companion of mpadam_step_noalloc; the paper has no counterpart).  Waits
+ * for `stream`, returns in *code the error bits the step kernel recorded
+ * since the last read (0 = none; non-zero: a bounded wait gave up and that
+ * step's results are incomplete), and clears them.  The word is shared by
+ * every allocation-free call on the device, like the tables: issue this on
+ * the stream the steps went to.  It allocates nothing (the word lives in the
+ * same file-scope array).  Errors: EINVAL (code NULL), EUNSUPPORTED, ECUDA. */
+int32_t mpadam_noalloc_status(struct CUstream_st* stream, int32_t* code);
 
 /* ------------------------------------------------------------------------
  * BF16-stored matrix-fitting diagnostic (the toy diagnostic of Sec. 5.1 and

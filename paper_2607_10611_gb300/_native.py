@@ -22,7 +22,7 @@ ROUNDING = {"nearest": MPADAM_ROUND_NEAREST, "stochastic": MPADAM_ROUND_STOCHAST
 
 EXPORTED = ["mpadam_create", "mpadam_create_ex", "mpadam_fp8_init", "mpadam_step", "mpadam_step_host",
             "mpadam_destroy", "mpadam_last_error", "mpadam_global_offset", "mpadam_global_length", "mpadam_set_grid",
-            "mpadam_set_tail_pool", "mpadam_launch_info", "mpadam_rng_lanes", "mpadam_step_noalloc", "mpadam_device_status",
+            "mpadam_set_tail_pool", "mpadam_launch_info", "mpadam_rng_lanes", "mpadam_step_noalloc", "mpadam_noalloc_status", "mpadam_device_status",
             "mpadam_toy_create", "mpadam_toy_step", "mpadam_toy_run", "mpadam_toy_destroy", "mpadam_host_buffer_alloc",
             "mpadam_host_buffer_free", "mpadam_debug_fail_allocation", "mpadam_debug_tile_schedule"]
 
@@ -115,6 +115,7 @@ def lib() -> ctypes.CDLL:
             "mpadam_rng_lanes": [u64, i64, i32, i64, i64, P, P],
             "mpadam_step_noalloc": [P, i32, P, P, P, P, i64, P],
             "mpadam_device_status": [P, P],
+            "mpadam_noalloc_status": [P, P],
             "mpadam_toy_create": [i64, P, P],
             "mpadam_toy_step": [P, P, P, i64, P, P],
             "mpadam_toy_run": [P, P, P, i64, i64, P, P],
@@ -242,6 +243,14 @@ def mpadam_step_noalloc(tensors: Sequence[tuple], grads: Sequence[int], cfg: mpa
         arr[i] = mpadam_tensor(w, m, v, ve, n)
     _check(lib().mpadam_step_noalloc(arr, len(tensors), _ptr_array(grads), ctypes.byref(cfg),
                                      fp8_exp or None, fp8_amax or None, step, stream or None))
+
+
+def mpadam_noalloc_status(stream: int = 0) -> int:
+    """Waits for `stream`; returns and clears the allocation-free steps'
+    device error bits (0: no bounded wait gave up)."""
+    out = ctypes.c_int32()
+    _check(lib().mpadam_noalloc_status(stream or None, ctypes.byref(out)))
+    return out.value
 
 
 def mpadam_toy_create(n: int, cfg: mpadam_toy_config) -> int:

@@ -1113,9 +1113,16 @@ namespace {
 
 constexpr int32_t kNoAllocMaxTensors = 8192;
 constexpr int32_t kNoAllocMaxCtas = 4096;
-constexpr size_t kNoAllocScratchBytes =
+constexpr size_t kNoAllocTableBytes =
     sizeof(TensorDesc) * kNoAllocMaxTensors + sizeof(void*) * kNoAllocMaxTensors +
     sizeof(int32_t) * kNoAllocMaxCtas;  // 606,208 bytes
+// The step kernel's device error word (a bounded wait that gave up) sits in
+// its own 256-byte slot after the tables.  It is sticky: every call ORs into
+// it, and only mpadam_noalloc_status reads and clears it.  The array starts
+// zeroed when the library's module loads.
+constexpr size_t kNoAllocErrOffset = kNoAllocTableBytes;
+constexpr size_t kNoAllocScratchBytes = kNoAllocTableBytes + 256;  // 606,464 bytes
+static_assert(kNoAllocErrOffset % 256 == 0, "the error word keeps the array's alignment");
 
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
 
@@ -1271,11 +1278,32 @@ extern "C" int32_t mpadam_step_noalloc(const mpadam_tensor* tensors, int32_t n, 
   a.desc = d_desc;
   a.grads = d_grads;
   a.cta_first = d_first;
-  a.err = nullptr;
+  a.err = reinterpret_cast<int32_t*>(scratch + kNoAllocErrOffset);
   fill_step(a, *cfg, step);
   void* params[] = {&a};
   e = cudaLaunchKernel(kernel, dim3(grid), dim3(mpadam::kThreads), params, (size_t)geo.dyn_smem, stream);
   if (e != cudaSuccess) return cuda_fail(e, "launch of the step kernel");
+  return MPADAM_OK;
+}
+
+extern "C" int32_t mpadam_noalloc_status(cudaStream_t stream, int32_t* code) {
+  if (!code) return fail(MPADAM_EINVAL, "code is NULL");
+  *code = 0;
+  int dev = -1;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+  unsigned char* scratch = nullptr;
+  int sms = 0;
+  int32_t rc = noalloc_setup(dev, &scratch, &sms);
+  if (rc) return rc;
+  int32_t* err = reinterpret_cast<int32_t*>(scratch + kNoAllocErrOffset);
+  // read after the stream's steps, then clear for the calls that follow
+  e = cudaMemcpyAsync(code, err, sizeof(int32_t), cudaMemcpyDeviceToHost, stream);
+  if (e != cudaSuccess) return cuda_fail(e, "reading the error word");
+  e = cudaMemsetAsync(err, 0, sizeof(int32_t), stream);
+  if (e != cudaSuccess) return cuda_fail(e, "clearing the error word");
+  e = cudaStreamSynchronize(stream);
+  if (e != cudaSuccess) return cuda_fail(e, "cudaStreamSynchronize");
   return MPADAM_OK;
 }
 

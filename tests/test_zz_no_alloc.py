@@ -4,7 +4,14 @@ allocator or memory pool, or a service that fixes its device-memory budget at
 start-up).  It keeps its tables in one device array built into the library
 instead of allocating, so it must give exactly what mpadam_step gives on the
 same inputs -- checked here bit for bit, the tolerance of every other parity
-test, over two calls in a row that reuse that shared array.
+test, over two calls in a row that reuse that shared array.  After the calls,
+mpadam_noalloc_status must report that no bounded wait inside the step kernel
+gave up (that word lives in the same array).
+
+Lists covered: more tensors than one table-fill launch carries (384), the
+E4M3 and BF16-moment formats, empty tensors passed with NULL pointers, and
+exactly the 8192-tensor limit.  The per-CTA table's own limit (4096 CTAs) is
+not reachable here: the step kernel runs one CTA per SM.
 
 The file name makes pytest collect it last, so a failure here leaves every
 other test already run; it also passes alone in a fresh process.
@@ -24,10 +31,18 @@ def N():
     return _native
 
 
+def _with_empty_tensors():
+    """A ragged list with zero-length tensors at the start, the middle and the end."""
+    specs = W.ragged_specs(40, 14, 5)
+    empty = W.TensorSpec("empty", 0, "flat")
+    specs = (empty,) + specs[:20] + (empty, empty) + specs[20:] + (empty,)
+    return W.replace(W.SMALL["ragged_20k"], specs=specs, name="ragged_with_empty")
+
+
 def _lists():
-    # more tensors than one table-fill launch carries (384), ragged sizes
     ragged = W.replace(W.SMALL["ragged_20k"], specs=W.ragged_specs(1000, 10, 3), name="ragged_1000")
-    return [ragged, W.SMALL["llama_1p5b"], W.SMALL["llama_7b"]]
+    limit = W.replace(W.SMALL["ragged_20k"], specs=W.ragged_specs(8192, 6, 9), name="ragged_8192")
+    return [ragged, W.SMALL["llama_1p5b"], W.SMALL["llama_7b"], _with_empty_tensors(), limit]
 
 
 def _device(mt):
@@ -49,15 +64,19 @@ def test_noalloc_matches_mpadam_step_on_two_calls(N, wl):
         torch.cuda.synchronize()
         exp_ring = ref.fp8_exp_ring.clone()
         amax_ring = ref.fp8_amax_ring.clone()
-    tensors = [(w.data_ptr(), m.data_ptr(), v.data_ptr(), ve.data_ptr(), w.numel())
+
+    def ptr(t):  # empty tensors go in with NULL pointers
+        return t.data_ptr() if t.numel() else 0
+
+    tensors = [(ptr(w), ptr(m), ptr(v), ptr(ve), w.numel())
                for w, m, v, ve in zip(b["w"], b["m"], b["v"], b["ve"])]
-    grads = [g.data_ptr() for g in b["g"]]
+    grads = [ptr(g) for g in b["g"]]
+    stream = torch.cuda.current_stream().cuda_stream
     for t in (1, 2):
         ref.step(a["g"], t)
         N.mpadam_step_noalloc(tensors, grads, cfg, t,
                               exp_ring.data_ptr() if exp_ring is not None else 0,
-                              amax_ring.data_ptr() if amax_ring is not None else 0,
-                              torch.cuda.current_stream().cuda_stream)
+                              amax_ring.data_ptr() if amax_ring is not None else 0, stream)
         torch.cuda.synchronize()
         for key in ("w", "m", "v", "ve"):
             for x, y in zip(a[key], b[key]):
@@ -65,6 +84,8 @@ def test_noalloc_matches_mpadam_step_on_two_calls(N, wl):
         if exp_ring is not None:
             assert torch.equal(exp_ring, ref.fp8_exp_ring)
             assert torch.equal(amax_ring, ref.fp8_amax_ring)
+    assert N.mpadam_noalloc_status(stream) == 0, "a bounded wait in the allocation-free step gave up"
+    assert ref.device_status() == 0
     ref.close()
 
 
@@ -76,3 +97,6 @@ def test_noalloc_rejects_lists_beyond_its_limit(N):
     with pytest.raises(N.MPAdamError) as ei:
         N.mpadam_step_noalloc([t] * 8193, [m.data_ptr()] * 8193, cfg, 1)
     assert ei.value.status == N.MPADAM_EINVAL and "8192" in str(ei.value)
+    with pytest.raises(N.MPAdamError) as ei:  # no place for the code
+        N._check(N.lib().mpadam_noalloc_status(None, None))
+    assert ei.value.status == N.MPADAM_EINVAL
