@@ -63,6 +63,11 @@ def algorithmic_bytes_per_param(wl) -> float:
     return algorithmic_bytes(wl) / wl.n_params
 
 
+# GB300's nominal HBM3e bandwidth (8 stacks at 3996 MHz), for a second fraction
+# beside the measured copy peak
+NOMINAL_HBM_GBS = 7900.0
+
+
 def measured_peaks():
     p = ROOT / "MEASURED_PEAKS.json"
     if p.exists():
@@ -302,15 +307,16 @@ def run_gpu(wl, steps: int, warmup: int, rank: int, e2e_steps: int, flush_l2: bo
         opt.step_host(hgs, hws, t)  # warm (allocates the staging buffer)
         t += 1
         torch.cuda.synchronize()
-        e0 = torch.cuda.Event(enable_timing=True)
-        e1 = torch.cuda.Event(enable_timing=True)
-        e0.record(stream)
-        for _ in range(e2e_steps):
+        # one event per step boundary: the region's mean, and each step's own time
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(e2e_steps + 1)]
+        ev[0].record(stream)
+        for i in range(e2e_steps):
             opt.step_host(hgs, hws, t)
+            ev[i + 1].record(stream)
             t += 1
-        e1.record(stream)
         torch.cuda.synchronize()
-        res["e2e_ms"] = e0.elapsed_time(e1) / e2e_steps
+        res["e2e_ms"] = ev[0].elapsed_time(ev[-1]) / e2e_steps
+        res["e2e_step_ms"] = [ev[i].elapsed_time(ev[i + 1]) for i in range(e2e_steps)]
         res["h2d"] = sum(x.numel() for x in mt.g) * BYTES[wl.grad_dtype]
         res["d2h"] = sum(x.numel() for x in mt.w) * BYTES[wl.weight_dtype]
         res["link_ms"] = host_link_ms(hg, mt.flat["g"], hw, mt.flat["w"], stream)
@@ -461,31 +467,102 @@ def summarize(wl, res, n_gpus, peak, peak_kind):
     avg_launch = sum(launch) / len(launch)
     achieved = algorithmic_bytes(wl) / (avg_launch * 1e-3) / 1e9
     out = {
-        "workload": wl.name, "params": n, "tensors": len(wl.specs),
+        "workload": wl.name, "rounding": wl.rounding, "params": n, "tensors": len(wl.specs),
         "l2": "flushed between launches (256 MB write, then 256 MB read)" if res.get("l2_flushed")
               else "inputs larger than L2",
         "ms_per_step": ms, "gparams_per_s": whole_job_rate(n, n_gpus, ms),
         "hbm_gbs": algorithmic_bytes(wl) / (ms * 1e-3) / 1e9,
         "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
                      "frac": round(achieved / peak, 4), "traffic": recorded_traffic(wl.name),
-                     "peak_source": peak_kind, "bytes_per_param": round(bpp, 4),
+                     "peak_source": peak_kind, "nominal_peak": NOMINAL_HBM_GBS,
+                     "frac_of_nominal": round(achieved / NOMINAL_HBM_GBS, 4),
+                     "bytes_per_param": round(bpp, 4),
                      "launches_per_step": res["launches_per_step"],
                      "kernel": "mpadam::step_kernel", "launch_ms_avg": round(avg_launch, 4),
-                     "launch_ms_min": round(launch[0], 4), "launch_ms_max": round(launch[-1], 4),
-                     "launch_ms_first_last": [round(res["launch_ms"][0], 4), round(res["launch_ms"][-1], 4)]},
+                     "launch_ms_min": round(launch[0], 4), "launch_ms_max": round(launch[-1], 4)},
+        "grid": res["grid"],
     }
     if res.get("copy_ms"):
         # context for lists that fit in L2: a plain copy of the same bytes, same flush
         out["roofline"]["copy_same_bytes_ms"] = round(res["copy_ms"], 4)
         out["roofline"]["frac_of_copy_same_bytes"] = round(res["copy_ms"] / avg_launch, 4)
     if "e2e_ms" in res:
+        per = sorted(res["e2e_step_ms"])
+        med = per[len(per) // 2] if len(per) % 2 else 0.5 * (per[len(per) // 2 - 1] + per[len(per) // 2])
         out["e2e"] = {"value": n_gpus * n / (res["e2e_ms"] * 1e-3) / 1e9, "unit": UNIT,
                       "h2d_bytes_per_step": res["h2d"], "d2h_bytes_per_step": res["d2h"],
-                      "ms_per_step": res["e2e_ms"],
-                      "host_link_ms": res["link_ms"],
-                      "host_link_gbs": (res["h2d"] + res["d2h"]) / (res["link_ms"] * 1e-3) / 1e9,
-                      "frac_of_host_link_bound": res["link_ms"] / res["e2e_ms"],
+                      "ms_per_step": round(res["e2e_ms"], 3), "steps": len(per),
+                      "ms_median": round(med, 3), "ms_worst": round(per[-1], 3), "ms_best": round(per[0], 3),
+                      "host_link_ms": round(res["link_ms"], 3),
+                      "host_link_gbs": round((res["h2d"] + res["d2h"]) / (res["link_ms"] * 1e-3) / 1e9, 1),
+                      "frac_of_host_link_bound": round(res["link_ms"] / res["e2e_ms"], 4),
+                      "frac_of_host_link_bound_median": round(res["link_ms"] / med, 4),
                       "host_buffers": res.get("host_buffers")}
+    return out
+
+
+def compact(sec) -> dict:
+    """One secondary list in a few keys: the driver keeps only the tail of
+    the line, so the full record goes to the details file."""
+    c = {"workload": sec["workload"] + ("" if sec["rounding"] == W_DEFAULT_ROUNDING.get(sec["workload"]) else
+                                         ":" + sec["rounding"]),
+         "ms": round(sec["ms_per_step"], 4), "gparam_s": round(sec["gparams_per_s"], 1),
+         "gbs": round(sec["roofline"]["achieved"], 0), "frac": sec["roofline"]["frac"]}
+    if "frac_of_copy_same_bytes" in sec["roofline"]:
+        c["frac_of_copy"] = sec["roofline"]["frac_of_copy_same_bytes"]
+    clk = sec.get("clocks") or {}
+    c["sm_mhz"] = clk.get("sm_mhz")
+    if clk.get("reasons"):
+        c["reasons"] = clk["reasons"]
+    return c
+
+
+W_DEFAULT_ROUNDING = {}  # workload name -> its configured rounding (filled in main)
+
+
+def workload_config(wl, world: int, l2: str) -> dict:
+    """The `config` of the JSON line: what the workload is (both arms print the same)."""
+    return {"workload": wl.name, "params": wl.n_params, "tensors": len(wl.specs),
+            "weights": wl.weight_dtype, "grads": wl.grad_dtype, "moments": wl.moment_dtype,
+            "rounding": wl.rounding, "l2": l2,
+            "parallelism": f"replicas x{world}" if world > 1 else "single GPU"}
+
+
+def result_line(wl, world, steps, warmup, l2_desc, main_sum, cpu, clocks, toy, details, secondary,
+                launches) -> dict:
+    """The one JSON line rank 0 prints.  The driver keeps only the line's
+    tail, so it stays short: the full per-workload record (every roofline
+    field, the diagnostic's per-regime table) is in the details file, and
+    the compact secondary entries come last."""
+    roof = main_sum["roofline"]
+    return {
+        "metric": METRIC, "value": round(main_sum["gparams_per_s"], 3), "unit": UNIT, "n_gpus": world,
+        "steps": steps, "warmup": warmup, "ms_per_step": round(main_sum["ms_per_step"], 4),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": workload_config(wl, world, l2_desc),
+        "hbm_gbs": round(main_sum["hbm_gbs"], 1),
+        "roofline": {k: roof[k] for k in ("bound", "achieved", "peak", "unit", "frac", "traffic", "peak_source",
+                                          "nominal_peak", "frac_of_nominal", "bytes_per_param", "launch_ms_avg")},
+        "cpu_baseline": cpu,
+        "e2e": main_sum.get("e2e"),
+        "gpu_launches": launches,
+        "grid": main_sum["grid"],
+        "clocks": clocks,
+        "toy_us_per_step": round(toy["us_per_step"], 2) if toy else None,
+        "details": str(details),
+        # last, so that the tail of the line the driver keeps holds every list
+        "secondary": [compact(x) for x in secondary],
+    }
+
+
+def parse_secondary(spec: str):
+    """'name' or 'name:rounding', comma-separated."""
+    import workloads as W
+    out = []
+    for item in filter(None, spec.split(",")):
+        name, _, rnd = item.partition(":")
+        wl = W.CONFIGS[name]
+        out.append(W.replace(wl, rounding=rnd) if rnd else wl)
     return out
 
 
@@ -495,16 +572,18 @@ def main():
     ap.add_argument("--steps", type=int, default=50)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--config", default="llama_7b")
-    ap.add_argument("--secondary", default="llama_1p5b,llama_1p5b_mixed,llama_1p5b_nvfp4,gpt2_124m,ragged_20k,flat_1m",
-                    help="'' to skip")
+    ap.add_argument("--secondary", default="llama_1p5b,llama_1p5b_mixed,llama_1p5b_nvfp4,"
+                                           "llama_1p5b_nvfp4:stochastic,gpt2_124m,ragged_20k,flat_1m",
+                    help="comma-separated workload[:rounding] list measured after the main one ('' to skip)")
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--e2e-steps", type=int, default=5)
+    ap.add_argument("--e2e-steps", type=int, default=20)
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
     ap.add_argument("--toy-steps", type=int, default=2048, help="matrix-fitting diagnostic steps per run (0 skips)")
     ap.add_argument("--rounding", default=None, choices=["nearest", "stochastic"],
                     help="override the workload's weight rounding")
     ap.add_argument("--clocks-dir", default=None,
-                    help="directory for the raw nvidia-smi clock samples (clocks_rank0.csv); default: the temp dir")
+                    help="directory for the raw nvidia-smi clock samples (clocks_rank0.csv) and the full "
+                         "per-workload record (bench_details.json); default: the temp dir")
     ap.add_argument("--tail-pool", default=None, metavar="Q,CHUNK",
                     help="static share (1/1024) and chunk tiles of the step's tail pool (default: the library's)")
     ap.add_argument("--max-params", type=int, default=0,
@@ -513,6 +592,8 @@ def main():
     warmup = max(3, args.warmup)
 
     import workloads as W
+    for name, w in W.CONFIGS.items():
+        W_DEFAULT_ROUNDING[name] = w.rounding
     wl = W.CONFIGS[args.config]
     if args.rounding:
         wl = W.replace(wl, rounding=args.rounding)
@@ -524,28 +605,32 @@ def main():
         wl = W.replace(wl, name=f"{wl.name}[:{got}]")
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
+    l2_desc = ("flushed between launches (256 MB write, then 256 MB read)" if algorithmic_bytes(wl) < 512e6
+               else "inputs larger than L2 (no flush needed)")
 
     if args.impl == "reference":
         # the oracle is the reference: rank 0 only, on the host cores
         if rank != 0:
             return
         per_step = []
-        sample_desc = None
         for i in range(warmup + args.steps):
             got, dt, rate = time_oracle(wl, target_s=1.0, t_step=1 + i)
             if i >= warmup:
                 per_step.append((got, dt))
-            sample_desc = f"first {got} elements of the {wl.name} list per step, one step each"
         elems = sum(g for g, _ in per_step)
         secs = sum(d for _, d in per_step)
         value = elems / secs / 1e9
+        sample_ms = 1e3 * secs / len(per_step)
+        sample = (f"each step: one oracle step over the first {per_step[-1][0]} elements of the {wl.name} list "
+                  f"(single thread); ms_per_step is that sample's time")
         line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
-                "steps": args.steps, "warmup": warmup, "ms_per_step": 1e3 * wl.n_params / (value * 1e9),
+                "steps": args.steps, "warmup": warmup, "ms_per_step": round(sample_ms, 3),
                 "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
-                "data": "synthetic",
-                "config": {"workload": wl.name, "params": wl.n_params, "tensors": len(wl.specs)},
-                "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
-                                 "sample": sample_desc},
+                "data": "synthetic", "config": workload_config(wl, 1, l2_desc),
+                "sample_elements_per_step": per_step[-1][0],
+                "whole_list_ms_per_step_extrapolated": round(1e3 * wl.n_params / (value * 1e9), 1),
+                "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "nproc": os.cpu_count(),
+                                 "kind": "oracle", "sample": sample},
                 "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
         print(json.dumps(line), flush=True)
         return
@@ -572,8 +657,7 @@ def main():
 
     secondary = []
     if args.secondary and rank == 0 and world == 1:
-        for name in args.secondary.split(","):
-            wl2 = W.CONFIGS[name]
+        for wl2 in parse_secondary(args.secondary):
             r2 = run_gpu(wl2, args.steps, warmup, rank, 0, flush_l2=algorithmic_bytes(wl2) < 512e6)
             s2 = summarize(wl2, r2, 1, peak, peak_kind)
             s2["clocks"] = sampler.summary(*r2["wall"]) if sampler else None
@@ -586,34 +670,15 @@ def main():
             torch.distributed.destroy_process_group()
         return
 
-    cpu = None
-    if world == 1 or rank == 0:
-        got, dt, rate = time_oracle(wl, target_s=args.cpu_seconds)
-        cpu = {"value": rate / 1e9, "unit": UNIT, "cores": 1, "kind": "oracle",
-               "sample": f"one step over the first {got} elements of the {wl.name} list "
-                         f"({dt:.1f} s, single thread)"}
+    got, dt, rate = time_oracle(wl, target_s=args.cpu_seconds)
+    cpu = {"value": rate / 1e9, "unit": UNIT, "cores": 1, "nproc": os.cpu_count(), "kind": "oracle",
+           "sample": f"one step over the first {got} elements of the {wl.name} list ({dt:.1f} s, single thread)"}
 
-    ms = main_sum["ms_per_step"]
-    line = {
-        "metric": METRIC, "value": round(main_sum["gparams_per_s"], 3), "unit": UNIT, "n_gpus": world,
-        "steps": args.steps, "warmup": warmup, "ms_per_step": round(ms, 4), "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-        "config": {"workload": wl.name, "params": wl.n_params, "tensors": len(wl.specs),
-                   "weights": wl.weight_dtype, "grads": wl.grad_dtype, "moments": wl.moment_dtype,
-                   "rounding": wl.rounding,
-                   "l2": main_sum["l2"] if res.get("l2_flushed") else "inputs larger than L2 (no flush needed)",
-                   "parallelism": f"replicas x{world}" if world > 1 else "single GPU",
-                   "grid": res["grid"][0], "threads": res["grid"][1]},
-        "hbm_gbs": round(main_sum["hbm_gbs"], 1),
-        "hbm_frac_of_peak": round(main_sum["hbm_gbs"] / peak, 4),
-        "roofline": main_sum["roofline"],
-        "cpu_baseline": cpu,
-        "e2e": main_sum.get("e2e"),
-        "gpu_launches": args.steps * res["launches_per_step"],
-        "clocks": clocks,
-        "secondary": secondary,
-        "toy": toy,
-    }
+    details = out_dir / "bench_details.json"
+    details.write_text(json.dumps({"main": main_sum, "secondary": secondary, "toy": toy, "clocks": clocks,
+                                   "cpu_baseline": cpu}, indent=1))
+    line = result_line(wl, world, args.steps, warmup, l2_desc, main_sum, cpu, clocks, toy, details, secondary,
+                       args.steps * res["launches_per_step"])
     print(json.dumps(line), flush=True)
     if world > 1:
         torch.distributed.destroy_process_group()

@@ -56,6 +56,15 @@ def test_reference_arm_prints_one_json_line():
     d = json.loads(lines[0])
     assert d["impl"] == "reference" and d["unit"] == "Gparams/s" and d["value"] > 0
     assert d["cpu_baseline"]["kind"] == "oracle" and d["cpu_baseline"]["cores"] == 1
+    assert d["cpu_baseline"]["nproc"] == os.cpu_count()
+    # the timed sample's own step time, and the sample's size, not an extrapolation
+    assert d["sample_elements_per_step"] > 0
+    assert d["ms_per_step"] == pytest.approx(1e3 * d["sample_elements_per_step"] / (d["value"] * 1e9), rel=0.5)
+    # the same workload description as the GPU arm's line
+    import bench
+    import workloads as W
+    wl = W.CONFIGS["gpt2_124m"]
+    assert d["config"] == bench.workload_config(wl, 1, "inputs larger than L2 (no flush needed)")
     assert d["e2e"]["h2d_bytes_per_step"] == 0 and d["e2e"]["d2h_bytes_per_step"] == 0
     assert d["higher_is_better"] is True and d["config"]["workload"] == "gpt2_124m"
 
@@ -105,3 +114,48 @@ def test_roofline_bytes_per_element(name, per_matrix, per_other):
     wl = W.CONFIGS[name]
     want = sum(s.numel * (per_matrix if s.role == "matrix" else per_other) for s in wl.specs)
     assert bench.algorithmic_bytes(wl) == pytest.approx(want, rel=1e-9)
+
+
+def _fake_res(wl, ms, e2e=False):
+    """What run_gpu returns, with plausible timings (full-precision floats)."""
+    res = {"total_ms": ms * 20 * 1.0000123, "launch_ms": [ms * (1 + 1e-3 * i / 7) for i in range(20)],
+           "wall": (0.0, 1.0), "grid": (152, 512), "launches_per_step": 1 + (wl.weight_dtype != "bf16"),
+           "l2_flushed": wl.name == "flat_1m", "copy_ms": 0.0081234567 if wl.name == "flat_1m" else None}
+    if e2e:
+        res.update(e2e_ms=101.234567, e2e_step_ms=[100.0 + 1.2345678 * i for i in range(20)],
+                   h2d=13476831232, d2h=13476831232, link_ms=94.12345678, host_buffers="huge_pages")
+    return res
+
+
+def test_result_line_keeps_every_secondary_list_in_the_driver_tail():
+    """The driver records only the last ~1500 characters of the line: the
+    secondary lists (the 1.5B target among them) must all sit there."""
+    sys.path.insert(0, str(ROOT))
+    import bench
+    import workloads as W
+    for name, w in W.CONFIGS.items():
+        bench.W_DEFAULT_ROUNDING[name] = w.rounding
+    wl = W.CONFIGS["llama_7b"]
+    main = bench.summarize(wl, _fake_res(wl, 18.7654321, e2e=True), 1, 6783.5, "measured")
+    secs = []
+    for wl2 in bench.parse_secondary("llama_1p5b,llama_1p5b_mixed,llama_1p5b_nvfp4,"
+                                     "llama_1p5b_nvfp4:stochastic,gpt2_124m,ragged_20k,flat_1m"):
+        s2 = bench.summarize(wl2, _fake_res(wl2, 6.1234567), 1, 6783.5, "measured")
+        s2["clocks"] = {"sm_mhz": 2070.0, "sm_max_mhz": 2070.0, "reasons": [], "samples": 12}
+        secs.append(s2)
+    cpu = {"value": 0.018728084501097277, "unit": "Gparams/s", "cores": 1, "nproc": 72, "kind": "oracle",
+           "sample": "one step over the first 181498738 elements of the llama_7b list (9.7 s, single thread)"}
+    clocks = {"sm_mhz": 2070.0, "sm_max_mhz": 2070.0, "reasons": [], "samples": 5}
+    line = bench.result_line(wl, 1, 20, 5, "inputs larger than L2 (no flush needed)", main, cpu, clocks,
+                             {"us_per_step": 15.51234}, "/tmp/bench_details.json", secs, 20)
+    text = json.dumps(line)
+    assert len(text) < 3000, len(text)
+    tail = text[-1400:]
+    for s2 in secs:
+        c = bench.compact(s2)
+        assert json.dumps(c) in tail, c["workload"]
+    assert '"workload": "llama_1p5b_nvfp4:stochastic"' in tail and '"workload": "llama_1p5b"' in tail
+    for key in ("metric", "value", "unit", "ms_per_step", "roofline", "cpu_baseline", "e2e", "clocks"):
+        assert key in line
+    assert line["e2e"]["steps"] == 20 and line["e2e"]["ms_worst"] >= line["e2e"]["ms_median"]
+    assert line["roofline"]["frac_of_nominal"] < line["roofline"]["frac"]
