@@ -62,7 +62,10 @@
  * The caller owns two device rings that hold this state:
  *   fp8_exp  : int32[2 n],  e_t of tensor k at fp8_exp[(t mod 2) n + k];
  *   fp8_amax : uint32[3 n], binary32 bits of A_t at fp8_amax[(t mod 3) n + k].
- * Step t reads slot t, writes slot t+1 and clears amax slot t+2.
+ * Step t reads slot t, writes slot t+1 and clears amax slot t+2.  Amax
+ * slot t+1 must hold 0 when step t starts (mpadam_fp8_init and step t-1
+ * leave it so): the step raises it with exact |w'| values only, and also
+ * reads it while it runs as a lower bound of A_{t+1}.
  *
  * Conventions for every entry point:
  *   - returns MPADAM_OK (0) or a positive mpadam_status; never aborts or
@@ -317,9 +320,8 @@ int32_t mpadam_launch_info(const mpadam_state* s, int32_t* ctas, int32_t* thread
  * chunk_tiles tiles, which the CTAs that finish first claim one at a time.
  * SMs do not all stream memory at the same rate, so without the pool a
  * launch waits on the slowest.  static_q = 1024 turns the pool off.
- * Default: static_q = 768, chunk_tiles = 4, except that lists' per-tensor
- * scaled E4M3 tensors keep static runs until this is called (they measured
- * slower with the pool).  Results do not depend on either value.
+ * Default: static_q = 768, chunk_tiles = 4, for every weight format.
+ * Results do not depend on either value.
  * Synchronises the device.  The host-buffer and allocation-free entry
  * points always use static runs.
  * Errors: EINVAL (static_q outside [0, 1024], chunk_tiles outside

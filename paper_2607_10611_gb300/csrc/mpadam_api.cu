@@ -327,11 +327,8 @@ struct mpadam_state {
   std::vector<int64_t> chunk_tile;            // chunk c covers tiles [chunk_tile[c], chunk_tile[c+1])
   std::vector<int64_t> chunk_elem;            // and global elements [chunk_elem[2c], chunk_elem[2c+1])
   int32_t* d_chunk_first = nullptr;           // [chunks][grid] CTA start tensors
-  // tail pool of mpadam_step's launches: static prefix of each CTA's range (1/1024) and chunk length.
-  // Until set_tail_pool is called, per-tensor-scaled E4M3 groups keep static ranges: measured
-  // slower with the pool (the other formats gain 3-12 %).
+  // tail pool of mpadam_step's launches: static prefix of each CTA's range (1/1024) and chunk length
   int32_t pool_q = 768, pool_chunk = 4;
-  bool pool_set = false;
   uint32_t* d_pool_next = nullptr;            // [groups] claim counters, zeroed before each step
 };
 
@@ -453,9 +450,12 @@ int32_t upload_pool(Group& g, int32_t grid, int32_t q, int32_t chunk) {
   return MPADAM_OK;
 }
 
-// The static share a group's launches use.
+// The static share a group's launches use (every format: per-tensor E4M3
+// groups too, since their consumers seed the exact-maximum threshold from the
+// amax ring after each tensor change).
 int32_t pool_q_of(const mpadam_state* s, const Group& g) {
-  return g.wd == MPADAM_E4M3 && !s->pool_set ? 1024 : s->pool_q;
+  (void)g;
+  return s->pool_q;
 }
 
 void fill_common(StepArgs& a, const mpadam_config& cfg, const Geometry& geo, int64_t total_tiles, int32_t n,
@@ -862,7 +862,6 @@ int32_t mpadam_set_tail_pool(mpadam_state* s, int32_t static_q, int32_t chunk_ti
   if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceSynchronize");
   s->pool_q = static_q;
   s->pool_chunk = chunk_tiles;
-  s->pool_set = true;
   for (auto& g : s->groups) {
     rc = upload_pool(g, g.grid, pool_q_of(s, g), s->pool_chunk);
     if (rc) return rc;

@@ -582,6 +582,7 @@ struct TensorCtx {
   void* scale;         // kE4M3B (FP16) / kNVFP4 (E4M3) block scales
   uint16_t* cc;        // BF16 compute copy, or nullptr
   float gscale;        // kNVFP4 tensor scale
+  float amax_seed;     // kE4M3: a lower bound of the tensor's largest exact |w'| of this step
 };
 
 template <int WD, int GD, int MD>
@@ -598,6 +599,7 @@ __device__ __forceinline__ void load_tensor(const StepArgs& a, int k, TensorCtx&
   c.scale = nullptr;
   c.cc = nullptr;
   c.gscale = 1.0f;
+  c.amax_seed = 0.0f;
   if (WD != kBF16 && a.aux) {
     const TensorAux x = a.aux[k];
     c.scale = x.scale;
@@ -713,11 +715,13 @@ __device__ __forceinline__ void finish_group(const StepArgs& a, const TensorCtx&
   } else if (WD == kE4M3 && !OPT && a.s.cert_ok) {
     // Certified fast path for E4M3: both ends of the bound are scaled by 2^-e
     // with outward rounding and encoded; the largest |w'| must be exact, so an
-    // element whose bound reaches this thread's running maximum (of exact
-    // values) is recomputed as well -- no other element can be the maximum.
+    // element whose bound reaches the threshold is recomputed as well.  The
+    // threshold is the larger of this thread's running maximum and the
+    // tensor's maximum flushed so far in this step: both are exact |w'| of
+    // elements of this tensor, so no element below them can be the maximum.
     uint32_t code[8];
     uint32_t redo = 0u;
-    const float amax_f = __uint_as_float(amax_bits);
+    const float amax_f = fmaxf(__uint_as_float(amax_bits), x.amax_seed);
 #pragma unroll
     for (int j = 0; j < kGroup; ++j) {
       const CertUpd u = madam_update_cert<false>(a.s, w[j], g[j], m[j], v[j], ve[j]);
@@ -1515,6 +1519,16 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
       x.dec_scale = pow2f(e_cur);
       x.enc_scale = pow2f(-e_next);
       x.cc_scale = pow2f(e_next);
+      // The tensor's maximum flushed so far in this step, read through L2:
+      // the slot was zeroed before this step and is raised only with exact
+      // values, so it seeds the recomputation threshold after a tensor change
+      // (under the tail pool a CTA changes tensor at almost every chunk).
+      uint32_t seed;
+      asm volatile("ld.global.cg.u32 %0, [%1];"
+                   : "=r"(seed)
+                   : "l"(a.fp8_amax + static_cast<int64_t>(a.a_next_slot) * n + x.d.ring)
+                   : "memory");
+      x.amax_seed = __uint_as_float(seed);
     }
   };
   // The first tile posted is the first of this CTA's own range when it has

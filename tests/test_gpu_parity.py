@@ -43,6 +43,26 @@ def test_small_workloads_bit_exact(name, warm):
         r.close()
 
 
+# Past the first steps: from the zero state of Algorithm 1, the bias
+# corrections change with t, the moments grow, and the E4M3 scale rings rotate
+# with period 6 (exponent slot t mod 2, amax slot t mod 3).  Twelve steps cover
+# two full periods; the GPT-2 list runs its configuration's 100 steps.  Every
+# array and both rings are compared after every step.
+@pytest.mark.parametrize("name", list(W.SMALL))
+def test_small_workloads_many_steps(name):
+    p = P()
+    steps = 100 if name == "gpt2_124m" else 12
+    r = p.Run(W.SMALL[name])
+    try:
+        for t in range(1, steps + 1):
+            r.step(t)
+            res = r.compare(t + 1)
+            assert res["contract_ok"]
+            p.assert_exact(res, f"{name} step {t}")
+    finally:
+        r.close()
+
+
 # -----------------------------------------------------------------------------
 # Every kernel instance on ragged sizes (tails, tiny tensors, empty tensors)
 # -----------------------------------------------------------------------------
