@@ -250,8 +250,9 @@ __device__ __forceinline__ Upd madam_update(const StepScalars& s, float w, float
 // only decides how much work that takes.
 // ---------------------------------------------------------------------------
 // FTZ selects the flushing forms.  Both forms are covered by the same bound
-// (flushing is the larger error); which one runs is a measured choice per
-// storage format: the flushing forms for BF16 weights, the others for E4M3.
+// (flushing is the larger error); every storage format uses the flushing
+// forms, which take fewer instructions (the non-flushing ones also handle
+// subnormal operands).
 template <bool FTZ>
 __device__ __forceinline__ float sqrt_approx(float x) {
   float y;
@@ -724,7 +725,7 @@ __device__ __forceinline__ void finish_group(const StepArgs& a, const TensorCtx&
     const float amax_f = fmaxf(__uint_as_float(amax_bits), x.amax_seed);
 #pragma unroll
     for (int j = 0; j < kGroup; ++j) {
-      const CertUpd u = madam_update_cert<false>(a.s, w[j], g[j], m[j], v[j], ve[j]);
+      const CertUpd u = madam_update_cert<true>(a.s, w[j], g[j], m[j], v[j], ve[j]);
       bool same;
       code[j] = e4m3_pair_normal<SR>(__fmul_rd(u.lo, x.enc_scale), __fmul_ru(u.hi, x.enc_scale),
                                      SR ? rnd[j] : 0u, same);
@@ -852,7 +853,7 @@ __device__ __forceinline__ void finish_block(const StepArgs& a, const TensorCtx&
     uint32_t bad = 0u;
 #pragma unroll
     for (int j = 0; j < kGroup; ++j) {
-      const CertUpd u = madam_update_cert<false>(a.s, w[j], g[j], m[j], v[j], ve[j]);
+      const CertUpd u = madam_update_cert<true>(a.s, w[j], g[j], m[j], v[j], ve[j]);
       wf[j] = u.wn;
       m[j] = u.m; v[j] = u.v; ve[j] = u.ve;
       if (!u.ok) {
@@ -1205,7 +1206,7 @@ __device__ __forceinline__ void finish_fp4(const StepArgs& a, const TensorCtx& x
     uint32_t bad = 0u;
 #pragma unroll
     for (int j = 0; j < kGroup; ++j) {
-      const CertUpd u = madam_update_cert<false>(a.s, w[j], g[j], m[j], v[j], ve[j]);
+      const CertUpd u = madam_update_cert<true>(a.s, w[j], g[j], m[j], v[j], ve[j]);
       wf[j] = u.wn;
       m[j] = u.m; v[j] = u.v; ve[j] = u.ve;
       if (!u.ok) {
