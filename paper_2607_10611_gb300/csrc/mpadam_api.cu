@@ -295,6 +295,8 @@ struct Group {
   int32_t cta_cap = 0;
   mpadam::PoolChunk* d_pool = nullptr;  // tail pool of the current grid (none when static_q is 1024)
   int32_t pool_chunks = 0, pool_cap = 0;
+  std::vector<TensorDesc> h_desc;       // host copies of its table entries (inline in short launches)
+  std::vector<TensorAux> h_aux;
 };
 
 struct mpadam_state {
@@ -327,8 +329,11 @@ struct mpadam_state {
   std::vector<int64_t> chunk_tile;            // chunk c covers tiles [chunk_tile[c], chunk_tile[c+1])
   std::vector<int64_t> chunk_elem;            // and global elements [chunk_elem[2c], chunk_elem[2c+1])
   int32_t* d_chunk_first = nullptr;           // [chunks][grid] CTA start tensors
-  // tail pool of mpadam_step's launches: static prefix of each CTA's range (1/1024) and chunk length
+  // tail pool of mpadam_step's launches: static prefix of each CTA's range (1/1024) and chunk length;
+  // until set_tail_pool is called, groups of fewer than kPoolMinTilesPerCta tiles per CTA keep
+  // static runs (with a tile or two per CTA, greedy claims would pile chunks on a few CTAs)
   int32_t pool_q = 768, pool_chunk = 4;
+  bool pool_set = false;
   uint32_t* d_pool_next = nullptr;            // [groups] claim counters, zeroed before each step
 };
 
@@ -450,11 +455,16 @@ int32_t upload_pool(Group& g, int32_t grid, int32_t q, int32_t chunk) {
   return MPADAM_OK;
 }
 
-// The static share a group's launches use (every format: per-tensor E4M3
-// groups too, since their consumers seed the exact-maximum threshold from the
-// amax ring after each tensor change).
+// The static share a group's launches use: every format (per-tensor E4M3
+// too, whose consumers seed the exact-maximum threshold from the amax ring
+// after each tensor change), but by default only groups with at least
+// kPoolMinTilesPerCta tiles per CTA.  A producer claims chunks while its ring
+// has free stages, so with a tile or two per CTA the first CTAs to reach the
+// pool take several chunks each and the launch waits on them (measured on a
+// 1 Mi-element list: 16.2 us pooled, 14.5 us static).
+constexpr int64_t kPoolMinTilesPerCta = 8;
 int32_t pool_q_of(const mpadam_state* s, const Group& g) {
-  (void)g;
+  if (!s->pool_set && g.tiles < kPoolMinTilesPerCta * g.grid) return 1024;
   return s->pool_q;
 }
 
@@ -619,6 +629,8 @@ int32_t create_state(const std::vector<TensorIn>& t, const mpadam_config* cfg, i
         s->tile_off[k] = g.tiles;
         desc.push_back(TensorDesc{t[k].w, t[k].m, t[k].v, t[k].ve, t[k].numel, s->goff[k], g.tiles, k, 0});
         aux.push_back(TensorAux{t[k].scale, t[k].compute, t[k].gscale, 0});
+        g.h_desc.push_back(desc.back());
+        g.h_aux.push_back(aux.back());
         g.aux = g.aux || t[k].scale != nullptr || t[k].compute != nullptr;
         g.numel.push_back(t[k].numel);
         g.tiles += tiles_of(t[k].numel);
@@ -710,6 +722,16 @@ int32_t launch_step(mpadam_state* s, const Group& g, int64_t step, cudaStream_t 
     a.pool_next = pool_next;
     a.pool_chunks = g.pool_chunks;
     a.static_q = pool_q_of(s, g);
+  }
+  if (tile_base == 0 && count == g.tiles && g.count <= mpadam::kInlineTensors) {
+    // a short whole-group launch carries its tables (the gradient pointers as
+    // staged for this step's upload, in group order)
+    a.n_inline = g.count;
+    for (int32_t i = 0; i < g.count; ++i) {
+      a.inl_desc[i] = g.h_desc[i];
+      a.inl_aux[i] = g.h_aux[i];
+      a.inl_grads[i] = s->h_grads[g.first + i];
+    }
   }
   fill_step(a, s->cfg, step);
   void* params[] = {&a};
@@ -862,6 +884,7 @@ int32_t mpadam_set_tail_pool(mpadam_state* s, int32_t static_q, int32_t chunk_ti
   if (e != cudaSuccess) return cuda_fail(e, "cudaDeviceSynchronize");
   s->pool_q = static_q;
   s->pool_chunk = chunk_tiles;
+  s->pool_set = true;
   for (auto& g : s->groups) {
     rc = upload_pool(g, g.grid, pool_q_of(s, g), s->pool_chunk);
     if (rc) return rc;

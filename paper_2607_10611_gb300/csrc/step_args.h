@@ -41,6 +41,7 @@ constexpr int kConsumers = 32 * kConsumerWarps;     // 480 consumer threads
 constexpr int kThreads = kConsumers + 32;           // + 1 producer warp
 constexpr int kTile = kConsumers * kGroup;          // 3840 elements per tile (16-byte multiple in every format)
 constexpr int kMaxStages = 8;
+constexpr int kInlineTensors = 4;                   // launches of at most this many tensors carry their tables inline
 constexpr int kPhiloxRounds = 10;
 constexpr int kBlock = 32;                          // elements per block scale (block-scaled E4M3)
 constexpr int kTileBlocks = kTile / kBlock;         // 120 block scales per tile (240 bytes)
@@ -132,7 +133,14 @@ struct StepArgs {
   const PoolChunk* pool;     // [pool_chunks] tail pool, or nullptr (static ranges only)
   uint32_t* pool_next;       // next unclaimed pool chunk; zero when the launch starts
   int32_t pool_chunks;
-  int32_t pad2;
+  // Launches of at most kInlineTensors tensors (a flat parameter buffer, a
+  // short list) carry their descriptors, aux entries and gradient pointers
+  // here as well, so that a CTA finds its first tensor and issues its first
+  // copies without dependent loads from global memory.  0: use the tables.
+  int32_t n_inline;
+  TensorDesc inl_desc[kInlineTensors];
+  TensorAux inl_aux[kInlineTensors];
+  const void* inl_grads[kInlineTensors];
 };
 
 // Kernel entry for the given formats (grad f32/bf16, moments f32/bf16,

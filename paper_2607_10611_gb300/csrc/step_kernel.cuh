@@ -233,6 +233,9 @@ __device__ __forceinline__ Upd madam_update(const StepScalars& s, float w, float
 // for an operand or result flushed from the subnormal range, the fast weight
 // wn' differs from the canonical wn by at most
 //     eps = (|w u_m'| + |u_a'|) 2^-17 + (|w + w u_m'| + |wn'|) 2^-22 + 2^-96
+// (computed in the looser form (|w u_m'| + |u_a'|)(2^-17 + 2^-20)
+// + |w| 2^-21 (1 + 2^-20) + 2^-96, since |t| <= (|w| + |w u_m'|)(1 + 2^-24)
+// and |wn'| <= (|t| + |u_a'|)(1 + 2^-24))
 // (the relative errors propagate through the divisions, the clamp is
 // 1-Lipschitz, each of the two final roundings adds at most one ulp, and the
 // constants carry a further factor-of-two margin).  Flushing stays inside
@@ -292,8 +295,10 @@ __device__ __forceinline__ CertUpd madam_update_cert(const StepScalars& s, float
   um = fmaxf(s.lo, fminf(um, s.hi));
   const float t = __fmaf_rn(w, um, w);
   o.wn = __fadd_rn(t, ua);
-  const float e = __fmaf_rn(__fadd_rn(fabsf(__fmul_rn(w, um)), fabsf(ua)), 7.62939453125e-06f /* 2^-17 */,
-                            __fmaf_rn(__fadd_rn(fabsf(t), fabsf(o.wn)), 2.384185791015625e-07f /* 2^-22 */,
+  // eps with (|t| + |wn'|) 2^-22 <= (2 |w| + 2 |w u_m'| + |u_a'|)(1 + 2^-23) 2^-22
+  // folded into the other two terms
+  const float e = __fmaf_rn(__fadd_rn(fabsf(__fmul_rn(w, um)), fabsf(ua)), 8.58306884765625e-06f /* 2^-17 + 2^-20 */,
+                            __fmaf_rn(fabsf(w), 4.768376129504759e-07f /* 2^-21 (1 + 2^-20) */,
                                       1.2621774483536189e-29f /* 2^-96 */));
   o.e = e;
   o.lo = __fsub_rd(o.wn, e);
@@ -571,6 +576,26 @@ __device__ __forceinline__ void put_e4m3(const uint32_t (&o)[2], void* g, int64_
 
 __host__ __device__ constexpr int esize_of(int dt) { return dt == kF32 ? 4 : (dt == kBF16 ? 2 : 1); }
 
+// A tensor's table entries: from the kernel parameters when the launch
+// carries them inline, else from global memory.
+__device__ __forceinline__ TensorDesc desc_of(const StepArgs& a, int k) {
+  return k < a.n_inline ? a.inl_desc[k] : a.desc[k];
+}
+__device__ __forceinline__ const void* grad_of(const StepArgs& a, int k) {
+  return k < a.n_inline ? a.inl_grads[k] : a.grads[k];
+}
+__device__ __forceinline__ TensorAux aux_of(const StepArgs& a, int k) {
+  return k < a.n_inline ? a.inl_aux[k] : a.aux[k];
+}
+// The tensor holding this CTA's first tile tb (which exists): scanned from
+// the inline descriptors, else the host-computed table.
+__device__ __forceinline__ int first_tensor(const StepArgs& a, int64_t tb) {
+  if (a.n_inline == 0) return a.cta_first[blockIdx.x];
+  int k = 0;
+  while (k < a.n_inline - 1 && a.inl_desc[k].tile_off + (a.inl_desc[k].numel + kTile - 1) / kTile <= tb) ++k;
+  return k;
+}
+
 // Per-tensor values the consumers keep while walking a tensor's tiles.
 struct TensorCtx {
   TensorDesc d;
@@ -588,8 +613,8 @@ struct TensorCtx {
 
 template <int WD, int GD, int MD>
 __device__ __forceinline__ void load_tensor(const StepArgs& a, int k, TensorCtx& c) {
-  c.d = a.desc[k];
-  c.g = a.grads[k];
+  c.d = desc_of(a, k);
+  c.g = grad_of(a, k);
   c.tiles = (c.d.numel + kTile - 1) / kTile;
   c.vec = aligned(c.d.w, WD == kBF16 ? 16 : (WD == kNVFP4 ? 4 : 8)) && aligned(c.g, GD == kF32 ? 32 : 16) &&
           aligned(c.d.m, MD == kF32 ? 32 : 16) && aligned(c.d.v, MD == kF32 ? 32 : 16) &&
@@ -601,8 +626,8 @@ __device__ __forceinline__ void load_tensor(const StepArgs& a, int k, TensorCtx&
   c.cc = nullptr;
   c.gscale = 1.0f;
   c.amax_seed = 0.0f;
-  if (WD != kBF16 && a.aux) {
-    const TensorAux x = a.aux[k];
+  if (WD != kBF16 && a.aux) {  // the launch has aux entries (inline ones too, when it carries its tables)
+    const TensorAux x = aux_of(a, k);
     c.scale = x.scale;
     c.cc = x.compute;
     c.gscale = x.gscale;
@@ -1034,19 +1059,27 @@ __device__ __forceinline__ uint32_t e2m1x2_rn(float x0, float x1) {
   return p;
 }
 
-// Stochastic E2M1 codes of both ends of an interval [xl, xh] (the same
-// random bits), sharing the binade of xl: the code of xl, and whether xh has
-// the same code (an end in another binade or sign reports false).
-__device__ __forceinline__ uint32_t e2m1_pair_sr(float xl, float xh, uint32_t r, bool& same) {
-  const float al = fminf(fabsf(xl), 6.0f), ah = fminf(fabsf(xh), 6.0f);
-  const float rsp = al < 2.0f ? 2.0f : (al < 4.0f ? 1.0f : 0.5f);
-  const uint32_t off = al < 2.0f ? 0u : (al < 4.0f ? 2u : 4u);
-  const float ql = __fmul_rn(al, rsp), qh = __fmul_rn(ah, rsp);  // exact (powers of two)
-  const float kl = truncf(ql), kh = truncf(qh);
-  const uint32_t ul = r < __float2uint_rz(__fmul_rn(__fsub_rn(ql, kl), 4294967296.0f)) ? 1u : 0u;
-  const uint32_t uh = r < __float2uint_rz(__fmul_rn(__fsub_rn(qh, kh), 4294967296.0f)) ? 1u : 0u;
-  same = kl == kh && ul == uh && ((__float_as_uint(xl) ^ __float_as_uint(xh)) >> 31) == 0u && xl == xl && xh == xh;
-  return ((__float_as_uint(xl) >> 28) & 8u) | (__float2uint_rz(kl) + off + ul);
+// Stochastic E2M1 code shared by every value of an interval of magnitudes
+// [xm, xM] (sign: that of q), decided from its smaller end xm alone, given
+// lim = 2^32 - W with W >= 2 (xM - xm) 2^32 + 1.  In xm's binade the grid
+// position is Q = |x| rsp (rsp = 2, 1, 1/2 on [0, 2), [2, 4), [4, 6]; 6 and
+// above saturate at Q = 3), exact in binary32; with k its integer part and
+// F = floor(frac(Q) 2^32), the code is off + k + [r < F].  Every binade edge
+// and the saturation point lie at an integer Q of xm's scale, and Q 2^32
+// grows by less than W over the interval (slope rsp <= 2); so when F + W and
+// ((F + 2^32 - 1 - r) mod 2^32) + W both stay below 2^32, no value of the
+// interval crosses a step or changes its rounding decision (same = true).
+// xm <= 0 or NaN (an interval reaching zero) reports false.
+__device__ __forceinline__ uint32_t e2m1_sr_interval(float xm, float q, uint32_t r, uint32_t lim, bool& same) {
+  const float am = fminf(xm, 6.0f);
+  const float rsp = am < 2.0f ? 2.0f : (am < 4.0f ? 1.0f : 0.5f);
+  const uint32_t off = am < 2.0f ? 0u : (am < 4.0f ? 2u : 4u);
+  const float qq = __fmul_rn(am, rsp);  // exact (a power of two)
+  const float kf = truncf(qq);
+  const uint32_t F = __float2uint_rz(__fmul_rn(__fsub_rn(qq, kf), 4294967296.0f));  // exact
+  const uint32_t sl = F + ~r;
+  same = xm > 0.0f && max(F, sl) < lim;
+  return ((__float_as_uint(q) >> 28) & 8u) | (__float2uint_rz(kf) + off + (r < F ? 1u : 0u));
 }
 
 // A block scale code with the two products its covering test and the encode
@@ -1260,12 +1293,23 @@ __device__ __forceinline__ void finish_fp4(const StepArgs& a, const TensorCtx& x
       if (SR) {
         uint32_t rnd[8];
         group_random_bits<kNVFP4>(a, gi << 3, rnd);
+        // lim = 2^32 - W for the group.  An interval's magnitudes span
+        // xM - xm <= 2.3 e2 (e2 of ends(), plus one directed rounding at each
+        // end, each within e2 / 8 since e2 >= |q| 2^-20), and e2 <=
+        // (8 2^-20 + ei)(1 + 2^-23) while |q| <= 8; so 2 (xM - xm) 2^32 + 1 <=
+        // (2^-17 + ei) 2^35 + 2.  Larger |q| saturates at both ends (or, with
+        // ei > 1, leaves lim = 0: nothing is certified).
+        const float wq = __fmaf_ru(ei, 34359738368.0f /* 2^35 */, 262144.0f /* 2^18 */);
+        const uint32_t lim = __float2uint_rd(__fsub_rd(4294967296.0f, __fadd_ru(wq, 2.0f)));
 #pragma unroll
         for (int j = 0; j < kGroup; ++j) {
-          float xl, xh;
-          ends(j, xl, xh);
+          const float q = __fmul_rn(wf[j], inv);
+          const float aq = fabsf(q);
+          // a lower bound of the smaller magnitude of ends() (|q| - e2, up to
+          // its roundings): |q| (1 - 2^-20) - ei, rounded down once
+          const float xm = __fmaf_rd(aq, 0.99999904632568359375f /* 1 - 2^-20 */, -ei);
           bool same;
-          packed |= (e2m1_pair_sr(xl, xh, rnd[j], same) & 0xFu) << (4 * j);
+          packed |= (e2m1_sr_interval(xm, q, rnd[j], lim, same) & 0xFu) << (4 * j);
           if (!same) redo |= 1u << j;
         }
       } else {  // two elements at a time, both ends
@@ -1433,13 +1477,13 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
     int64_t tiles = 0;
     auto load = [&](int kk) {
       k = kk;
-      d = a.desc[k];
-      gp = a.grads[k];
-      if (WD == kE4M3B || WD == kNVFP4) sp = static_cast<const uint8_t*>(a.aux[k].scale);
+      d = desc_of(a, k);
+      gp = grad_of(a, k);
+      if (WD == kE4M3B || WD == kNVFP4) sp = static_cast<const uint8_t*>(aux_of(a, k).scale);
       tiles = (d.numel + kTile - 1) / kTile;
     };
     int64_t t = tb, t_end = ts;  // the current run of consecutive tiles
-    if (t < t_end) load(a.cta_first[blockIdx.x]);
+    if (t < t_end) load(first_tensor(a, tb));
     int s = 0;
     uint32_t use = 0;
     int64_t issued = 0;
@@ -1534,7 +1578,7 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
   };
   // The first tile posted is the first of this CTA's own range when it has
   // one: take up its tensor while the copies are in flight.
-  if (tb < ts) enter(a.cta_first[blockIdx.x]);
+  if (tb < ts) enter(first_tensor(a, tb));
   uint32_t amax_bits = 0u;
   int s = 0;
   uint32_t use = 0;
