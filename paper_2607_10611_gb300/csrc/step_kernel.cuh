@@ -707,21 +707,23 @@ __device__ __forceinline__ void finish_group(const StepArgs& a, const TensorCtx&
   if (SR) group_random_bits<WD>(a, static_cast<uint64_t>(x.d.goff + e0), rnd);
 
   if (WD == kBF16 && !OPT && a.s.cert_ok) {  // certified fast path (see madam_update_cert)
-    uint32_t out[8];
+    uint32_t ow[4] = {0u, 0u, 0u, 0u};
     uint32_t redo = 0u;
 #pragma unroll
     for (int j = 0; j < kGroup; ++j) {
       const CertUpd u = madam_update_cert<true>(a.s, w[j], g[j], m[j], v[j], ve[j]);
       bool same;
+      uint32_t code;
       if (SR) {
         const uint32_t slo = __float_as_uint(u.lo) + rnd[j], shi = __float_as_uint(u.hi) + rnd[j];
         same = ((slo ^ shi) >> 16) == 0u;
-        out[j] = slo >> 16;
+        code = slo >> 16;
       } else {
         const uint32_t pair = bf16x2_rn(u.lo, u.hi);
         same = ((pair ^ (pair >> 16)) & 0xFFFFu) == 0u;
-        out[j] = pair & 0xFFFFu;
+        code = pair & 0xFFFFu;
       }
+      ow[j >> 1] |= code << (16 * (j & 1));
       if (!(u.ok && same)) redo |= 1u << j;
       m[j] = u.m; v[j] = u.v; ve[j] = u.ve;
     }
@@ -730,13 +732,12 @@ __device__ __forceinline__ void finish_group(const StepArgs& a, const TensorCtx&
       for (int j = 0; j < kGroup; ++j) {
         if ((redo >> j) & 1u) {
           const float xe = madam_wn_exact(a.s, w[j], g[j], m[j], v[j], ve[j]);
-          out[j] = SR ? (bf16_sr_sum(xe, rnd[j]) >> 16) : (bf16x2_rn(xe, xe) & 0xFFFFu);
+          const uint32_t code = SR ? (bf16_sr_sum(xe, rnd[j]) >> 16) : (bf16x2_rn(xe, xe) & 0xFFFFu);
+          const int sh = 16 * (j & 1);
+          ow[j >> 1] = (ow[j >> 1] & ~(0xFFFFu << sh)) | (code << sh);
         }
       }
     }
-    uint32_t ow[4];
-#pragma unroll
-    for (int i = 0; i < 4; ++i) ow[i] = out[2 * i] | (out[2 * i + 1] << 16);
     put_bf16(ow, x.d.w, e0, valid, x.vec);
   } else if (WD == kE4M3 && !OPT && a.s.cert_ok) {
     // Certified fast path for E4M3: both ends of the bound are scaled by 2^-e
@@ -745,15 +746,18 @@ __device__ __forceinline__ void finish_group(const StepArgs& a, const TensorCtx&
     // threshold is the larger of this thread's running maximum and the
     // tensor's maximum flushed so far in this step: both are exact |w'| of
     // elements of this tensor, so no element below them can be the maximum.
-    uint32_t code[8];
+    uint32_t ow[2] = {0u, 0u};
     uint32_t redo = 0u;
     const float amax_f = fmaxf(__uint_as_float(amax_bits), x.amax_seed);
 #pragma unroll
     for (int j = 0; j < kGroup; ++j) {
       const CertUpd u = madam_update_cert<true>(a.s, w[j], g[j], m[j], v[j], ve[j]);
       bool same;
-      code[j] = e4m3_pair_normal<SR>(__fmul_rd(u.lo, x.enc_scale), __fmul_ru(u.hi, x.enc_scale),
-                                     SR ? rnd[j] : 0u, same);
+      const uint32_t code = e4m3_pair_normal<SR>(__fmul_rd(u.lo, x.enc_scale), __fmul_ru(u.hi, x.enc_scale),
+                                                 SR ? rnd[j] : 0u, same);
+      // an undecided element's code may be out of range (it is replaced
+      // below): keep it inside its own byte
+      ow[j >> 2] |= (code & 0xFFu) << (8 * (j & 3));
       if (!(u.ok && same) || fmaxf(fabsf(u.lo), fabsf(u.hi)) >= amax_f) redo |= 1u << j;
       m[j] = u.m; v[j] = u.v; ve[j] = u.ve;
     }
@@ -764,13 +768,12 @@ __device__ __forceinline__ void finish_group(const StepArgs& a, const TensorCtx&
           const float xe = madam_wn_exact(a.s, w[j], g[j], m[j], v[j], ve[j]);
           const uint32_t wb = __float_as_uint(xe) & 0x7FFFFFFFu;
           if (j < valid && wb < 0x7F800000u) amax_bits = max(amax_bits, wb);
-          code[j] = e4m3_encode<SR>(__fmul_rn(xe, x.enc_scale), SR ? rnd[j] : 0u);
+          const uint32_t code = e4m3_encode<SR>(__fmul_rn(xe, x.enc_scale), SR ? rnd[j] : 0u);
+          const int sh = 8 * (j & 3);
+          ow[j >> 2] = (ow[j >> 2] & ~(0xFFu << sh)) | (code << sh);
         }
       }
     }
-    uint32_t ow[2];
-    ow[0] = code[0] | (code[1] << 8) | (code[2] << 16) | (code[3] << 24);
-    ow[1] = code[4] | (code[5] << 8) | (code[6] << 16) | (code[7] << 24);
     put_e4m3(ow, x.d.w, e0, valid, x.vec);
     if (x.cc) put_compute(ow, x.cc_scale, x.cc, e0, valid, x.vec);
   } else {

@@ -165,6 +165,34 @@ def test_nan_and_inf_propagate_like_the_oracle(wd):
 
 
 # -----------------------------------------------------------------------------
+# E4M3 codes over their whole range (subnormal codes, values far below the
+# smallest code after the update, saturation), where the certified path's
+# fast encode is out of range and the exact branch must take over without
+# touching its neighbours' bytes
+# -----------------------------------------------------------------------------
+@pytest.mark.parametrize("md", ["f32", "bf16"])
+@pytest.mark.parametrize("rnd", ["nearest", "stochastic"])
+def test_e4m3_codes_over_their_whole_range(md, rnd):
+    import torch
+    p = P()
+    wl = W.replace(W.SMALL["llama_1p5b"], moment_dtype=md, rounding=rnd, name="e4m3_all_codes")
+    mt = W.materialize(wl, "cpu", warm_state=True)
+    gen = torch.Generator().manual_seed(5)
+    finite = torch.tensor([c for c in range(256) if c & 0x7F != 0x7F], dtype=torch.uint8)
+    for k, w in enumerate(mt.w):
+        w.copy_(finite[torch.randint(0, finite.numel(), (w.numel(),), generator=gen)])
+    r = p.Run(wl, mt=mt, hp=dict(lr_add=1e-2, lr_mul=0.05))
+    try:
+        for t in range(1, 5):
+            r.step(t)
+            res = r.compare(t + 1)
+            assert res["contract_ok"]
+            p.assert_exact(res, f"all codes {md}/{rnd} step {t}")
+    finally:
+        r.close()
+
+
+# -----------------------------------------------------------------------------
 # Launch shape and list structure do not change any bit
 # -----------------------------------------------------------------------------
 def test_grid_size_does_not_change_results():
