@@ -696,12 +696,56 @@ __device__ __forceinline__ void group_random_bits(const StepArgs& a, uint64_t gi
   }
 }
 
+// The canonical weight of slot j of consumer c (a runtime index), from the
+// original inputs in the stage at st (BF16 weights, or E4M3 codes times
+// `scale`); the stage must still be allocated.
+template <int WD, int GD, int MD>
+__device__ __forceinline__ float exact_wn_from_stage(const StepArgs& a, uint32_t st, int c, int j, float scale) {
+  constexpr int GS = esize_of(GD), MS = esize_of(MD);
+  const uint32_t i = static_cast<uint32_t>(kGroup * c + j);
+  const float w =
+      WD == kBF16 ? __uint_as_float(lds_u16(st + 2u * i) << 16) : __fmul_rn(e4m3_value(lds_u8(st + i)), scale);
+  auto ld = [&](uint32_t base, int es) -> float {
+    return es == 4 ? __uint_as_float(lds_u32(base + 4u * i)) : __uint_as_float(lds_u16(base + 2u * i) << 16);
+  };
+  return madam_update<false>(a.s, w, ld(st + a.off_g, GS), ld(st + a.off_m, MS), ld(st + a.off_v, MS),
+                             ld(st + a.off_ve, MS)).wn;
+}
+
+// The random lane of element j (a runtime index) of the group starting at
+// global index gidx, as group_random_bits draws it: one Philox block.
+template <int WD>
+__device__ __forceinline__ uint32_t element_random_bits(const StepArgs& a, uint64_t gidx, int j) {
+  const uint64_t gi = gidx >> 3;
+  if (WD == kBF16) {
+    const uint4 r = philox4x32_10(static_cast<uint32_t>(gi), static_cast<uint32_t>(gi >> 32), a.t_lo, a.t_hi,
+                                  a.rk0, a.rk1);
+    const int q = j >> 1;
+    const uint32_t wd = q == 0 ? r.x : (q == 1 ? r.y : (q == 2 ? r.z : r.w));
+    return (j & 1) ? (~wd >> 16) : (~wd & 0xFFFFu);
+  } else {
+    const uint64_t b = 2ull * gi + static_cast<uint64_t>(j >> 2);
+    const uint4 r = philox4x32_10(static_cast<uint32_t>(b), static_cast<uint32_t>(b >> 32), a.t_lo, a.t_hi,
+                                  a.rk0, a.rk1);
+    const int q = j & 3;
+    return q == 0 ? r.x : (q == 1 ? r.y : (q == 2 ? r.z : r.w));
+  }
+}
+
 // Update 8 loaded elements and store them (vector stores when `vec` and
-// whole, else element by element).
-template <int WD, int GD, int MD, bool SR, bool OPT>
+// whole, else element by element).  STAGED (BF16 weights, whole staged
+// tiles): the stage at st stays allocated until this returns, and the
+// certified path's rare exact branch takes the undecided elements one at a
+// time from there (c: the consumer), in a loop over the set bits.  Otherwise
+// that branch uses the inputs held in registers.  (Measured on the 7B list:
+// keeping the inputs live through the certified loop for the exact branch,
+// 18.64 ms per step; this, 18.27 ms.  Reloading them from global memory was
+// slower still, 21.6 ms: about a tenth of the warps' groups take the branch,
+// and each reload waits on DRAM while the other warps wait for its stage.)
+template <int WD, int GD, int MD, bool SR, bool OPT, bool STAGED>
 __device__ __forceinline__ void finish_group(const StepArgs& a, const TensorCtx& x, int64_t e0, int valid,
                                              float (&w)[8], float (&g)[8], float (&m)[8], float (&v)[8],
-                                             float (&ve)[8], uint32_t& amax_bits) {
+                                             float (&ve)[8], uint32_t& amax_bits, uint32_t st, int c) {
   // random bits: one Philox block per 8 BF16 lanes, two per 8 E4M3 lanes
   uint32_t rnd[8];
   if (SR) group_random_bits<WD>(a, static_cast<uint64_t>(x.d.goff + e0), rnd);
@@ -728,13 +772,28 @@ __device__ __forceinline__ void finish_group(const StepArgs& a, const TensorCtx&
       m[j] = u.m; v[j] = u.v; ve[j] = u.ve;
     }
     if (redo) {  // rare: encode the canonical weight of the undecided elements
-#pragma unroll
-      for (int j = 0; j < kGroup; ++j) {
-        if ((redo >> j) & 1u) {
-          const float xe = madam_wn_exact(a.s, w[j], g[j], m[j], v[j], ve[j]);
-          const uint32_t code = SR ? (bf16_sr_sum(xe, rnd[j]) >> 16) : (bf16x2_rn(xe, xe) & 0xFFFFu);
+      if constexpr (STAGED) {
+#pragma unroll 1
+        for (uint32_t rm = redo; rm != 0u; rm &= rm - 1u) {
+          const int j = __ffs(rm) - 1;
+          const float xe = exact_wn_from_stage<kBF16, GD, MD>(a, st, c, j, 1.0f);
+          const uint32_t code =
+              SR ? (bf16_sr_sum(xe, element_random_bits<kBF16>(a, static_cast<uint64_t>(x.d.goff + e0), j)) >> 16)
+                 : (bf16x2_rn(xe, xe) & 0xFFFFu);
           const int sh = 16 * (j & 1);
-          ow[j >> 1] = (ow[j >> 1] & ~(0xFFFFu << sh)) | (code << sh);
+#pragma unroll
+          for (int i = 0; i < 4; ++i)
+            if (i == (j >> 1)) ow[i] = (ow[i] & ~(0xFFFFu << sh)) | (code << sh);
+        }
+      } else {
+#pragma unroll
+        for (int j = 0; j < kGroup; ++j) {
+          if ((redo >> j) & 1u) {
+            const float xe = madam_wn_exact(a.s, w[j], g[j], m[j], v[j], ve[j]);
+            const uint32_t code = SR ? (bf16_sr_sum(xe, rnd[j]) >> 16) : (bf16x2_rn(xe, xe) & 0xFFFFu);
+            const int sh = 16 * (j & 1);
+            ow[j >> 1] = (ow[j >> 1] & ~(0xFFFFu << sh)) | (code << sh);
+          }
         }
       }
     }
@@ -841,7 +900,7 @@ __device__ __noinline__ uint32_t general_group(const StepArgs& a, const TensorCt
     get_bf16<false>(v, v_st, st + a.off_v + kGroup * MS * c, x.d.v, e0, valid, x.vec);
     get_bf16<false>(ve, e_st, st + a.off_ve + kGroup * MS * c, x.d.ve, e0, valid, x.vec);
   }
-  finish_group<WD, GD, MD, SR, OPT>(a, x, e0, valid, w, g, m, v, ve, amax_bits);
+  finish_group<WD, GD, MD, SR, OPT, false>(a, x, e0, valid, w, g, m, v, ve, amax_bits, st, c);
   return amax_bits;
 }
 
@@ -1646,11 +1705,17 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
         finish_fp4<GD, MD, SR, OPT, kExactStage>(a, x, e0, kGroup, h_old, w, g, m, v, ve, st, c);
         __syncwarp();
         if (lane == 0) mbar_arrive(smem_addr(&empty_bar[s]));
+      } else if constexpr (WD == kBF16) {
+        // the stage stays until the group is done: the rare exact branch reads
+        // its inputs there
+        finish_group<WD, GD, MD, SR, OPT, true>(a, x, e0, kGroup, w, g, m, v, ve, amax_bits, st, c);
+        __syncwarp();
+        if (lane == 0) mbar_arrive(smem_addr(&empty_bar[s]));
       } else {
         __syncwarp();
         if (lane == 0) mbar_arrive(smem_addr(&empty_bar[s]));
         if constexpr (WD == kE4M3B) finish_block<GD, MD, SR, OPT>(a, x, e0, kGroup, h_old, w, g, m, v, ve);
-        else finish_group<WD, GD, MD, SR, OPT>(a, x, e0, kGroup, w, g, m, v, ve, amax_bits);
+        else finish_group<WD, GD, MD, SR, OPT, false>(a, x, e0, kGroup, w, g, m, v, ve, amax_bits, st, c);
       }
       if (++s == S) { s = 0; ++use; }
       continue;
