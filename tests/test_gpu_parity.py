@@ -165,6 +165,28 @@ def test_nan_and_inf_propagate_like_the_oracle(wd):
 
 
 # -----------------------------------------------------------------------------
+# Many undecided elements: large learning rates (eta_m = 4 is the largest the
+# certified path accepts) widen its error bound several times, so whole tiles
+# send many more elements through the exact branch (for BF16 weights, one
+# element at a time from the stage, with its random lane drawn again)
+# -----------------------------------------------------------------------------
+@pytest.mark.parametrize("wd", ["bf16", "e4m3"])
+@pytest.mark.parametrize("gd,md", [("bf16", "bf16"), ("f32", "f32"), ("bf16", "f32")])
+@pytest.mark.parametrize("rnd", ["nearest", "stochastic"])
+def test_many_undecided_elements(wd, gd, md, rnd):
+    p = P()
+    wl = W.replace(W.SMALL["llama_7b"], weight_dtype=wd, grad_dtype=gd, moment_dtype=md, rounding=rnd,
+                   name=f"undecided_{wd}")
+    r = p.Run(wl, warm=True, hp=dict(lr_mul=4.0, lr_add=0.3))
+    try:
+        for t in range(1, 4):
+            r.step(t)
+            p.assert_exact(r.compare(t + 1), f"{wd}/{gd}/{md}/{rnd} step {t}")
+    finally:
+        r.close()
+
+
+# -----------------------------------------------------------------------------
 # E4M3 codes over their whole range (subnormal codes, values far below the
 # smallest code after the update, saturation), where the certified path's
 # fast encode is out of range and the exact branch must take over without
