@@ -291,16 +291,34 @@ def run_gpu(wl, steps: int, warmup: int, rank: int, e2e_steps: int, flush_l2: bo
         # page-locked host buffers: huge-page ones from mpadam_host_buffer_alloc,
         # or the driver's (torch pin_memory), whichever copies faster here
         from paper_2607_10611_gb300.optimizer import HostBuffer
-        kind = pinned_kind_for_this_host(stream)
-        if kind == "huge_pages":
-            hg_buf = HostBuffer(mt.flat["g"].numel(), mt.flat["g"].dtype)
-            hw_buf = HostBuffer(mt.flat["w"].numel(), mt.flat["w"].dtype)
-            hg, hw = hg_buf.tensor, hw_buf.tensor
-        else:
-            hg_buf = hw_buf = None
-            hg = torch.empty(mt.flat["g"].shape, dtype=mt.flat["g"].dtype, pin_memory=True)
-            hw = torch.empty(mt.flat["w"].shape, dtype=mt.flat["w"].dtype, pin_memory=True)
+        probe = pinned_probe_gbs(stream)
+        kinds = sorted(probe, key=lambda k: -probe[k])
+        nbytes = sum(x.numel() for x in mt.g) * BYTES[wl.grad_dtype] + sum(x.numel() for x in mt.w) * BYTES[wl.weight_dtype]
+        for attempt, kind in enumerate(kinds):
+            if kind == "huge_pages":
+                hg_buf = HostBuffer(mt.flat["g"].numel(), mt.flat["g"].dtype)
+                hw_buf = HostBuffer(mt.flat["w"].numel(), mt.flat["w"].dtype)
+                hg, hw = hg_buf.tensor, hw_buf.tensor
+            else:
+                hg_buf = hw_buf = None
+                hg = torch.empty(mt.flat["g"].shape, dtype=mt.flat["g"].dtype, pin_memory=True)
+                hw = torch.empty(mt.flat["w"].shape, dtype=mt.flat["w"].dtype, pin_memory=True)
+            # the full-size buffers can land elsewhere than the 1 GiB probe's
+            # (pages on a far memory node once the near one is full): check the
+            # link on them, and take the other kind if they run at under half
+            # the probe's rate
+            link = host_link_ms(hg, mt.flat["g"], hw, mt.flat["w"], stream)
+            gbs = nbytes / (link * 1e-3) / 1e9
+            if gbs >= 0.5 * probe[kind] or attempt == len(kinds) - 1:
+                break
+            del hg, hw
+            if hg_buf is not None:
+                hg_buf.free()
+                hw_buf.free()
+            torch.cuda.synchronize()
         res["host_buffers"] = kind
+        res["host_probe_gbs"] = {k: round(v, 1) for k, v in probe.items()}
+        res["host_buffers_tried"] = attempt + 1
         hg.copy_(mt.flat["g"])
         hgs = [hg[o:o + x.numel()] for o, x in zip(mt.offsets, mt.g)]
         hws = [hw[o:o + x.numel()] for o, x in zip(mt.offsets, mt.w)]
@@ -353,9 +371,10 @@ def same_size_copy_ms(nbytes: float, flush, flush_rd, stream, reps: int = 20) ->
     return sorted(ts)[len(ts) // 2]
 
 
-def pinned_kind_for_this_host(stream) -> str:
-    """'huge_pages' (mpadam_host_buffer_alloc) or 'driver' (torch pin_memory):
-    the faster of a 1 GiB host-to-device copy from each, best of three."""
+def pinned_probe_gbs(stream) -> dict:
+    """GB/s of a 1 GiB host-to-device copy from each kind of page-locked host
+    buffer, best of three: 'huge_pages' (mpadam_host_buffer_alloc) and
+    'driver' (torch pin_memory)."""
     import torch
     from paper_2607_10611_gb300.optimizer import HostBuffer
     n = 1 << 29
@@ -377,7 +396,7 @@ def pinned_kind_for_this_host(stream) -> str:
     hp = torch.empty(n, dtype=torch.bfloat16, pin_memory=True)
     t_drv = best(hp)
     del hp, dev
-    return "huge_pages" if t_huge <= t_drv else "driver"
+    return {"huge_pages": 2 * n / (t_huge * 1e-3) / 1e9, "driver": 2 * n / (t_drv * 1e-3) / 1e9}
 
 
 def host_link_ms(h_src, d_dst, h_dst, d_src, stream, reps: int = 3) -> float:
@@ -497,7 +516,8 @@ def summarize(wl, res, n_gpus, peak, peak_kind):
                       "host_link_gbs": round((res["h2d"] + res["d2h"]) / (res["link_ms"] * 1e-3) / 1e9, 1),
                       "frac_of_host_link_bound": round(res["link_ms"] / res["e2e_ms"], 4),
                       "frac_of_host_link_bound_median": round(res["link_ms"] / med, 4),
-                      "host_buffers": res.get("host_buffers")}
+                      "host_buffers": res.get("host_buffers"), "host_probe_gbs": res.get("host_probe_gbs"),
+                      "host_buffers_tried": res.get("host_buffers_tried")}
     return out
 
 

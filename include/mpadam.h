@@ -320,8 +320,10 @@ int32_t mpadam_launch_info(const mpadam_state* s, int32_t* ctas, int32_t* thread
  * chunk_tiles tiles, which the CTAs that finish first claim one at a time.
  * SMs do not all stream memory at the same rate, so without the pool a
  * launch waits on the slowest.  static_q = 1024 turns the pool off.
- * Default: static_q = 768, chunk_tiles = 4, for every weight format.
- * Results do not depend on either value.
+ * Default: static_q = 768, chunk_tiles = 4, for every weight format, except
+ * that until this is called a format group with fewer than 8 tiles per CTA
+ * keeps static runs (with a tile or two per CTA the pool's first claimants
+ * would take several chunks each).  Results do not depend on any of this.
  * Synchronises the device.  The host-buffer and allocation-free entry
  * points always use static runs.
  * Errors: EINVAL (static_q outside [0, 1024], chunk_tiles outside

@@ -697,14 +697,13 @@ __device__ __forceinline__ void group_random_bits(const StepArgs& a, uint64_t gi
 }
 
 // The canonical weight of slot j of consumer c (a runtime index), from the
-// original inputs in the stage at st (BF16 weights, or E4M3 codes times
-// `scale`); the stage must still be allocated.
-template <int WD, int GD, int MD>
-__device__ __forceinline__ float exact_wn_from_stage(const StepArgs& a, uint32_t st, int c, int j, float scale) {
+// original inputs in the stage at st (BF16 weights); the stage must still be
+// allocated.
+template <int GD, int MD>
+__device__ __forceinline__ float exact_wn_from_stage(const StepArgs& a, uint32_t st, int c, int j) {
   constexpr int GS = esize_of(GD), MS = esize_of(MD);
   const uint32_t i = static_cast<uint32_t>(kGroup * c + j);
-  const float w =
-      WD == kBF16 ? __uint_as_float(lds_u16(st + 2u * i) << 16) : __fmul_rn(e4m3_value(lds_u8(st + i)), scale);
+  const float w = __uint_as_float(lds_u16(st + 2u * i) << 16);
   auto ld = [&](uint32_t base, int es) -> float {
     return es == 4 ? __uint_as_float(lds_u32(base + 4u * i)) : __uint_as_float(lds_u16(base + 2u * i) << 16);
   };
@@ -712,24 +711,15 @@ __device__ __forceinline__ float exact_wn_from_stage(const StepArgs& a, uint32_t
                              ld(st + a.off_ve, MS)).wn;
 }
 
-// The random lane of element j (a runtime index) of the group starting at
-// global index gidx, as group_random_bits draws it: one Philox block.
-template <int WD>
-__device__ __forceinline__ uint32_t element_random_bits(const StepArgs& a, uint64_t gidx, int j) {
+// The complemented 16-bit random lane of BF16 element j (a runtime index) of
+// the group starting at global index gidx, as group_random_bits draws it.
+__device__ __forceinline__ uint32_t bf16_element_random_bits(const StepArgs& a, uint64_t gidx, int j) {
   const uint64_t gi = gidx >> 3;
-  if (WD == kBF16) {
-    const uint4 r = philox4x32_10(static_cast<uint32_t>(gi), static_cast<uint32_t>(gi >> 32), a.t_lo, a.t_hi,
-                                  a.rk0, a.rk1);
-    const int q = j >> 1;
-    const uint32_t wd = q == 0 ? r.x : (q == 1 ? r.y : (q == 2 ? r.z : r.w));
-    return (j & 1) ? (~wd >> 16) : (~wd & 0xFFFFu);
-  } else {
-    const uint64_t b = 2ull * gi + static_cast<uint64_t>(j >> 2);
-    const uint4 r = philox4x32_10(static_cast<uint32_t>(b), static_cast<uint32_t>(b >> 32), a.t_lo, a.t_hi,
-                                  a.rk0, a.rk1);
-    const int q = j & 3;
-    return q == 0 ? r.x : (q == 1 ? r.y : (q == 2 ? r.z : r.w));
-  }
+  const uint4 r = philox4x32_10(static_cast<uint32_t>(gi), static_cast<uint32_t>(gi >> 32), a.t_lo, a.t_hi,
+                                a.rk0, a.rk1);
+  const int q = j >> 1;
+  const uint32_t wd = q == 0 ? r.x : (q == 1 ? r.y : (q == 2 ? r.z : r.w));
+  return (j & 1) ? (~wd >> 16) : (~wd & 0xFFFFu);
 }
 
 // Update 8 loaded elements and store them (vector stores when `vec` and
@@ -776,9 +766,9 @@ __device__ __forceinline__ void finish_group(const StepArgs& a, const TensorCtx&
 #pragma unroll 1
         for (uint32_t rm = redo; rm != 0u; rm &= rm - 1u) {
           const int j = __ffs(rm) - 1;
-          const float xe = exact_wn_from_stage<kBF16, GD, MD>(a, st, c, j, 1.0f);
+          const float xe = exact_wn_from_stage<GD, MD>(a, st, c, j);
           const uint32_t code =
-              SR ? (bf16_sr_sum(xe, element_random_bits<kBF16>(a, static_cast<uint64_t>(x.d.goff + e0), j)) >> 16)
+              SR ? (bf16_sr_sum(xe, bf16_element_random_bits(a, static_cast<uint64_t>(x.d.goff + e0), j)) >> 16)
                  : (bf16x2_rn(xe, xe) & 0xFFFFu);
           const int sh = 16 * (j & 1);
 #pragma unroll

@@ -123,7 +123,8 @@ def _fake_res(wl, ms, e2e=False):
            "l2_flushed": wl.name == "flat_1m", "copy_ms": 0.0081234567 if wl.name == "flat_1m" else None}
     if e2e:
         res.update(e2e_ms=101.234567, e2e_step_ms=[100.0 + 1.2345678 * i for i in range(20)],
-                   h2d=13476831232, d2h=13476831232, link_ms=94.12345678, host_buffers="huge_pages")
+                   h2d=13476831232, d2h=13476831232, link_ms=94.12345678, host_buffers="huge_pages",
+                   host_probe_gbs={"huge_pages": 212.3, "driver": 204.9}, host_buffers_tried=2)
     return res
 
 
