@@ -303,9 +303,14 @@ __device__ __forceinline__ CertUpd madam_update_cert(const StepScalars& s, float
   o.e = e;
   o.lo = __fsub_rd(o.wn, e);
   o.hi = __fadd_ru(o.wn, e);
-  // divisors must stay below 2^125 (their lower bounds eps, tau >= 2^-125 are
-  // checked on the host), and wn' must be finite
-  o.ok = fmaxf(fmaxf(den_a, den_e), rho) <= 4.253529586511731e+37f /* 2^125 */ && fabsf(o.wn) < INFINITY;
+  // The two denominators must stay below 2^125 (their lower bound eps >=
+  // 2^-28 is checked on the host), and wn' must be finite.  The third divisor,
+  // rho = max(|w|, tau) >= tau >= 2^-125, needs no upper check: when |w| >
+  // 2^125 the canonical |w u_m| <= eta_m |n| <= 4 (1 - beta2)^(-1/2) <= 2^14
+  // (nu_e' >= (1 - beta2) g_e^2 bounds |n|; eta_m <= 4 on the host) is far
+  // below half an ulp of w, so w + w u_m rounds to w, as it does with the
+  // approximate quotient (documented within 2 ulp up to 2^126 and 0 above).
+  o.ok = fmaxf(den_a, den_e) <= 4.253529586511731e+37f /* 2^125 */ && fabsf(o.wn) < INFINITY;
   return o;
 }
 
@@ -1346,22 +1351,26 @@ __device__ __forceinline__ void finish_fp4(const StepArgs& a, const TensorCtx& x
         uint32_t rnd[8];
         group_random_bits<kNVFP4>(a, gi << 3, rnd);
         // lim = 2^32 - W for the group.  An interval's magnitudes span
-        // xM - xm <= 2.3 e2 (e2 of ends(), plus one directed rounding at each
-        // end, each within e2 / 8 since e2 >= |q| 2^-20), and e2 <=
-        // (8 2^-20 + ei)(1 + 2^-23) while |q| <= 8; so 2 (xM - xm) 2^32 + 1 <=
+        // xM - xm <= 3.5 e2: 2 e2 from ends() (e2 its bound), one directed
+        // rounding at each end (each within e2 / 8, since e2 >= |q| 2^-20)
+        // and the lower end below taken |q| 2^-20 lower still.  With e2 <=
+        // (8 2^-20 + ei)(1 + 2^-23) while |q| <= 8, 2 (xM - xm) 2^32 + 1 <=
         // (2^-17 + ei) 2^35 + 2.  Larger |q| saturates at both ends (or, with
         // ei > 1, leaves lim = 0: nothing is certified).
-        const float wq = __fmaf_ru(ei, 34359738368.0f /* 2^35 */, 262144.0f /* 2^18 */);
-        const uint32_t lim = __float2uint_rd(__fsub_rd(4294967296.0f, __fadd_ru(wq, 2.0f)));
+        const uint32_t lim =
+            ei <= 5.9604644775390625e-08f /* 2^-24 */
+                ? 4294701056u /* 2^32 - (2^18 + 2^12): W <= 2^18 + 2^11 + 2 when ei <= 2^-24 */
+                : __float2uint_rd(__fsub_rd(4294967296.0f,
+                                            __fadd_ru(__fmaf_ru(ei, 34359738368.0f /* 2^35 */, 262144.0f /* 2^18 */),
+                                                      2.0f)));
+        const float inv_lo = __fmul_rd(inv, 0.999998092651367188f /* 1 - 2^-19 */);
 #pragma unroll
         for (int j = 0; j < kGroup; ++j) {
-          const float q = __fmul_rn(wf[j], inv);
-          const float aq = fabsf(q);
-          // a lower bound of the smaller magnitude of ends() (|q| - e2, up to
-          // its roundings): |q| (1 - 2^-20) - ei, rounded down once
-          const float xm = __fmaf_rd(aq, 0.99999904632568359375f /* 1 - 2^-20 */, -ei);
+          // a lower bound of the smaller magnitude of ends(): |wf| inv (1 - 2^-19)
+          // (below |q| (1 - 2^-20), q = wf inv rounded) less ei, rounded down
+          const float xm = __fmaf_rd(fabsf(wf[j]), inv_lo, -ei);
           bool same;
-          packed |= (e2m1_sr_interval(xm, q, rnd[j], lim, same) & 0xFu) << (4 * j);
+          packed |= e2m1_sr_interval(xm, wf[j], rnd[j], lim, same) << (4 * j);
           if (!same) redo |= 1u << j;
         }
       } else {  // two elements at a time, both ends

@@ -215,6 +215,32 @@ def test_e4m3_codes_over_their_whole_range(md, rnd):
 
 
 # -----------------------------------------------------------------------------
+# Weights far above 2^125 (up to near BF16's largest value): the certified
+# path's third divisor max(|w|, tau) leaves the approximate division's range,
+# where w + w u_m must still round to w as in the canonical sequence
+# -----------------------------------------------------------------------------
+@pytest.mark.parametrize("md", ["f32", "bf16"])
+@pytest.mark.parametrize("rnd", ["nearest", "stochastic"])
+def test_huge_weights(md, rnd):
+    import torch
+    p = P()
+    wl = W.replace(W.SMALL["llama_7b"], moment_dtype=md, rounding=rnd, name="huge_weights")
+    mt = W.materialize(wl, "cpu", warm_state=True)
+    big = max(range(len(mt.w)), key=lambda k: mt.w[k].numel())
+    w = mt.w[big]
+    vals = torch.tensor([2.0 ** 125, -2.0 ** 126, 3.0e38, -3.3e38, 5.0e37, 2.0 ** 127], dtype=torch.float32)
+    idx = torch.arange(0, w.numel(), 7)
+    w[idx] = vals[torch.arange(idx.numel()) % vals.numel()].to(torch.bfloat16)
+    r = p.Run(wl, mt=mt, hp=dict(lr_mul=4.0))
+    try:
+        for t in range(1, 4):
+            r.step(t)
+            p.assert_exact(r.compare(t + 1), f"huge weights {md}/{rnd} step {t}")
+    finally:
+        r.close()
+
+
+# -----------------------------------------------------------------------------
 # Launch shape and list structure do not change any bit
 # -----------------------------------------------------------------------------
 def test_grid_size_does_not_change_results():
