@@ -517,7 +517,8 @@ def summarize(wl, res, n_gpus, peak, peak_kind):
                       "frac_of_host_link_bound": round(res["link_ms"] / res["e2e_ms"], 4),
                       "frac_of_host_link_bound_median": round(res["link_ms"] / med, 4),
                       "host_buffers": res.get("host_buffers"), "host_probe_gbs": res.get("host_probe_gbs"),
-                      "host_buffers_tried": res.get("host_buffers_tried")}
+                      "host_buffers_tried": res.get("host_buffers_tried"),
+                      "step_ms": [round(x, 3) for x in res["e2e_step_ms"]]}
     return out
 
 
@@ -564,7 +565,7 @@ def result_line(wl, world, steps, warmup, l2_desc, main_sum, cpu, clocks, toy, d
         "roofline": {k: roof[k] for k in ("bound", "achieved", "peak", "unit", "frac", "traffic", "peak_source",
                                           "nominal_peak", "frac_of_nominal", "bytes_per_param", "launch_ms_avg")},
         "cpu_baseline": cpu,
-        "e2e": main_sum.get("e2e"),
+        "e2e": {k: v for k, v in main_sum["e2e"].items() if k != "step_ms"} if main_sum.get("e2e") else None,
         "gpu_launches": launches,
         "grid": main_sum["grid"],
         "clocks": clocks,
