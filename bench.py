@@ -232,16 +232,11 @@ def run_gpu(wl, steps: int, warmup: int, rank: int, e2e_steps: int, flush_l2: bo
     import torch
     import workloads as W
     from paper_2607_10611_gb300 import build
-    from paper_2607_10611_gb300.optimizer import MPAdam
 
     build()
     dev = torch.device("cuda", torch.cuda.current_device())
     mt = W.materialize(wl, dev, layout="flat")
-    extended = wl.weight_dtype not in ("bf16", "e4m3") or wl.compute_copy
-    opt = MPAdam(mt.w, mt.m, mt.v, mt.ve, weight_dtype=mt.formats if extended else wl.weight_dtype,
-                 grad_dtype=wl.grad_dtype, moment_dtype=wl.moment_dtype, rounding=wl.rounding,
-                 seed=wl.seed + rank, fp8_exp=mt.fp8_exp, block_scales=mt.bscale if extended else None,
-                 compute=mt.cc if extended else None, global_scales=mt.gscale if extended else None)
+    opt = make_optimizer(wl, mt, rank)
     if TAIL_POOL:
         opt.set_tail_pool(*TAIL_POOL)
     launches_per_step = len(set(mt.formats))
@@ -281,9 +276,10 @@ def run_gpu(wl, steps: int, warmup: int, rank: int, e2e_steps: int, flush_l2: bo
     total_ms = region0.elapsed_time(region1)
     launch_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
     copy_ms = same_size_copy_ms(algorithmic_bytes(wl), flush, flush_rd, stream) if flush is not None else None
+    one_tile = one_tile_step_ms(wl, rank, flush, flush_rd, stream) if flush is not None else None
     res = {"total_ms": total_ms, "launch_ms": launch_ms, "wall": (wall0, wall1),
            "grid": opt.launch_info(), "launches_per_step": launches_per_step, "l2_flushed": flush is not None,
-           "copy_ms": copy_ms}
+           "copy_ms": copy_ms, "one_tile_ms": one_tile}
     del flush, flush_rd
 
     # end to end through the host-buffer entry point (one weight format: flat host buffers)
@@ -347,6 +343,47 @@ def run_gpu(wl, steps: int, warmup: int, rank: int, e2e_steps: int, flush_l2: bo
     torch.cuda.synchronize()
     torch.cuda.empty_cache()
     return res
+
+
+def make_optimizer(wl, mt, rank: int):
+    """The optimizer over a materialized list, as a user builds it."""
+    from paper_2607_10611_gb300.optimizer import MPAdam
+    extended = wl.weight_dtype not in ("bf16", "e4m3") or wl.compute_copy
+    return MPAdam(mt.w, mt.m, mt.v, mt.ve, weight_dtype=mt.formats if extended else wl.weight_dtype,
+                  grad_dtype=wl.grad_dtype, moment_dtype=wl.moment_dtype, rounding=wl.rounding,
+                  seed=wl.seed + rank, fp8_exp=mt.fp8_exp, block_scales=mt.bscale if extended else None,
+                  compute=mt.cc if extended else None, global_scales=mt.gscale if extended else None)
+
+
+def one_tile_step_ms(wl, rank: int, flush, flush_rd, stream, reps: int = 20):
+    """Median event-timed step over a one-tile list (3840 elements) of the
+    first tensor's format, under the same flush: the launch, the kernel's
+    start-up and one tile, which no list of this format can go below.
+    None for lists that mix formats (two launches per step)."""
+    import dataclasses
+    import torch
+    import workloads as W
+    if len(set(wl.formats)) != 1:
+        return None
+    one = dataclasses.replace(wl, specs=(W.TensorSpec("one_tile", 3840, wl.specs[0].role),),
+                              format_list=tuple(wl.formats[:1]) if wl.format_list else (),
+                              name=wl.name + "_one_tile")
+    mt = W.materialize(one, stream.device, layout="flat")
+    opt = make_optimizer(one, mt, rank)
+    gptrs = [g.data_ptr() for g in mt.g]
+    ts = []
+    for i in range(reps + 3):
+        flush.fill_(float(i))
+        flush_rd.amax()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        opt.step_ptrs(gptrs, i + 1, stream.cuda_stream)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        if i >= 3:
+            ts.append(e0.elapsed_time(e1))
+    del opt, mt
+    return sorted(ts)[len(ts) // 2]
 
 
 def same_size_copy_ms(nbytes: float, flush, flush_rd, stream, reps: int = 20) -> float:
@@ -505,6 +542,9 @@ def summarize(wl, res, n_gpus, peak, peak_kind):
         # context for lists that fit in L2: a plain copy of the same bytes, same flush
         out["roofline"]["copy_same_bytes_ms"] = round(res["copy_ms"], 4)
         out["roofline"]["frac_of_copy_same_bytes"] = round(res["copy_ms"] / avg_launch, 4)
+    if res.get("one_tile_ms"):
+        # the same kernel over one tile, same flush: the floor of a step of this format
+        out["roofline"]["one_tile_step_ms"] = round(res["one_tile_ms"], 4)
     if "e2e_ms" in res:
         per = sorted(res["e2e_step_ms"])
         med = per[len(per) // 2] if len(per) % 2 else 0.5 * (per[len(per) // 2 - 1] + per[len(per) // 2])
@@ -531,6 +571,8 @@ def compact(sec) -> dict:
          "gbs": round(sec["roofline"]["achieved"], 0), "frac": sec["roofline"]["frac"]}
     if "frac_of_copy_same_bytes" in sec["roofline"]:
         c["frac_of_copy"] = sec["roofline"]["frac_of_copy_same_bytes"]
+    if "one_tile_step_ms" in sec["roofline"]:
+        c["one_tile_ms"] = sec["roofline"]["one_tile_step_ms"]
     clk = sec.get("clocks") or {}
     c["sm_mhz"] = clk.get("sm_mhz")
     if clk.get("reasons"):

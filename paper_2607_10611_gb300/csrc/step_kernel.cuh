@@ -1510,15 +1510,6 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
   const int tid = threadIdx.x;
   const int warp = tid >> 5, lane = tid & 31;
   const int S = a.stages;
-  if (tid == 0) {
-    for (int s = 0; s < S; ++s) {
-      mbar_init(smem_addr(&full_bar[s]), 1);
-      mbar_init(smem_addr(&empty_bar[s]), kConsumerWarps);
-    }
-    mbar_init_fence();
-  }
-  __syncthreads();
-
   const int64_t T = a.total_tiles;
   const int64_t tb = a.tile_base + static_cast<int64_t>(blockIdx.x) * T / gridDim.x;
   const int64_t te = a.tile_base + (static_cast<int64_t>(blockIdx.x) + 1) * T / gridDim.x;
@@ -1528,26 +1519,72 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
   const uint32_t smem0 = smem_addr(smem);
 
   // ------------------------------------------------------------ producer --
+  // One thread (lane 0 of the last warp) fills the ring.  Its state:
+  uint64_t pol = 0;  // L2 policy of the bulk copies
+  int pk = -1;       // tensor of tile t
+  TensorDesc d{};
+  const void* gp = nullptr;
+  const uint8_t* sp = nullptr;
+  int64_t tiles = 0;
+  int64_t t = tb, t_end = ts;  // the current run of consecutive tiles
+  int ps = 0;                  // next stage to fill, and how many times the ring has wrapped
+  uint32_t puse = 0;
+  int64_t issued = 0;
+  auto load = [&](int kk) {
+    pk = kk;
+    d = desc_of(a, pk);
+    gp = grad_of(a, pk);
+    if (WD == kE4M3B || WD == kNVFP4) sp = static_cast<const uint8_t*>(aux_of(a, pk).scale);
+    tiles = (d.numel + kTile - 1) / kTile;
+  };
+  auto issue = [&]() {  // the copies of tile t (of tensor pk) into stage ps, which is free
+    const int64_t e0 = (t - d.tile_off) * kTile;
+    const int count = static_cast<int>(d.numel - e0 < kTile ? d.numel - e0 : kTile);
+    // NVFP4 weights: half a byte per element (tile starts stay 16-byte aligned: 1920 bytes per tile)
+    const uint32_t nw = WD == kNVFP4 ? staged_bytes(d.w, (count + 1) / 2, 1) : staged_bytes(d.w, count, WS);
+    const uint32_t ng = staged_bytes(gp, count, GS);
+    const uint32_t nm = staged_bytes(d.m, count, MS), nv = staged_bytes(d.v, count, MS);
+    const uint32_t nve = staged_bytes(d.ve, count, MS);
+    const int64_t s0 = WD == kE4M3B ? 2 * (e0 / kBlock) : e0 / kFp4Block;  // the tile's first scale byte
+    const uint32_t ns = WD == kE4M3B   ? staged_bytes(sp + s0, 2 * ((count + kBlock - 1) / kBlock), 1)
+                        : WD == kNVFP4 ? staged_bytes(sp + s0, (count + kFp4Block - 1) / kFp4Block, 1)
+                                       : 0u;
+    const uint32_t bar = smem_addr(&full_bar[ps]);
+    const uint32_t st = smem0 + static_cast<uint32_t>(ps * a.stage_bytes);
+    stage_tile[ps] = t;  // published by the arrive below (release)
+    stage_k[ps] = pk;
+    mbar_arrive_expect_tx(bar, nw + ng + nm + nv + nve + ns);
+    if (nw) tma_load(st, static_cast<const uint8_t*>(d.w) + (WD == kNVFP4 ? e0 / 2 : e0 * WS), nw, bar, pol);
+    if (ng) tma_load(st + a.off_g, static_cast<const uint8_t*>(gp) + e0 * GS, ng, bar, pol);
+    if (nm) tma_load(st + a.off_m, static_cast<const uint8_t*>(d.m) + e0 * MS, nm, bar, pol);
+    if (nv) tma_load(st + a.off_v, static_cast<const uint8_t*>(d.v) + e0 * MS, nv, bar, pol);
+    if (nve) tma_load(st + a.off_ve, static_cast<const uint8_t*>(d.ve) + e0 * MS, nve, bar, pol);
+    if (ns) tma_load(st + a.off_s, sp + s0, ns, bar, pol);
+    ++issued;
+    ++t;
+    if (++ps == S) { ps = 0; ++puse; }
+  };
+  if (tid == kConsumers) {
+    // The producer sets up the ring and issues the copies of its first tile
+    // before the block-wide barrier, in straight-line code next to the
+    // kernel's entry: on a launch of a tile or two per CTA these copies are
+    // on the critical path, and the full loop below starts some 1.5 us later.
+    for (int i = 0; i < S; ++i) {
+      mbar_init(smem_addr(&full_bar[i]), 1);
+      mbar_init(smem_addr(&empty_bar[i]), kConsumerWarps);
+    }
+    mbar_init_fence();
+    pol = evict_first_policy();
+    if (t < t_end) {
+      load(first_tensor(a, tb));
+      while (t >= d.tile_off + tiles) load(pk + 1);
+      issue();
+    }
+  }
+  __syncthreads();
+
   if (warp == kConsumerWarps) {
     if (lane != 0) return;
-    const uint64_t pol = evict_first_policy();
-    int k = -1;
-    TensorDesc d{};
-    const void* gp = nullptr;
-    const uint8_t* sp = nullptr;
-    int64_t tiles = 0;
-    auto load = [&](int kk) {
-      k = kk;
-      d = desc_of(a, k);
-      gp = grad_of(a, k);
-      if (WD == kE4M3B || WD == kNVFP4) sp = static_cast<const uint8_t*>(aux_of(a, k).scale);
-      tiles = (d.numel + kTile - 1) / kTile;
-    };
-    int64_t t = tb, t_end = ts;  // the current run of consecutive tiles
-    if (t < t_end) load(first_tensor(a, tb));
-    int s = 0;
-    uint32_t use = 0;
-    int64_t issued = 0;
     bool failed = false;
     for (;;) {
       if (t >= t_end) {  // static part done: next chunk of the tail pool, if any
@@ -1557,39 +1594,15 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
         const PoolChunk pc = a.pool[j];
         t = pc.start;
         t_end = pc.start + pc.count;
-        if (pc.first != k) load(pc.first);
+        if (pc.first != pk) load(pc.first);
       }
-      while (t >= d.tile_off + tiles) load(k + 1);
-      if (use > 0 && !mbar_wait(smem_addr(&empty_bar[s]), (use - 1) & 1u)) {
+      while (t >= d.tile_off + tiles) load(pk + 1);
+      if (puse > 0 && !mbar_wait(smem_addr(&empty_bar[ps]), (puse - 1) & 1u)) {
         if (a.err) atomicOr(a.err, kErrEmptyWait);
         failed = true;
         break;
       }
-      const int64_t e0 = (t - d.tile_off) * kTile;
-      const int count = static_cast<int>(d.numel - e0 < kTile ? d.numel - e0 : kTile);
-      // NVFP4 weights: half a byte per element (tile starts stay 16-byte aligned: 1920 bytes per tile)
-      const uint32_t nw = WD == kNVFP4 ? staged_bytes(d.w, (count + 1) / 2, 1) : staged_bytes(d.w, count, WS);
-      const uint32_t ng = staged_bytes(gp, count, GS);
-      const uint32_t nm = staged_bytes(d.m, count, MS), nv = staged_bytes(d.v, count, MS);
-      const uint32_t nve = staged_bytes(d.ve, count, MS);
-      const int64_t s0 = WD == kE4M3B ? 2 * (e0 / kBlock) : e0 / kFp4Block;  // the tile's first scale byte
-      const uint32_t ns = WD == kE4M3B   ? staged_bytes(sp + s0, 2 * ((count + kBlock - 1) / kBlock), 1)
-                          : WD == kNVFP4 ? staged_bytes(sp + s0, (count + kFp4Block - 1) / kFp4Block, 1)
-                                         : 0u;
-      const uint32_t bar = smem_addr(&full_bar[s]);
-      const uint32_t st = smem0 + static_cast<uint32_t>(s * a.stage_bytes);
-      stage_tile[s] = t;  // published by the arrive below (release)
-      stage_k[s] = k;
-      mbar_arrive_expect_tx(bar, nw + ng + nm + nv + nve + ns);
-      if (nw) tma_load(st, static_cast<const uint8_t*>(d.w) + (WD == kNVFP4 ? e0 / 2 : e0 * WS), nw, bar, pol);
-      if (ng) tma_load(st + a.off_g, static_cast<const uint8_t*>(gp) + e0 * GS, ng, bar, pol);
-      if (nm) tma_load(st + a.off_m, static_cast<const uint8_t*>(d.m) + e0 * MS, nm, bar, pol);
-      if (nv) tma_load(st + a.off_v, static_cast<const uint8_t*>(d.v) + e0 * MS, nv, bar, pol);
-      if (nve) tma_load(st + a.off_ve, static_cast<const uint8_t*>(d.ve) + e0 * MS, nve, bar, pol);
-      if (ns) tma_load(st + a.off_s, sp + s0, ns, bar, pol);
-      ++issued;
-      ++t;
-      if (++s == S) { s = 0; ++use; }
+      issue();
     }
     if (failed) {  // wait (bounded) for this CTA's copies still in flight, then leave
       const int64_t last = issued < S ? issued : S;
@@ -1601,12 +1614,12 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
       return;
     }
     // no more work: once the next stage is free, post the end marker there
-    if (use > 0 && !mbar_wait(smem_addr(&empty_bar[s]), (use - 1) & 1u)) {
+    if (puse > 0 && !mbar_wait(smem_addr(&empty_bar[ps]), (puse - 1) & 1u)) {
       if (a.err) atomicOr(a.err, kErrEmptyWait);
       return;
     }
-    stage_tile[s] = -1;
-    mbar_arrive(smem_addr(&full_bar[s]));
+    stage_tile[ps] = -1;
+    mbar_arrive(smem_addr(&full_bar[ps]));
     return;
   }
 
@@ -1666,7 +1679,11 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
       a.fp8_amax[static_cast<int64_t>(a.a_zero_slot) * n + x.d.ring] = 0u;
     }
     const int count = static_cast<int>(x.d.numel - tile_e0 < kTile ? x.d.numel - tile_e0 : kTile);
-    if (count == kTile && x.fast) {  // whole tile, every array staged: straight-line group
+    // Straight-line group: every array aligned, and this warp's 256 elements
+    // all inside the tile (every warp of a whole tile; the whole warps of a
+    // tensor's last tile, whose bytes the producer staged as well).  A warp
+    // that holds the end of a partial tile takes the element-wise path below.
+    if (x.fast && kGroup * 32 * (warp + 1) <= count) {
       const uint32_t st = smem0 + static_cast<uint32_t>(s * a.stage_bytes);
       const int64_t e0 = tile_e0 + kGroup * c;
       float w[8], g[8], m[8], v[8], ve[8];

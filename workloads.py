@@ -236,7 +236,7 @@ CONFIGS: Dict[str, Workload] = {
 }
 
 # Same distributions and formats at sizes the oracle finishes in seconds,
-# still spanning many 2048-element CTA tiles and ragged tails.
+# still spanning many 3840-element tiles and ragged tails.
 SMALL: Dict[str, Workload] = {
     "flat_1m": replace(_flat1m(), specs=(TensorSpec("flat", (1 << 16) + 5, "flat"),), name="flat_small"),
     "gpt2_124m": _gpt2(layers=2, d=64, vocab=1003, ctx=64, name="gpt2_small"),
