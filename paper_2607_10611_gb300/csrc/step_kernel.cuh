@@ -863,12 +863,11 @@ __device__ __forceinline__ void finish_group(const StepArgs& a, const TensorCtx&
 
 // One group of a partial tile, or of a tensor whose arrays are not all staged
 // or aligned: loads each array from the stage when its bytes were staged, else
-// from global memory; kept out of line so the whole-tile path stays lean.  The
-// running E4M3 maximum goes in and comes back by value: a reference would pin
-// the caller's copy to local memory for the whole loop.
+// from global memory.  The running E4M3 maximum goes in and comes back by
+// value: a reference would pin the caller's copy to local memory.
 template <int WD, int GD, int MD, bool SR, bool OPT>
-__device__ __noinline__ uint32_t general_group(const StepArgs& a, const TensorCtx& x, int64_t tile_e0, int count,
-                                               int c, uint32_t st, uint32_t amax_bits) {
+__device__ __forceinline__ uint32_t general_group(const StepArgs& a, const TensorCtx& x, int64_t tile_e0,
+                                                  int count, int c, uint32_t st, uint32_t amax_bits) {
   constexpr int WS = esize_of(WD), GS = esize_of(GD), MS = esize_of(MD);
   if (kGroup * c >= count) return amax_bits;
   const int valid = count - kGroup * c < kGroup ? count - kGroup * c : kGroup;
@@ -897,6 +896,20 @@ __device__ __noinline__ uint32_t general_group(const StepArgs& a, const TensorCt
   }
   finish_group<WD, GD, MD, SR, OPT, false>(a, x, e0, valid, w, g, m, v, ve, amax_bits, st, c);
   return amax_bits;
+}
+
+// The same, as a call.  Which form a kernel instance uses was measured per
+// moment format.  Called, the group costs the caller a stack frame (the live
+// state saved around the call), and on a short launch after an L2 flush those
+// first local-memory accesses wait on DRAM: a 1 Mi-element list with
+// binary32 moments ran 15.9-17.1 us called against 13.0-13.1 us inline, and
+// GPT-2, the ragged list and the 1.5B list ran 0.7-1.1 % faster inline.  With
+// BF16 moments the inline form slowed the whole-tile loop instead: the 7B list
+// took 18.44 ms per step against 18.21 ms called (three runs each).
+template <int WD, int GD, int MD, bool SR, bool OPT>
+__device__ __noinline__ uint32_t general_group_call(const StepArgs& a, const TensorCtx& x, int64_t tile_e0,
+                                                    int count, int c, uint32_t st, uint32_t amax_bits) {
+  return general_group<WD, GD, MD, SR, OPT>(a, x, tile_e0, count, c, st, amax_bits);
 }
 
 // ---------------------------------------------------------------------------
@@ -1016,7 +1029,7 @@ __device__ __forceinline__ void finish_block(const StepArgs& a, const TensorCtx&
 // elements), loading each array from the stage when its bytes were staged,
 // else from global memory.
 template <int GD, int MD, bool SR, bool OPT>
-__device__ __noinline__ void general_block_group(const StepArgs& a, const TensorCtx& x, int64_t tile_e0, int count,
+__device__ __forceinline__ void general_block_group(const StepArgs& a, const TensorCtx& x, int64_t tile_e0, int count,
                                                  int c, uint32_t st) {
   constexpr int GS = esize_of(GD), MS = esize_of(MD);
   const int rem = count - kGroup * c;
@@ -1050,6 +1063,16 @@ __device__ __noinline__ void general_block_group(const StepArgs& a, const Tensor
   }
   finish_block<GD, MD, SR, OPT>(a, x, e0, valid, h, w, g, m, v, ve);
 }
+
+// The same, as a call: with BF16 moments, as for general_group_call.  Inline,
+// the FP8-regime list (block-scaled linears, binary32 moments) ran 6.02 ms per
+// step against 6.08 ms called.
+template <int GD, int MD, bool SR, bool OPT>
+__device__ __noinline__ void general_block_group_call(const StepArgs& a, const TensorCtx& x, int64_t tile_e0, int count,
+                                             int c, uint32_t st) {
+  general_block_group<GD, MD, SR, OPT>(a, x, tile_e0, count, c, st);
+}
+
 
 // ---------------------------------------------------------------------------
 // NVFP4 weights: E2M1 codes (OCP FP4: sign, 2 exponent bits with bias 1, one
@@ -1736,14 +1759,23 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
       if (++s == S) { s = 0; ++use; }
       continue;
     }
-    // partial tile or unstaged arrays: element-wise fallback, out of line
-    if constexpr (WD == kE4M3B)
-      general_block_group<GD, MD, SR, OPT>(a, x, tile_e0, count, c, smem0 + static_cast<uint32_t>(s * a.stage_bytes));
-    else if constexpr (WD == kNVFP4)
+    // partial tile or unstaged arrays: element-wise fallback (inline or a
+    // call, by moment format; the NVFP4 one is always a call: inline it slowed
+    // the stochastic-rounding loop by 5 %)
+    if constexpr (WD == kE4M3B) {
+      if constexpr (MD == kF32)
+        general_block_group<GD, MD, SR, OPT>(a, x, tile_e0, count, c, smem0 + static_cast<uint32_t>(s * a.stage_bytes));
+      else
+        general_block_group_call<GD, MD, SR, OPT>(a, x, tile_e0, count, c,
+                                                  smem0 + static_cast<uint32_t>(s * a.stage_bytes));
+    } else if constexpr (WD == kNVFP4)
       general_fp4_group<GD, MD, SR, OPT>(a, x, tile_e0, count, c, smem0 + static_cast<uint32_t>(s * a.stage_bytes));
     else
-      amax_bits = general_group<WD, GD, MD, SR, OPT>(a, x, tile_e0, count, c,
-                                                     smem0 + static_cast<uint32_t>(s * a.stage_bytes), amax_bits);
+      amax_bits = MD == kF32 ? general_group<WD, GD, MD, SR, OPT>(a, x, tile_e0, count, c,
+                                                                   smem0 + static_cast<uint32_t>(s * a.stage_bytes),
+                                                                   amax_bits)
+                             : general_group_call<WD, GD, MD, SR, OPT>(
+                                   a, x, tile_e0, count, c, smem0 + static_cast<uint32_t>(s * a.stage_bytes), amax_bits);
     __syncwarp();
     if (lane == 0) mbar_arrive(smem_addr(&empty_bar[s]));
     if (++s == S) { s = 0; ++use; }
