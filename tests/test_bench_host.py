@@ -120,7 +120,8 @@ def _fake_res(wl, ms, e2e=False):
     """What run_gpu returns, with plausible timings (full-precision floats)."""
     res = {"total_ms": ms * 20 * 1.0000123, "launch_ms": [ms * (1 + 1e-3 * i / 7) for i in range(20)],
            "wall": (0.0, 1.0), "grid": (152, 512), "launches_per_step": 1 + (wl.weight_dtype != "bf16"),
-           "l2_flushed": wl.name == "flat_1m", "copy_ms": 0.0081234567 if wl.name == "flat_1m" else None}
+           "l2_flushed": wl.name == "flat_1m", "copy_ms": 0.0081234567 if wl.name == "flat_1m" else None,
+           "one_tile_ms": 0.0082345678 if wl.name == "flat_1m" else None}
     if e2e:
         res.update(e2e_ms=101.234567, e2e_step_ms=[100.0 + 1.2345678 * i for i in range(20)],
                    h2d=13476831232, d2h=13476831232, link_ms=94.12345678, host_buffers="huge_pages",
@@ -160,3 +161,7 @@ def test_result_line_keeps_every_secondary_list_in_the_driver_tail():
         assert key in line
     assert line["e2e"]["steps"] == 20 and line["e2e"]["ms_worst"] >= line["e2e"]["ms_median"]
     assert line["roofline"]["frac_of_nominal"] < line["roofline"]["frac"]
+    # the e2e per-step times go to the details file only
+    assert "step_ms" not in line["e2e"] and len(main["e2e"]["step_ms"]) == 20
+    flat = [bench.compact(s2) for s2 in secs if s2["workload"] == "flat_1m"][0]
+    assert flat["one_tile_ms"] == 0.0082 and flat["frac_of_copy"] > 0
