@@ -4,8 +4,8 @@ gradient pointers in the kernel parameters, and each CTA finds its first
 tensor by scanning them instead of reading the host-computed table.  Every
 stored bit must still match the oracle: each weight format, one to five
 tensors (five uses the tables), empty tensors at either end and in the
-middle, tensors shorter than a tile, grids with more CTAs than tiles, and the
-tail pool on and off."""
+middle, tensors shorter than a tile, last tiles of whole warps only, grids
+with more CTAs than tiles, and the tail pool on and off."""
 import pytest
 
 import workloads as W
@@ -17,6 +17,9 @@ LISTS = {
     "two_empty_ends": (0, 9000, 5),
     "four": (3, 0, 20000, 7700),
     "five_tables": (3841, 1, 0, 12000, 64),
+    # last tiles made of whole warps only (256 elements each): they take the
+    # whole-tile path with no element-wise warp
+    "warp_tails": (4096, 8448, 512),
 }
 
 
