@@ -607,7 +607,7 @@ struct TensorCtx {
   const void* g;
   int64_t tiles;
   bool vec;            // all pointers aligned for vector access by whole groups
-  bool fast;           // whole tiles are fully staged and stored with vector stores
+  bool fast;           // every array 16-byte aligned: whole warps of a tile are staged, stored with vector stores
   float dec_scale, enc_scale;
   float cc_scale;      // E4M3 per-tensor: 2^e of the new encode (compute copy)
   void* scale;         // kE4M3B (FP16) / kNVFP4 (E4M3) block scales
