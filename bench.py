@@ -222,6 +222,19 @@ def time_oracle(wl, target_s: float, t_step: int = 1):
         n = int(min(rate * target_s, 1 << 29))
 
 
+def oracle_whole_lists(spec: str) -> dict:
+    """The oracle's single-core rate on whole lists (one step each, step 1):
+    ns per parameter and parameters per second."""
+    import workloads as W
+    out = {}
+    for name in filter(None, spec.split(",")):
+        wl = W.CONFIGS[name]
+        got, dt, rate = time_oracle(wl, target_s=1e9)  # grows to the whole list
+        out[name] = {"params": got, "whole_list": got == wl.n_params, "seconds": round(dt, 3),
+                     "ns_per_param": round(1e9 / rate, 2), "gparams_per_s": rate / 1e9, "cores": 1}
+    return out
+
+
 # ---------------------------------------------------------------------------
 # GPU arm
 # ---------------------------------------------------------------------------
@@ -592,7 +605,7 @@ def workload_config(wl, world: int, l2: str) -> dict:
 
 
 def result_line(wl, world, steps, warmup, l2_desc, main_sum, cpu, clocks, toy, details, secondary,
-                launches) -> dict:
+                launches, cpu_lists=None) -> dict:
     """The one JSON line rank 0 prints.  The driver keeps only the line's
     tail, so it stays short: the full per-workload record (every roofline
     field, the diagnostic's per-regime table) is in the details file, and
@@ -607,6 +620,7 @@ def result_line(wl, world, steps, warmup, l2_desc, main_sum, cpu, clocks, toy, d
         "roofline": {k: roof[k] for k in ("bound", "achieved", "peak", "unit", "frac", "traffic", "peak_source",
                                           "nominal_peak", "frac_of_nominal", "bytes_per_param", "launch_ms_avg")},
         "cpu_baseline": cpu,
+        "cpu_ns_per_param": {k: v["ns_per_param"] for k, v in (cpu_lists or {}).items()},
         "e2e": {k: v for k, v in main_sum["e2e"].items() if k != "step_ms"} if main_sum.get("e2e") else None,
         "gpu_launches": launches,
         "grid": main_sum["grid"],
@@ -641,6 +655,8 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--e2e-steps", type=int, default=20)
     ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    ap.add_argument("--cpu-lists", default="flat_1m,gpt2_124m",
+                    help="lists the oracle also steps whole, once each, for its single-core rate ('' skips)")
     ap.add_argument("--toy-steps", type=int, default=2048, help="matrix-fitting diagnostic steps per run (0 skips)")
     ap.add_argument("--rounding", default=None, choices=["nearest", "stochastic"],
                     help="override the workload's weight rounding")
@@ -736,12 +752,13 @@ def main():
     got, dt, rate = time_oracle(wl, target_s=args.cpu_seconds)
     cpu = {"value": rate / 1e9, "unit": UNIT, "cores": 1, "nproc": os.cpu_count(), "kind": "oracle",
            "sample": f"one step over the first {got} elements of the {wl.name} list ({dt:.1f} s, single thread)"}
+    cpu_lists = oracle_whole_lists(args.cpu_lists)
 
     details = out_dir / "bench_details.json"
     details.write_text(json.dumps({"main": main_sum, "secondary": secondary, "toy": toy, "clocks": clocks,
-                                   "cpu_baseline": cpu}, indent=1))
+                                   "cpu_baseline": cpu, "cpu_lists": cpu_lists}, indent=1))
     line = result_line(wl, world, args.steps, warmup, l2_desc, main_sum, cpu, clocks, toy, details, secondary,
-                       args.steps * res["launches_per_step"])
+                       args.steps * res["launches_per_step"], cpu_lists)
     print(json.dumps(line), flush=True)
     if world > 1:
         torch.distributed.destroy_process_group()

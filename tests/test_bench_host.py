@@ -148,8 +148,12 @@ def test_result_line_keeps_every_secondary_list_in_the_driver_tail():
     cpu = {"value": 0.018728084501097277, "unit": "Gparams/s", "cores": 1, "nproc": 72, "kind": "oracle",
            "sample": "one step over the first 181498738 elements of the llama_7b list (9.7 s, single thread)"}
     clocks = {"sm_mhz": 2070.0, "sm_max_mhz": 2070.0, "reasons": [], "samples": 5}
+    cpu_lists = {"flat_1m": {"params": 1048576, "whole_list": True, "seconds": 0.063, "ns_per_param": 60.12,
+                             "gparams_per_s": 0.016634534016404936, "cores": 1},
+                 "gpt2_124m": {"params": 124439808, "whole_list": True, "seconds": 7.291, "ns_per_param": 58.59,
+                               "gparams_per_s": 0.017066754888876722, "cores": 1}}
     line = bench.result_line(wl, 1, 20, 5, "inputs larger than L2 (no flush needed)", main, cpu, clocks,
-                             {"us_per_step": 15.51234}, "/tmp/bench_details.json", secs, 20)
+                             {"us_per_step": 15.51234}, "/tmp/bench_details.json", secs, 20, cpu_lists)
     text = json.dumps(line)
     assert len(text) < 3000, len(text)
     tail = text[-1400:]
@@ -159,6 +163,7 @@ def test_result_line_keeps_every_secondary_list_in_the_driver_tail():
     assert '"workload": "llama_1p5b_nvfp4:stochastic"' in tail and '"workload": "llama_1p5b"' in tail
     for key in ("metric", "value", "unit", "ms_per_step", "roofline", "cpu_baseline", "e2e", "clocks"):
         assert key in line
+    assert line["cpu_ns_per_param"] == {"flat_1m": 60.12, "gpt2_124m": 58.59}
     assert line["e2e"]["steps"] == 20 and line["e2e"]["ms_worst"] >= line["e2e"]["ms_median"]
     assert line["roofline"]["frac_of_nominal"] < line["roofline"]["frac"]
     # the e2e per-step times go to the details file only
