@@ -510,7 +510,7 @@ def run_toy(steps: int):
             d.close()
             del w
     return {"n": W.TOY_N, "batch": 65536, "steps_per_run": steps, "runs": 15,
-            "us_per_step": 1e3 * total_ms / (15 * steps), "launches_per_step": 3, "regimes": out}
+            "us_per_step": 1e3 * total_ms / (15 * steps), "launches_per_step": 2, "regimes": out}
 
 
 def max_over_ranks(ms: float, device: str) -> float:

@@ -1372,8 +1372,6 @@ extern "C" int32_t mpadam_toy_create(int64_t n, const mpadam_toy_config* cfg, mp
   const size_t B = (size_t)cfg->batch;
   if (dev_malloc(&a.cnt, sizeof(int32_t) * n) != cudaSuccess || dev_malloc(&a.first, sizeof(int32_t) * n) != cudaSuccess ||
       dev_malloc(&a.idx, sizeof(int32_t) * B) != cudaSuccess || dev_malloc(&a.res, sizeof(float) * B) != cudaSuccess ||
-      dev_malloc(&a.sq, sizeof(double) * B) != cudaSuccess || dev_malloc(&a.alpha, sizeof(float) * 2) != cudaSuccess ||
-      dev_malloc(&a.loss_h, sizeof(double) * 2) != cudaSuccess ||
       dev_malloc(&st->t_dev, sizeof(int64_t) * 2) != cudaSuccess ||
       dev_malloc(&a.partial, sizeof(double) * (B / 2048 + 2)) != cudaSuccess) {
     mpadam_toy_destroy(st);
@@ -1477,8 +1475,7 @@ extern "C" int32_t mpadam_toy_destroy(mpadam_toy_state* s) {
   if (s->cap) cudaStreamDestroy(s->cap);
   if (s->t_dev) cudaFree(s->t_dev);
   mpadam::ToyArgs& a = s->a;
-  for (void* p : {(void*)a.cnt, (void*)a.first, (void*)a.idx, (void*)a.res, (void*)a.sq, (void*)a.alpha, (void*)a.loss_h,
-                  (void*)a.partial})
+  for (void* p : {(void*)a.cnt, (void*)a.first, (void*)a.idx, (void*)a.res, (void*)a.partial})
     if (p) cudaFree(p);
   delete s;
   return MPADAM_OK;

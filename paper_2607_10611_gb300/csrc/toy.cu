@@ -3,13 +3,14 @@
 // with replacement, forms the minibatch loss c (mean squared residual)^2
 // (per half when the halves are separate problems), and applies the
 // additive, multiplicative or combined step (no moments) to every sampled
-// entry, rounding it to BF16.  Three launches per step:
-//   1. sample (Philox lanes), residuals, hit counts and each entry's first
-//      sample (atomics on two n-entry scratch arrays, zero between steps);
-//   2. partial sums of the squared residuals over aligned chunks of 2048
-//      samples (subtrees of the perfect binary tree of binary64 sums over
-//      adjacent samples);
-//   3. every CTA completes the tree from the partials (at most 32 per
+// entry, rounding it to BF16.  Two launches per step:
+//   1. one CTA per aligned chunk of 2048 samples draws them (Philox lanes;
+//      residuals, hit counts and each entry's first sample, with atomics on
+//      two n-entry scratch arrays that are zero between steps) and sums
+//      their squared residuals as a subtree of the perfect binary tree of
+//      binary64 sums over adjacent samples: each thread draws the adjacent
+//      pair that is the tree's first level;
+//   2. every CTA completes the tree from the partials (at most 32 per
 //      problem), forms M, the loss and alpha = 4 c M / B_h; the first sample
 //      of each entry applies the entry's update (its contribution alpha r
 //      added once per hit) and clears the scratch.
@@ -42,46 +43,48 @@ __global__ void toy_set_step_kernel(int64_t* t_dev, int64_t first) {
   t_dev[1] = first;
 }
 
-__global__ void toy_sample_kernel(const __grid_constant__ ToyArgs a) {
-  const int64_t s = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x;
-  if (s >= a.batch) return;
-  uint32_t t_lo, t_hi;
-  toy_step_number(a, t_lo, t_hi);
+// Sample s drawn with 32-bit lane `lane` of this step: its entry, residual,
+// hit count and first-sample mark.  Returns r^2, exact in binary64.
+__device__ __forceinline__ double toy_draw(const ToyArgs& a, int64_t s, uint32_t lane) {
   const int64_t Bh = a.batch / (a.split ? 2 : 1);
   const int64_t range = a.n / (a.split ? 2 : 1);
   const int64_t h = a.split ? s / Bh : 0;
-  // 32-bit random lane s of step t: word s mod 4 of Philox block s / 4
-  const uint64_t blk = static_cast<uint64_t>(s) >> 2;
-  const uint4 r4 = philox4x32_10(static_cast<uint32_t>(blk), static_cast<uint32_t>(blk >> 32), t_lo, t_hi, a.rk0,
-                                 a.rk1);
-  const uint32_t lanes[4] = {r4.x, r4.y, r4.z, r4.w};
-  const uint32_t lane = lanes[s & 3];
   const int64_t idx = h * range + static_cast<int64_t>(static_cast<uint64_t>(lane) & static_cast<uint64_t>(range - 1));
   const float wv = __uint_as_float(static_cast<uint32_t>(a.w[idx]) << 16);
   const float r = __fsub_rn(wv, a.wstar[idx]);
   a.idx[s] = static_cast<int32_t>(idx);
   a.res[s] = r;
-  a.sq[s] = static_cast<double>(r) * static_cast<double>(r);  // exact
   atomicAdd(&a.cnt[idx], 1);
   atomicMax(&a.first[idx], INT_MAX - static_cast<int32_t>(s));  // the smallest sample wins
+  return static_cast<double>(r) * static_cast<double>(r);
 }
 
-// Tree sum of the squared residuals, stage 1: CTA b of a problem sums the
-// aligned chunk of C = min(2048, B_h) samples [bC, bC + C) as a perfect
-// binary tree (adjacent pairs per thread, then adjacent lanes, then adjacent
-// warps) into partial[problem][b].
+// Stage 1: CTA b of a problem draws the aligned chunk of C = min(2048, B_h)
+// samples [bC, bC + C) and sums their squared residuals as a perfect binary
+// tree (adjacent pairs per thread, then adjacent lanes, then adjacent warps)
+// into partial[problem][b].
 constexpr int kToyChunk = 2048;
 
-__global__ void __launch_bounds__(kToyChunk / 2) toy_partial_kernel(const __grid_constant__ ToyArgs a) {
+__global__ void __launch_bounds__(kToyChunk / 2) toy_sample_partial_kernel(const __grid_constant__ ToyArgs a) {
   __shared__ double warp_sum[32];
   const int64_t Bh = a.batch / (a.split ? 2 : 1);
   const int64_t C = Bh < kToyChunk ? Bh : kToyChunk;
   const int64_t per = Bh / C;  // chunks per problem
   const int h = static_cast<int>(blockIdx.x / per), b = static_cast<int>(blockIdx.x % per);
-  const double* v = a.sq + h * Bh + b * C;
   const int pairs = static_cast<int>(C / 2);
   const int t = threadIdx.x;
-  double x = t < pairs ? v[2 * t] + v[2 * t + 1] : 0.0;
+  double x = 0.0;
+  if (t < pairs) {
+    uint32_t t_lo, t_hi;
+    toy_step_number(a, t_lo, t_hi);
+    // samples s and s + 1 (s even): lanes s mod 4 and s mod 4 + 1 of Philox block s / 4
+    const int64_t s = h * Bh + b * C + 2 * t;
+    const uint64_t blk = static_cast<uint64_t>(s) >> 2;
+    const uint4 r4 = philox4x32_10(static_cast<uint32_t>(blk), static_cast<uint32_t>(blk >> 32), t_lo, t_hi, a.rk0,
+                                   a.rk1);
+    const bool upper = (s & 2) != 0;
+    x = toy_draw(a, s, upper ? r4.z : r4.x) + toy_draw(a, s + 1, upper ? r4.w : r4.y);
+  }
   const int span = pairs < 32 ? pairs : 32;  // lanes holding pair sums
   for (int off = 1; off < span; off <<= 1) {
     const double y = __shfl_xor_sync(0xFFFFFFFFu, x, off);
@@ -174,14 +177,11 @@ __global__ void toy_update_kernel(const __grid_constant__ ToyArgs a) {
 cudaError_t launch_toy_step(const ToyArgs& a, cudaStream_t stream) {
   const int halves = a.split ? 2 : 1;
   const int64_t Bh = a.batch / halves;
-  const unsigned blocks = static_cast<unsigned>((a.batch + 255) / 256);
-  toy_sample_kernel<<<blocks, 256, 0, stream>>>(a);
+  const int64_t C = Bh < kToyChunk ? Bh : kToyChunk;
+  toy_sample_partial_kernel<<<static_cast<unsigned>(halves * (Bh / C)), kToyChunk / 2, 0, stream>>>(a);
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  const int64_t C = Bh < kToyChunk ? Bh : kToyChunk;
-  toy_partial_kernel<<<static_cast<unsigned>(halves * (Bh / C)), kToyChunk / 2, 0, stream>>>(a);
-  e = cudaGetLastError();
-  if (e != cudaSuccess) return e;
+  const unsigned blocks = static_cast<unsigned>((a.batch + 255) / 256);
   toy_update_kernel<<<blocks, 256, 0, stream>>>(a);
   return cudaGetLastError();
 }
