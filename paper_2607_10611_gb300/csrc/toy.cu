@@ -124,6 +124,21 @@ __device__ __forceinline__ void toy_finish_mean(const ToyArgs& a, int h, double&
 __global__ void toy_update_kernel(const __grid_constant__ ToyArgs a) {
   __shared__ double s_loss[2];
   __shared__ float s_alpha[2];
+  const int64_t s = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x;
+  // This sample's inputs, loaded while warps 0 and 1 form the mean: the
+  // entry's first-sample mark, hit count and weight are independent reads
+  // (a sample that is not its entry's first uses none of them; only the first
+  // writes the entry, after reading it).
+  int32_t idx = 0, first = 0, k = 0;
+  uint16_t wbits = 0;
+  float r = 0.0f;
+  if (s < a.batch) {
+    idx = a.idx[s];
+    first = a.first[idx];
+    k = a.cnt[idx];
+    wbits = a.w[idx];
+    r = a.res[s];
+  }
   if (threadIdx.x < 64) {  // warp 0: the first problem, warp 1: the second
     const int h = threadIdx.x >> 5;
     if (h < (a.split ? 2 : 1)) {
@@ -134,7 +149,6 @@ __global__ void toy_update_kernel(const __grid_constant__ ToyArgs a) {
     }
   }
   __syncthreads();
-  const int64_t s = blockIdx.x * static_cast<int64_t>(blockDim.x) + threadIdx.x;
   if (s == 0) {
     const double loss = a.split ? (0.0 + s_loss[0]) + s_loss[1] : 0.0 + s_loss[0];
     if (a.t_dev) {  // run mode: record the loss by step, then advance the step counter
@@ -146,15 +160,13 @@ __global__ void toy_update_kernel(const __grid_constant__ ToyArgs a) {
     }
   }
   if (s >= a.batch) return;
-  const int32_t idx = a.idx[s];
-  if (a.first[idx] != INT_MAX - static_cast<int32_t>(s)) return;  // the entry's first sample applies its update
+  if (first != INT_MAX - static_cast<int32_t>(s)) return;  // the entry's first sample applies its update
   const int64_t Bh = a.batch / (a.split ? 2 : 1);
   const int h = a.split ? static_cast<int>(s / Bh) : 0;
-  const int32_t k = a.cnt[idx];
-  const float x = __fmul_rn(s_alpha[h], a.res[s]);
+  const float x = __fmul_rn(s_alpha[h], r);
   float g = x;
   for (int32_t i = 1; i < k; ++i) g = __fadd_rn(g, x);
-  const float wf = __uint_as_float(static_cast<uint32_t>(a.w[idx]) << 16);
+  const float wf = __uint_as_float(static_cast<uint32_t>(wbits) << 16);
   const float ln2 = 0.693147180559945309417232121458f;
   const float ua = __fmul_rn(-a.lr_add, g);
   const float ge = __fmul_rn(__fmul_rn(ln2, wf), g);
