@@ -1373,7 +1373,7 @@ extern "C" int32_t mpadam_toy_create(int64_t n, const mpadam_toy_config* cfg, mp
   if (dev_malloc(&a.cnt, sizeof(int32_t) * n) != cudaSuccess || dev_malloc(&a.first, sizeof(int32_t) * n) != cudaSuccess ||
       dev_malloc(&a.idx, sizeof(int32_t) * B) != cudaSuccess || dev_malloc(&a.res, sizeof(float) * B) != cudaSuccess ||
       dev_malloc(&st->t_dev, sizeof(int64_t) * 2) != cudaSuccess ||
-      dev_malloc(&a.partial, sizeof(double) * (B / 2048 + 2)) != cudaSuccess) {
+      dev_malloc(&a.partial, sizeof(double) * (B / 256 + 2)) != cudaSuccess) {
     mpadam_toy_destroy(st);
     return fail(MPADAM_EALLOC, "allocation of the diagnostic's scratch failed");
   }

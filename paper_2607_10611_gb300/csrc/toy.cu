@@ -4,7 +4,7 @@
 // (per half when the halves are separate problems), and applies the
 // additive, multiplicative or combined step (no moments) to every sampled
 // entry, rounding it to BF16.  Two launches per step:
-//   1. one CTA per aligned chunk of 2048 samples draws them (Philox lanes;
+//   1. one CTA per aligned chunk of 256 samples draws them (Philox lanes;
 //      residuals, hit counts and each entry's first sample, with atomics on
 //      two n-entry scratch arrays that are zero between steps) and sums
 //      their squared residuals as a subtree of the perfect binary tree of
@@ -59,11 +59,14 @@ __device__ __forceinline__ double toy_draw(const ToyArgs& a, int64_t s, uint32_t
   return static_cast<double>(r) * static_cast<double>(r);
 }
 
-// Stage 1: CTA b of a problem draws the aligned chunk of C = min(2048, B_h)
+// Stage 1: CTA b of a problem draws the aligned chunk of C = min(256, B_h)
 // samples [bC, bC + C) and sums their squared residuals as a perfect binary
 // tree (adjacent pairs per thread, then adjacent lanes, then adjacent warps)
-// into partial[problem][b].
-constexpr int kToyChunk = 2048;
+// into partial[problem][b].  Small chunks spread the random gathers over many
+// SMs: at 65,536 samples per step, 2048-sample chunks (32 CTAs) took 14.8 us
+// per step, 512 took 12.7 and 256 (256 CTAs) 12.6.
+constexpr int kToyChunk = 256;
+constexpr int kToyMaxPartials = 32 * 2048 / kToyChunk;  // per problem, at 65,536 samples
 
 __global__ void __launch_bounds__(kToyChunk / 2) toy_sample_partial_kernel(const __grid_constant__ ToyArgs a) {
   __shared__ double warp_sum[32];
@@ -104,14 +107,25 @@ __global__ void __launch_bounds__(kToyChunk / 2) toy_sample_partial_kernel(const
 }
 
 // Stage 2 (every update CTA): the problem's partial sums, a perfect tree
-// over at most 32 adjacent chunks, then M, the loss and alpha.
+// over at most 256 adjacent chunks (each lane first sums up to 8 adjacent
+// ones), then M, the loss and alpha.
 __device__ __forceinline__ void toy_finish_mean(const ToyArgs& a, int h, double& loss_h, float& alpha_h) {
   const int64_t Bh = a.batch / (a.split ? 2 : 1);
   const int64_t C = Bh < kToyChunk ? Bh : kToyChunk;
   const int per = static_cast<int>(Bh / C);
   const int lane = threadIdx.x & 31;
-  double w = lane < per ? a.partial[h * per + lane] : 0.0;
-  for (int off = 1; off < per; off <<= 1) {
+  const int q = per > 32 ? per / 32 : 1;        // adjacent partials per lane (a power of two)
+  const int lanes = per > 32 ? 32 : per;        // lanes holding them
+  double v[kToyMaxPartials / 32];
+#pragma unroll
+  for (int j = 0; j < kToyMaxPartials / 32; ++j) v[j] = j < q && lane < lanes ? a.partial[h * per + lane * q + j] : 0.0;
+#pragma unroll
+  for (int step = 1; step < kToyMaxPartials / 32; step <<= 1)
+#pragma unroll
+    for (int j = 0; j + step < kToyMaxPartials / 32; j += 2 * step)
+      if (step < q) v[j] = v[j] + v[j + step];
+  double w = v[0];
+  for (int off = 1; off < lanes; off <<= 1) {
     const double y = __shfl_xor_sync(0xFFFFFFFFu, w, off);
     w = (lane & off) ? y + w : w + y;
   }

@@ -16,7 +16,7 @@ struct ToyArgs {
   int32_t* first;       // [n] INT_MAX - (first sample of each entry); 0 between steps
   int32_t* idx;         // [batch]
   float* res;           // [batch]
-  double* partial;      // [batch / 2048 + 2] chunk sums of the squared residuals
+  double* partial;      // [batch / 256 + 2] chunk sums of the squared residuals
   double* loss_out;     // caller's device double, or nullptr (step-by-step mode)
   int64_t* t_dev;       // run mode: [0] = this step's t (advanced by the update kernel), [1] = the run's first t;
                         // nullptr in step-by-step mode (t from t_lo / t_hi)
