@@ -1073,7 +1073,6 @@ __device__ __noinline__ void general_block_group_call(const StepArgs& a, const T
   general_block_group<GD, MD, SR, OPT>(a, x, tile_e0, count, c, st);
 }
 
-
 // ---------------------------------------------------------------------------
 // NVFP4 weights: E2M1 codes (OCP FP4: sign, 2 exponent bits with bias 1, one
 // mantissa bit; +-{0, 0.5, 1, 1.5, 2, 3, 4, 6}), an E4M3 scale s per 16
@@ -1591,7 +1590,8 @@ __global__ void __launch_bounds__(kThreads, 1) step_kernel(const __grid_constant
     // The producer sets up the ring and issues the copies of its first tile
     // before the block-wide barrier, in straight-line code next to the
     // kernel's entry: on a launch of a tile or two per CTA these copies are
-    // on the critical path, and the full loop below starts some 1.5 us later.
+    // on the critical path (issued 1.3 us after entry, against 2.0 us from
+    // the loop below after the barrier).
     for (int i = 0; i < S; ++i) {
       mbar_init(smem_addr(&full_bar[i]), 1);
       mbar_init(smem_addr(&empty_bar[i]), kConsumerWarps);
