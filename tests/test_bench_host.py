@@ -170,3 +170,16 @@ def test_result_line_keeps_every_secondary_list_in_the_driver_tail():
     assert "step_ms" not in line["e2e"] and len(main["e2e"]["step_ms"]) == 20
     flat = [bench.compact(s2) for s2 in secs if s2["workload"] == "flat_1m"][0]
     assert flat["one_tile_ms"] == 0.0082 and flat["frac_of_copy"] > 0
+
+
+def test_oracle_rate_on_a_whole_list():
+    """The oracle's single-core rate is taken over one step of the whole list
+    (the 1 Mi flat list here), not a sample of it."""
+    sys.path.insert(0, str(ROOT))
+    import bench
+    r = bench.oracle_whole_lists("flat_1m")
+    assert list(r) == ["flat_1m"]
+    e = r["flat_1m"]
+    assert e["whole_list"] and e["params"] == 1_048_576 and e["cores"] == 1
+    assert e["ns_per_param"] > 0 and e["ns_per_param"] == pytest.approx(1.0 / e["gparams_per_s"], rel=1e-3)
+    assert bench.oracle_whole_lists("") == {}
