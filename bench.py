@@ -298,10 +298,16 @@ def run_gpu(wl, steps: int, warmup: int, rank: int, e2e_steps: int, flush_l2: bo
     # end to end through the host-buffer entry point (one weight format: flat host buffers)
     if e2e_steps > 0 and "w" in mt.flat:
         # page-locked host buffers: huge-page ones from mpadam_host_buffer_alloc,
-        # or the driver's (torch pin_memory), whichever copies faster here
+        # unless they copy clearly slower here than the driver's (torch
+        # pin_memory).  A plain 1 GiB copy runs at the same rate on both, but
+        # the step's chunked pipeline on the driver's buffers had steps of
+        # 100-190 ms among its 87.6 ms ones (about one in five, on some boxes),
+        # and none on huge pages over 40 alternating steps in one process.
         from paper_2607_10611_gb300.optimizer import HostBuffer
         probe = pinned_probe_gbs(stream)
         kinds = sorted(probe, key=lambda k: -probe[k])
+        if "huge_pages" in probe and probe["huge_pages"] >= 0.95 * max(probe.values()):
+            kinds = ["huge_pages"] + [k for k in kinds if k != "huge_pages"]
         nbytes = sum(x.numel() for x in mt.g) * BYTES[wl.grad_dtype] + sum(x.numel() for x in mt.w) * BYTES[wl.weight_dtype]
         for attempt, kind in enumerate(kinds):
             if kind == "huge_pages":

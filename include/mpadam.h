@@ -269,7 +269,10 @@ int32_t mpadam_step_host(mpadam_state* s, const void* const* host_grads, void* c
  * registers it with the CUDA driver (cudaHostRegister).  Copies
  * from such a buffer keep the host link's full rate: on GB300 (Grace) hosts,
  * copies from ordinary pinned memory of 64 KB pages measured 4x slower at
- * times for buffers of several GB, huge-page buffers did not.  Release with
+ * times for buffers of several GB, huge-page buffers did not.  On the 7B list
+ * (13.5 GB each way), mpadam_step_host on ordinary pinned buffers had steps of
+ * up to 3.2x the usual 87.6 ms on some hosts, about one in four; on huge-page
+ * buffers, none in 40 steps alternating with them.  Release with
  * mpadam_host_buffer_free (same size).  Errors: EINVAL, EALLOC, ECUDA. */
 int32_t mpadam_host_buffer_alloc(int64_t bytes, void** out);
 int32_t mpadam_host_buffer_free(void* ptr, int64_t bytes);
